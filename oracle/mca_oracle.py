@@ -1,0 +1,414 @@
+"""Plain fp64 CPU oracle of the Monte Carlo mutation-selection (MCA) trial loop.
+
+TEST INFRASTRUCTURE ONLY -- imported by tests/, __graft_entry__.smoke() and bench.py's CPU legs;
+never by the product path, and sharing no code with it.
+
+What it computes (paper "Beyond Backpropagation: Monte Carlo Method Can Train Deep Neural
+Networks", Section 2 Eq. 1 and Section 3.1 Eq. 6):
+
+    for tau = 0, 1, ...:
+        pick one parameter uniformly at random and draw its new value   (Eq. 1, Section 2)
+        reject without evaluating if the new value leaves the domain |w| < Delta   (Eq. 1)
+        W' = W with that one parameter changed
+        S' = sum over all N samples of the per-sample loss of f_W'   (full batch, Eq. 2 with R = 0)
+        keep W' iff S' <= S, else keep W   (greedy rule, Eq. 6)
+
+Two evaluation modes, which must agree (the invariant the incremental GPU path relies on):
+
+* ``run_full``: a full forward pass of all N samples after every mutation -- the definition.
+* ``run_incremental``: the paper's cached-field scheme (Section 2.4): only the mutated neuron's
+  field row changes (rank-1 in the mutated layer l), the next layer's fields change by the
+  mutated neuron's activation change times one weight column (rank-1 in l+1), and the layers from
+  l+2 on are recomputed densely.
+
+Readings of points the paper leaves open (each listed in the design doc):
+
+* Proposal stream: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), key = (seed_lo, seed_hi),
+  counter = (tau_lo, tau_hi, 0, 0); words r0 (index) and r1 (value) are used.
+* Index: idx = floor(r0 * P / 2^32) over the flat parameter space (layers in forward order,
+  each weight matrix [out x in] row-major).
+* Replacement value: u = (r1 >> 8) * 2^-24 in fp32, w' = lo + (hi - lo) * u with two fp32
+  roundings (for [lo, hi) = [-1, 1) this is exact). Perturbation: r = 2u - 1 (exact),
+  w' = w + delta * r in fp32.
+* Ternary layers: new code floor(r1 * 3 / 2^32) - 1 (may equal the old code: a no-op trial).
+  Masked layers: the mutation toggles the mask bit of the chosen fixed weight.
+* MSE loss: sum over outputs of (a_k - onehot_k)^2; CE: natural-log softmax cross-entropy.
+  Decisions use the loss sum S; the reported loss is S / N.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+import numpy as np
+from scipy.special import erf as _erf
+
+__all__ = [
+    "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
+    "forward", "total_loss", "run_full", "run_incremental", "Trace",
+]
+
+# ------------------------------------------------------------------------------------------------
+# Philox4x32-10 (Salmon et al., "Parallel random numbers: as easy as 1, 2, 3", SC'11, Section 3.2):
+# a 10-round bijection of a 128-bit counter under a 64-bit key.
+# ------------------------------------------------------------------------------------------------
+_M32 = np.uint64(0xFFFFFFFF)
+_PH_M0 = np.uint64(0xD2511F53)
+_PH_M1 = np.uint64(0xCD9E8D57)
+_PH_W0 = np.uint64(0x9E3779B9)
+_PH_W1 = np.uint64(0xBB67AE85)
+_S32 = np.uint64(32)
+
+
+def philox4x32_10(ctr, key) -> np.ndarray:
+    """ctr: (..., 4) and key: (..., 2) arrays of 32-bit words. Returns (..., 4) uint64 words."""
+    c = np.asarray(ctr, dtype=np.uint64)
+    k = np.asarray(key, dtype=np.uint64)
+    c0, c1, c2, c3 = c[..., 0], c[..., 1], c[..., 2], c[..., 3]
+    k0, k1 = k[..., 0], k[..., 1]
+    for rnd in range(10):
+        if rnd:
+            k0 = (k0 + _PH_W0) & _M32
+            k1 = (k1 + _PH_W1) & _M32
+        p0 = c0 * _PH_M0          # both factors < 2^32: the product fits in 64 bits
+        p1 = c2 * _PH_M1
+        c0, c1, c2, c3 = ((p1 >> _S32) ^ c1 ^ k0, p1 & _M32, (p0 >> _S32) ^ c3 ^ k1, p0 & _M32)
+    return np.stack([c0, c1, c2, c3], axis=-1)
+
+
+def draw_words(seed: int, tau) -> np.ndarray:
+    """The four Philox words of trial tau (scalar or array) under proposal key ``seed``."""
+    tau = np.asarray(tau, dtype=np.uint64)
+    ctr = np.stack([tau & _M32, tau >> _S32, np.zeros_like(tau), np.zeros_like(tau)], axis=-1)
+    s = np.uint64(seed)
+    key = np.broadcast_to(np.array([s & _M32, s >> _S32], dtype=np.uint64), ctr.shape[:-1] + (2,))
+    return philox4x32_10(ctr, key)
+
+
+# ------------------------------------------------------------------------------------------------
+# Parameters
+# ------------------------------------------------------------------------------------------------
+
+class Params:
+    """Per-layer weight state. fp32 layers: the weights; ternary layers: int8 codes in {-1,0,1}
+    (effective weight scale * code); masked layers: fixed fp32 weights and a 0/1 mask (effective
+    weight w * m). ``init`` is the flat fp32 vector (codes for ternary layers); masks start at 1."""
+
+    def __init__(self, layers, init: np.ndarray):
+        self.layers = layers
+        self.vals: List[np.ndarray] = []
+        self.mask: List[Optional[np.ndarray]] = []
+        o = 0
+        init = np.asarray(init, dtype=np.float32)
+        for L in layers:
+            n = L.n_in * L.n_out
+            block = init[o:o + n].reshape(L.n_out, L.n_in)
+            if L.wkind == "ternary_i8":
+                self.vals.append(block.astype(np.int8).copy())
+                self.mask.append(None)
+            elif L.wkind == "masked_fp32":
+                self.vals.append(block.astype(np.float32).copy())
+                self.mask.append(np.ones((L.n_out, L.n_in), dtype=np.uint8))
+            else:
+                self.vals.append(block.astype(np.float32).copy())
+                self.mask.append(None)
+            o += n
+        self.n_params = o
+        self.offsets = np.cumsum([0] + [L.n_in * L.n_out for L in layers])[:-1].tolist()
+
+    def copy(self) -> "Params":
+        p = Params.__new__(Params)
+        p.layers = self.layers
+        p.vals = [v.copy() for v in self.vals]
+        p.mask = [None if m is None else m.copy() for m in self.mask]
+        p.n_params = self.n_params
+        p.offsets = list(self.offsets)
+        return p
+
+    def eff32(self, l: int) -> np.ndarray:
+        L = self.layers[l]
+        if L.wkind == "ternary_i8":
+            return np.float32(L.scale) * self.vals[l].astype(np.float32)
+        if L.wkind == "masked_fp32":
+            return np.where(self.mask[l] != 0, self.vals[l], np.float32(0.0)).astype(np.float32)
+        return self.vals[l]
+
+    def eff64(self, l: int) -> np.ndarray:
+        return self.eff32(l).astype(np.float64)
+
+    def flat_eff32(self) -> np.ndarray:
+        return np.concatenate([self.eff32(l).ravel() for l in range(len(self.layers))])
+
+    def flat_codes(self) -> np.ndarray:
+        """int8 per parameter: ternary code, mask bit, or 0 for fp32 layers."""
+        out = []
+        for l, L in enumerate(self.layers):
+            if L.wkind == "ternary_i8":
+                out.append(self.vals[l].ravel().astype(np.int8))
+            elif L.wkind == "masked_fp32":
+                out.append(self.mask[l].ravel().astype(np.int8))
+            else:
+                out.append(np.zeros(L.n_in * L.n_out, dtype=np.int8))
+        return np.concatenate(out)
+
+
+# ------------------------------------------------------------------------------------------------
+# Proposal (Eq. 1): one parameter, one new value
+# ------------------------------------------------------------------------------------------------
+
+@dataclass
+class Proposal:
+    tau: int
+    idx: int
+    layer: int
+    row: int            # output neuron j of the layer
+    col: int            # input neuron i of the layer
+    old: float          # effective weights (exact fp32 values, held as Python floats)
+    new: float
+    old_code: int       # ternary code / mask bit (0 for fp32 layers)
+    new_code: int
+    new_raw: float      # the value stored in the fp32 slot (fp32 layers: == new)
+    valid: bool         # False: outside the weight domain, rejected without evaluation
+
+
+def propose(seed: int, tau: int, params: Params, domain) -> Proposal:
+    r = draw_words(seed, tau)
+    r0, r1 = int(r[0]), int(r[1])
+    P = params.n_params
+    idx = (r0 * P) >> 32
+    l = 0
+    while l + 1 < len(params.layers) and idx >= params.offsets[l + 1]:
+        l += 1
+    L = params.layers[l]
+    off = idx - params.offsets[l]
+    row, col = divmod(off, L.n_in)
+    f32 = np.float32
+    if L.wkind == "ternary_i8":
+        oc = int(params.vals[l][row, col])
+        nc = ((r1 * 3) >> 32) - 1
+        old = float(f32(L.scale) * f32(oc))
+        new = float(f32(L.scale) * f32(nc))
+        return Proposal(tau, idx, l, row, col, old, new, oc, nc, new, True)
+    if L.wkind == "masked_fp32":
+        w = f32(params.vals[l][row, col])
+        om = int(params.mask[l][row, col])
+        nm = 1 - om
+        old = float(w) if om else 0.0
+        new = float(w) if nm else 0.0
+        return Proposal(tau, idx, l, row, col, old, new, om, nm, float(w), True)
+    oldv = f32(params.vals[l][row, col])
+    u = f32(r1 >> 8) * f32(2.0 ** -24)                       # exact, in [0, 1)
+    if domain.op == "replace":
+        newv = f32(f32(domain.lo) + f32(f32(f32(domain.hi) - f32(domain.lo)) * u))
+    elif domain.op == "perturb":
+        rr = f32(f32(2.0) * u) - f32(1.0)                      # exact, in [-1, 1)
+        newv = f32(oldv + f32(f32(domain.delta) * rr))
+    else:
+        raise ValueError(domain.op)
+    valid = True
+    if domain.bound > 0 and not (abs(newv) < f32(domain.bound)):
+        valid = False
+    return Proposal(tau, idx, l, row, col, float(oldv), float(newv), 0, 0, float(newv), valid)
+
+
+def apply_proposal(params: Params, p: Proposal) -> None:
+    L = params.layers[p.layer]
+    if L.wkind == "ternary_i8":
+        params.vals[p.layer][p.row, p.col] = p.new_code
+    elif L.wkind == "masked_fp32":
+        params.mask[p.layer][p.row, p.col] = p.new_code
+    else:
+        params.vals[p.layer][p.row, p.col] = np.float32(p.new_raw)
+
+
+def revert_proposal(params: Params, p: Proposal) -> None:
+    L = params.layers[p.layer]
+    if L.wkind == "ternary_i8":
+        params.vals[p.layer][p.row, p.col] = p.old_code
+    elif L.wkind == "masked_fp32":
+        params.mask[p.layer][p.row, p.col] = p.old_code
+    else:
+        params.vals[p.layer][p.row, p.col] = np.float32(p.old)
+
+
+# ------------------------------------------------------------------------------------------------
+# Forward pass and loss (Section 2: transfer functions; Eq. 2 with R = 0)
+# ------------------------------------------------------------------------------------------------
+
+def act_fn(name: str, z: np.ndarray, gamma: float = 0.0) -> np.ndarray:
+    if name == "identity":
+        return z
+    if name == "tanh":
+        return np.tanh(z)
+    if name == "sigmoid":
+        with np.errstate(over="ignore"):
+            return 1.0 / (1.0 + np.exp(-z))
+    if name == "relu":
+        return np.maximum(z, 0.0)
+    if name == "gaussian":                     # f(x) = exp(-gamma x^2), Section 2
+        return np.exp(-gamma * z * z)
+    if name == "gelu":                         # exact-erf GELU
+        return 0.5 * z * (1.0 + _erf(z / np.sqrt(2.0)))
+    raise ValueError(name)
+
+
+def loss_per_sample(kind: str, out: np.ndarray, y: np.ndarray) -> np.ndarray:
+    """out: [C, N] output activations; y: [N] labels. Returns [N] per-sample losses."""
+    n = out.shape[1]
+    if kind == "mse_onehot":
+        t = np.zeros_like(out)
+        t[y, np.arange(n)] = 1.0
+        return ((out - t) ** 2).sum(axis=0)
+    if kind == "softmax_ce":
+        m = out.max(axis=0)
+        lse = m + np.log(np.exp(out - m).sum(axis=0))
+        return lse - out[y, np.arange(n)]
+    raise ValueError(kind)
+
+
+def forward(params: Params, XT: np.ndarray):
+    """XT: [D, N] float64. Returns (Z list of [n_out, N] fields, final activations [C, N])."""
+    a = XT
+    Zs = []
+    for l, L in enumerate(params.layers):
+        z = params.eff64(l) @ a
+        Zs.append(z)
+        a = act_fn(L.act, z, L.act_param)
+    return Zs, a
+
+
+def total_loss(params: Params, XT: np.ndarray, y: np.ndarray, loss: str) -> float:
+    _, out = forward(params, XT)
+    return float(loss_per_sample(loss, out, y).sum())
+
+
+# ------------------------------------------------------------------------------------------------
+# Trial loops
+# ------------------------------------------------------------------------------------------------
+
+class Trace:
+    """Per-trial record: tau, idx, layer, row, col, old, new (effective fp32 weights), valid,
+    S_before, dS (S' - S; NaN when not evaluated), accept."""
+    FIELDS = ("tau", "idx", "layer", "row", "col", "old", "new", "new_code", "valid", "S", "dS",
+              "accept")
+
+    def __init__(self):
+        self.rows = []
+
+    def add(self, p: Proposal, S: float, dS: float, accept: bool):
+        self.rows.append((p.tau, p.idx, p.layer, p.row, p.col, p.old, p.new, p.new_code, p.valid,
+                          S, dS, accept))
+
+    def arrays(self):
+        cols = list(zip(*self.rows)) if self.rows else [[] for _ in self.FIELDS]
+        dt = {"tau": np.int64, "idx": np.int64, "layer": np.int32, "row": np.int32,
+              "col": np.int32, "old": np.float64, "new": np.float64, "new_code": np.int32,
+              "valid": bool, "S": np.float64, "dS": np.float64, "accept": bool}
+        return {f: np.asarray(c, dtype=dt[f]) for f, c in zip(self.FIELDS, cols)}
+
+
+def _decide(dS: float, strict: bool) -> bool:
+    return (dS < 0.0) if strict else (dS <= 0.0)
+
+
+def run_full(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials: int, seed: int,
+             domain, tau0: int = 0, params: Optional[Params] = None):
+    """The definition: a full forward pass of all samples after every mutation.
+    Returns (trace arrays, final Params, final S)."""
+    XT = np.ascontiguousarray(np.asarray(X, dtype=np.float64).T)
+    y = np.asarray(y)
+    params = Params(layers, init) if params is None else params
+    S = total_loss(params, XT, y, loss)
+    tr = Trace()
+    for t in range(n_trials):
+        p = propose(seed, tau0 + t, params, domain)
+        if not p.valid:
+            tr.add(p, S, float("nan"), False)
+            continue
+        apply_proposal(params, p)
+        S_new = total_loss(params, XT, y, loss)
+        dS = S_new - S
+        acc = S_new < S if domain.strict else S_new <= S
+        tr.add(p, S, dS, acc)
+        if acc:
+            S = S_new
+        else:
+            revert_proposal(params, p)
+    return tr.arrays(), params, S
+
+
+class _Cache:
+    """Cached fields of every layer for all samples, plus the per-sample losses."""
+
+    def __init__(self, params: Params, XT: np.ndarray, y: np.ndarray, loss: str):
+        self.Z, out = forward(params, XT)
+        self.ell = loss_per_sample(loss, out, y)
+
+
+def _candidate(params: Params, cache: _Cache, XT, y, loss, p: Proposal):
+    """Incremental evaluation of one proposal against the cached state (Section 2.4).
+    Returns (dS, list of (layer, new field matrix or (row, new row)) to commit, new ell)."""
+    layers = params.layers
+    l, j, i = p.layer, p.row, p.col
+    nl = len(layers)
+    delta = p.new - p.old                                   # exact in fp64 (fp32 operands)
+    if l == 0:
+        a_prev_i = XT[i]
+    else:
+        Lp = layers[l - 1]
+        a_prev_i = act_fn(Lp.act, cache.Z[l - 1][i], Lp.act_param)
+    zrow = cache.Z[l][j] + delta * a_prev_i                 # rank-1 update of layer l, row j
+    updates = [(l, ("row", j, zrow))]
+    if l == nl - 1:
+        Zout = cache.Z[l].copy()
+        Zout[j] = zrow
+        out = act_fn(layers[l].act, Zout, layers[l].act_param)
+    else:
+        L = layers[l]
+        da = act_fn(L.act, zrow, L.act_param) - act_fn(L.act, cache.Z[l][j], L.act_param)
+        Wn = params.eff64(l + 1)
+        z = cache.Z[l + 1] + np.outer(Wn[:, j], da)         # rank-1 update of layer l+1
+        updates.append((l + 1, ("full", z)))
+        a = act_fn(layers[l + 1].act, z, layers[l + 1].act_param)
+        for m in range(l + 2, nl):                          # dense recompute from l+2 on
+            z = params.eff64(m) @ a
+            updates.append((m, ("full", z)))
+            a = act_fn(layers[m].act, z, layers[m].act_param)
+        out = a
+    ell_new = loss_per_sample(loss, out, y)
+    dS = float((ell_new - cache.ell).sum())
+    return dS, updates, ell_new
+
+
+def run_incremental(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials: int,
+                    seed: int, domain, tau0: int = 0, params: Optional[Params] = None,
+                    check_every: int = 0):
+    """The paper's cached-field scheme. ``check_every`` > 0 asserts, every that many trials, that
+    the cached S equals a full recompute within 1e-9 relative. Returns (trace, Params, S)."""
+    XT = np.ascontiguousarray(np.asarray(X, dtype=np.float64).T)
+    y = np.asarray(y)
+    params = Params(layers, init) if params is None else params
+    cache = _Cache(params, XT, y, loss)
+    S = float(cache.ell.sum())
+    tr = Trace()
+    for t in range(n_trials):
+        p = propose(seed, tau0 + t, params, domain)
+        if not p.valid:
+            tr.add(p, S, float("nan"), False)
+            continue
+        dS, updates, ell_new = _candidate(params, cache, XT, y, loss, p)
+        acc = _decide(dS, domain.strict)
+        tr.add(p, S, dS, acc)
+        if acc:
+            apply_proposal(params, p)
+            for m, upd in updates:
+                if upd[0] == "row":
+                    cache.Z[m][upd[1]] = upd[2]
+                else:
+                    cache.Z[m] = upd[1]
+            cache.ell = ell_new
+            S = S + dS
+        if check_every and (t + 1) % check_every == 0:
+            S_full = total_loss(params, XT, y, loss)
+            assert abs(S_full - S) <= 1e-9 * max(1.0, abs(S_full)), (t, S_full, S)
+    return tr.arrays(), params, S
