@@ -1,0 +1,345 @@
+"""Throughput of the MCA trial loop on one GB300 (trials/s), per the bench contract.
+
+Workload (default): the 784-16384-10 tanh / softmax-CE net on N = 60000 synthetic MNIST-shaped
+samples, K = 64 speculative candidates per batch, 1M-trial job, Philox seed 0. One step = one
+mca_run call of T trials continuing the same trajectory; warm-up + timed steps together cover the
+job's 1M trials (T = ceil(1e6 / (warmup + steps))). The cached hidden fields (3.9 GB) are far
+larger than L2, so no L2 flush is needed between steps.
+
+--impl reference times the CPU oracle (incremental mode, fp64 numpy) on the same workload, a
+bounded number of trials per step, on the host cores.
+
+Multi-GPU: the trial loop is sequential (each trial depends on the previous decision), so N GPUs run
+N independent replicas (proposal seed = rank); value = all ranks' trials / max time ("weak").
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roofline"
+UNIT = "trials/s"
+JOB_TRIALS = 1_000_000
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms while running."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def make_workload(args, rank):
+    from paper_2607_08406_gb300 import workloads as W
+    kw = {}
+    if args.N:
+        kw["N"] = args.N
+    if args.H:
+        kw["H"] = args.H
+    wl = W.make(args.workload, **kw)
+    wl.seed = args.seed + rank
+    if args.K:
+        wl.K = args.K
+    return wl
+
+
+def cpu_oracle_rate(wl, n_trials, warm=0):
+    """Trials/s of the oracle's incremental mode after its untimed cache build (forward pass)."""
+    from oracle import mca_oracle as O
+    XT = np.ascontiguousarray(wl.X.astype(np.float64).T)
+    params = O.Params(wl.layers, wl.init)
+    cache = O._Cache(params, XT, wl.y, wl.loss)
+    S = float(cache.ell.sum())
+
+    def trials(t0, n):
+        nonlocal S
+        for t in range(t0, t0 + n):
+            p = O.propose(wl.seed, t, params, wl.domain)
+            if not p.valid:
+                continue
+            dS, updates, ell_new = O._candidate(params, cache, XT, wl.y, wl.loss, p)
+            if dS <= 0.0:
+                O.apply_proposal(params, p)
+                for m, upd in updates:
+                    if upd[0] == "row":
+                        cache.Z[m][upd[1]] = upd[2]
+                    else:
+                        cache.Z[m] = upd[1]
+                cache.ell = ell_new
+                S += dS
+    return trials
+
+
+def run_reference(args):
+    rank, local_rank, world = dist_env()
+    if rank != 0:
+        return 0
+    wl = make_workload(args, 0)
+    per_step = args.ref_trials
+    trials = cpu_oracle_rate(wl, per_step)
+    tau = 0
+    for _ in range(args.warmup):
+        trials(tau, per_step)
+        tau += per_step
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        trials(tau, per_step)
+        tau += per_step
+    dt = time.perf_counter() - t0
+    rate = per_step * args.steps / dt
+    cores = len(os.sched_getaffinity(0))
+    sample = (f"oracle incremental mode (fp64 numpy), trials {per_step * args.warmup}.."
+              f"{tau} of {wl.name}, after an untimed forward pass")
+    line = {"impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": wl.name, "K": wl.K, "trials_per_step": per_step},
+            "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    from paper_2607_08406_gb300 import mca
+    from paper_2607_08406_gb300.build import build
+    build()
+    wl = make_workload(args, rank)
+    K, W_ = args.steps, args.warmup
+    T = args.trials_per_step or math.ceil(JOB_TRIALS / (K + W_))
+    stream = torch.cuda.current_stream()
+
+    Xd = torch.from_numpy(wl.X).cuda()
+    yd = torch.from_numpy(wl.y).cuda()
+    initd = torch.from_numpy(wl.init).cuda()
+    h = mca.mca_create(wl.layers, wl.loss, wl.domain, Xd, yd, initd, K=wl.K,
+                       resync_period=args.resync, stream=stream.cuda_stream)
+    # one full forward pass (the resync step), timed on its own
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    mca.mca_resync(h)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    resync_ms = ev0.elapsed_time(ev1)
+
+    for _ in range(W_):
+        mca.mca_run(h, T, wl.seed)
+    st0 = mca.mca_get_stats(h)
+    barrier()
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    with ClockSampler(local_rank) as clk:
+        evs[0].record(stream)
+        for k in range(K):
+            mca.mca_run(h, T, wl.seed)
+            evs[k + 1].record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    st1 = mca.mca_get_stats(h)
+    step_ms = [evs[k].elapsed_time(evs[k + 1]) for k in range(K)]
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    trials_timed = (st1["trials"] - st0["trials"]) * world
+    value = trials_timed / (total_ms / 1e3)
+    launches = st1["launches"] - st0["launches"]
+    # dominant kernel: the trial loop (one launch per step when no resync falls in the step)
+    peak, peak_kind = load_peaks()
+    bytes_timed = st1["alg_bytes"] - st0["alg_bytes"]
+    loop_launches = K
+    achieved = bytes_timed / loop_launches / (total_ms / K / 1e3) / 1e9
+    loss_end = mca.mca_loss(h)
+    h.close()
+
+    # end to end through the public API from pinned host memory: one step = the whole job
+    # (create from host arrays -> JOB_TRIALS trials -> parameters back to host)
+    e2e = None
+    if not args.no_e2e:
+        Xh = torch.from_numpy(wl.X).pin_memory()
+        yh = torch.from_numpy(wl.y).pin_memory()
+        ih = torch.from_numpy(wl.init).pin_memory()
+        out = torch.empty(wl.n_params, dtype=torch.float32).pin_memory()
+        e2e_trials = args.e2e_trials or JOB_TRIALS
+
+        def job():
+            hh = mca.mca_create(wl.layers, wl.loss, wl.domain, Xh, yh, ih, K=wl.K,
+                                resync_period=args.resync, stream=stream.cuda_stream)
+            mca.mca_run(hh, e2e_trials, wl.seed)
+            mca.mca_get_params(hh, wl.n_params, out)
+            lv = mca.mca_loss(hh)
+            hh.close()
+            return lv
+        job()
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            job()
+        torch.cuda.synchronize()
+        dt = time.perf_counter() - t0
+        if world > 1:
+            t = torch.tensor([dt], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            dt = float(t.item())
+        e2e = {"value": e2e_trials * args.e2e_steps * world / dt, "unit": UNIT,
+               "h2d_bytes_per_step": int(wl.X.nbytes + wl.y.nbytes + wl.init.nbytes),
+               "d2h_bytes_per_step": int(out.numel() * 4 + 8),
+               "step": f"create from pinned host arrays + {e2e_trials} trials + params to host"}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu:
+        trials = cpu_oracle_rate(wl, args.cpu_trials)
+        t0 = time.perf_counter()
+        trials(0, args.cpu_trials)
+        dt = time.perf_counter() - t0
+        cpu = {"value": args.cpu_trials / dt, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
+               "kind": "oracle",
+               "sample": f"first {args.cpu_trials} trials of {wl.name}, oracle incremental mode "
+                         f"(fp64 numpy), after an untimed forward pass"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": W_, "ms_per_step": total_ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": wl.name, "N": wl.N, "hidden": wl.layers[0].n_out,
+                       "K": wl.K, "trials_per_step": T,
+                       "trial_range": [W_ * T, (W_ + K) * T], "seed": args.seed,
+                       "resync_period": args.resync, "resync_ms": resync_ms,
+                       "l2": "no flush: cached hidden fields (3.9 GB) exceed L2",
+                       "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+                       "accepts_timed": st1["accepts"] - st0["accepts"],
+                       "candidates_timed": st1["candidates"] - st0["candidates"],
+                       "loss_end": loss_end},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "mlp2_trial_loop", "peak_kind": peak_kind,
+                         "bytes": "compulsory DRAM bytes counted by the kernel per candidate"},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "clocks": clk.summary(),
+            "gpu_launches": launches,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="mlp_wide")
+    ap.add_argument("--N", type=int, default=0)
+    ap.add_argument("--H", type=int, default=0)
+    ap.add_argument("--K", type=int, default=0)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--trials-per-step", dest="trials_per_step", type=int, default=0)
+    ap.add_argument("--resync", type=int, default=0)
+    ap.add_argument("--cpu-trials", dest="cpu_trials", type=int, default=2000)
+    ap.add_argument("--ref-trials", dest="ref_trials", type=int, default=200)
+    ap.add_argument("--e2e-steps", dest="e2e_steps", type=int, default=1)
+    ap.add_argument("--e2e-trials", dest="e2e_trials", type=int, default=0)
+    ap.add_argument("--no-e2e", dest="no_e2e", action="store_true")
+    ap.add_argument("--no-cpu", dest="no_cpu", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

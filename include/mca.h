@@ -1,0 +1,215 @@
+/*
+ * mca.h -- C ABI of the GB300 (sm_103a) Monte Carlo mutation-selection (MCA) trial loop.
+ *
+ * The method (paper "Beyond Backpropagation: Monte Carlo Method Can Train Deep Neural Networks"):
+ * pick one parameter at random, give it a new random value (Section 2, Eq. 1), re-evaluate the
+ * full-batch training loss (Eq. 2 with R = 0) and keep the change iff the loss does not rise
+ * (greedy rule, Section 3.1 Eq. 6); otherwise restore the old value and try again. The loss is
+ * re-evaluated from cached per-layer local fields (Section 2.4): a mutation of weight (j, i) of
+ * layer l changes only row j of that layer's fields (a rank-1 update over all samples) and, through
+ * neuron j's activation change, the next layer's fields by one weight column.
+ *
+ * Conventions shared by every call:
+ *  - Every call returns an mca_status; no C++ exception crosses this boundary. A failed call
+ *    leaves a message readable with mca_last_error().
+ *  - Pointers documented "host or device" may point to either (the library asks the CUDA driver
+ *    which); all others are host pointers.
+ *  - All GPU work of a handle is queued on the stream given at creation (mca_options.stream; NULL
+ *    = the legacy default stream). A handle is not thread-safe.
+ *  - Flat parameter order: layers in forward order; inside a layer the weight matrix
+ *    [n_out x n_in] row-major (weight (j, i) at offset j * n_in + i). There are no biases.
+ *  - Sizes: N < 2^31 samples, total parameter count P < 2^32.
+ */
+#ifndef MCA_H
+#define MCA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MCA_OK = 0,
+  MCA_ERR_INVALID = 1,     /* bad argument, size or spec */
+  MCA_ERR_CUDA = 2,        /* a CUDA call failed; the handle must be destroyed */
+  MCA_ERR_OOM = 3,         /* device memory exhausted, or the caller's workspace is too small */
+  MCA_ERR_TIMEOUT = 4,     /* a bounded device-side wait ran out; the handle must be destroyed */
+  MCA_ERR_NUMERIC = 5,     /* NaN or Inf in the data, the parameters or the loss */
+  MCA_ERR_UNSUPPORTED = 6  /* a valid spec this build does not implement */
+} mca_status;
+
+/* Transfer functions (Section 2: ReLU and the Gaussian exp(-gamma x^2); tanh, sigmoid and the
+ * exact-erf GELU of the Transformer section). */
+typedef enum {
+  MCA_ACT_IDENTITY = 0,
+  MCA_ACT_TANH = 1,
+  MCA_ACT_SIGMOID = 2,
+  MCA_ACT_RELU = 3,
+  MCA_ACT_GAUSSIAN = 4,    /* exp(-act_param * x^2) */
+  MCA_ACT_GELU = 5
+} mca_act;
+
+/* Per-sample loss on the last layer's activations a (Section 2; Eq. 2 with R = 0):
+ *   MSE_ONEHOT:  sum_k (a_k - [k == y])^2
+ *   SOFTMAX_CE:  log(sum_k exp(a_k)) - a_y   (natural log)
+ * Decisions use the loss sum S over all samples; mca_loss() reports S / N. */
+typedef enum { MCA_LOSS_MSE_ONEHOT = 0, MCA_LOSS_SOFTMAX_CE = 1 } mca_loss_kind;
+
+/* Weight storage of a layer (Section 2: discrete weights and pruning; Section 3.4 Eq. 12).
+ *   FP32:        the weight is an fp32 value; mutations draw a new value (mca_domain.op).
+ *   TERNARY_I8:  an int8 code t in {-1, 0, +1}; the effective weight is scale * t. A mutation
+ *                sets a uniformly drawn code (which may equal the old one: a no-op trial).
+ *   MASKED_FP32: a fixed fp32 weight w and a mask bit m (initially 1); the effective weight is
+ *                m ? w : 0. A mutation toggles m (pruning, and regrowth of a pruned weight). */
+typedef enum { MCA_W_FP32 = 0, MCA_W_TERNARY_I8 = 1, MCA_W_MASKED_FP32 = 2 } mca_wkind;
+
+/* Mutation operator of FP32 layers (Section 2, Eq. 1).
+ *   REPLACE: w' = lo + (hi - lo) * u,  u = (r1 >> 8) * 2^-24 (two fp32 roundings; exact for
+ *            [lo, hi) = [-1, 1)).
+ *   PERTURB: w' = w + delta * (2u - 1) in fp32 (Eq. 1's w + delta * rand). */
+typedef enum { MCA_OP_REPLACE = 0, MCA_OP_PERTURB = 1 } mca_op;
+
+typedef struct {
+  int32_t n_in, n_out;     /* fan-in and fan-out */
+  int32_t act;             /* mca_act applied to this layer's fields */
+  float act_param;         /* gamma of MCA_ACT_GAUSSIAN; ignored otherwise */
+  int32_t wkind;           /* mca_wkind */
+  float scale;             /* TERNARY_I8: effective weight = scale * code; ignored otherwise */
+} mca_layer;
+
+/* Weight domain and acceptance rule (Eq. 1, Eq. 6). */
+typedef struct {
+  int32_t op;              /* mca_op */
+  float lo, hi;            /* REPLACE range [lo, hi) */
+  float delta;             /* PERTURB amplitude */
+  float bound;             /* > 0: a proposal with !(|w'| < bound) is rejected unevaluated */
+  int32_t strict;          /* 0: accept iff dS <= 0 (Eq. 1, Eq. 6); 1: accept iff dS < 0 */
+} mca_domain;
+
+/* Training set. x: [n x d] fp32, sample-major (sample n's features at x + n * d); y: [n] int32
+ * labels in [0, n_classes). Host or device; copied at creation, not retained. */
+typedef struct {
+  const float* x;
+  const int32_t* y;
+  int64_t n;
+  int32_t d;
+} mca_dataset;
+
+typedef struct {
+  int32_t K;               /* speculative candidates per batch, 1..128 (the trajectory does not
+                              depend on K: the lowest-index improving candidate is accepted) */
+  int32_t resync_period;   /* > 0: recompute every cached field from scratch each time tau
+                              crosses a multiple of this; 0: only at creation and set_params */
+  void* stream;            /* cudaStream_t; NULL = legacy default stream */
+  int32_t trace_cap;       /* > 0: keep the last trace_cap trial records (mca_get_trace) */
+  int32_t grid;            /* > 0: CTAs of the trial-loop kernel (capped at what is co-resident);
+                              0: automatic */
+  void* workspace;         /* NULL: the library allocates its device memory itself; otherwise a
+                              caller-owned device buffer of >= mca_workspace_size() bytes,
+                              256-byte aligned, that must outlive the handle */
+  size_t workspace_bytes;
+} mca_options;
+
+typedef struct {
+  uint64_t trials;         /* trials consumed (sequential trials; discarded speculation excluded) */
+  uint64_t accepts;
+  uint64_t candidates;     /* candidates evaluated on the GPU */
+  uint64_t batches;
+  uint64_t wasted;         /* candidates evaluated after the accepted one in their batch */
+  uint64_t forced;         /* decisions taken from mca_force_decisions */
+  uint64_t resyncs;
+  uint64_t launches;       /* kernels this handle launched */
+  uint64_t tau;            /* next trial counter */
+  double S;                /* current loss sum */
+  uint64_t alg_bytes;      /* compulsory DRAM bytes of the evaluated candidates and commits: per
+                              first-layer candidate 32 B per hidden-field sector its input
+                              feature's non-zeros touch + 8 B per non-zero; per output-layer
+                              candidate 4 B per sample (one hidden-field row); per accepted
+                              first-layer candidate the sectors written back */
+} mca_run_stats;
+
+typedef struct {
+  uint64_t tau;            /* trial counter */
+  uint32_t idx;            /* flat parameter index */
+  int32_t accept;          /* 1 accepted, 0 rejected */
+  float old_w, new_w;      /* effective weights before / after the proposal */
+  int32_t valid;           /* 0: outside the weight domain, rejected unevaluated */
+  int32_t forced;          /* 1: decision taken from mca_force_decisions */
+  double dS;               /* S' - S of the candidate (NaN when not evaluated) */
+  double S;                /* loss sum before the trial */
+} mca_trace_rec;
+
+typedef struct mca_handle mca_handle;
+
+/* Bytes of device workspace mca_create needs for this spec and dataset (counts the non-zeros of
+ * the dataset, so data must be valid). Same argument rules as mca_create. */
+mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t loss,
+                              const mca_dataset* data, const mca_options* opt, size_t* bytes);
+
+/* Build a trial loop for the MLP `layers` (Section 2, Fig. 1a) on `data`.
+ *  init_params: [P] fp32, host or device, flat order; FP32 and MASKED layers hold the weight,
+ *               TERNARY layers hold the code (-1, 0 or 1) as a float.
+ *  Requirements: n_layers >= 2, layers[0].n_in == data->d, layers[l].n_out == layers[l+1].n_in,
+ *  the last layer's n_out <= 16 (the number of classes), labels in range.
+ *  Computes every cached field with a full forward pass (the trial counter tau starts at 0).
+ *  On success *out owns a handle to release with mca_destroy. Errors: INVALID (spec/sizes),
+ *  NUMERIC (non-finite x or init, or a non-finite initial loss), OOM, CUDA, UNSUPPORTED. */
+mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
+                      const mca_domain* dom, const mca_dataset* data, const float* init_params,
+                      const mca_options* opt, mca_handle** out);
+
+/* Run n_trials sequential trials tau, tau+1, ... (Eq. 1 proposals drawn from Philox4x32-10 with
+ * key = seed and counter = tau; Eq. 6 selection). Returns when they are done. stats: nullable.
+ * Errors: TIMEOUT (a device-side wait ran out), NUMERIC (the loss became non-finite), CUDA. */
+mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stats* stats);
+
+/* Current mean loss L = S / N (Eq. 2 with R = 0) from the cached fields. */
+mca_status mca_loss(mca_handle* h, double* L);
+
+/* Effective weights (fp32, flat order) into dst[0 .. n) (host or device); n must equal P. */
+mca_status mca_get_params(mca_handle* h, float* dst, size_t n);
+
+/* Per-parameter int8 codes into dst[0 .. n): ternary code, mask bit, or 0 for FP32 layers. */
+mca_status mca_get_codes(mca_handle* h, int8_t* dst, size_t n);
+
+/* Resume: load parameters in mca_create's init format (ternary codes; for MASKED layers the
+ * mask is taken from `codes`, nullable = all ones), set the trial counter to tau and recompute
+ * every cached field. Host or device pointers. */
+mca_status mca_set_params(mca_handle* h, const float* params, const int8_t* codes, size_t n,
+                          uint64_t tau);
+
+/* Recompute every cached field and S from the parameters with a full forward pass. */
+mca_status mca_resync(mca_handle* h);
+
+/* Copy up to cap of the most recent trial records, oldest first, into dst (host); *n gets the
+ * count. Requires trace_cap > 0 at creation. */
+mca_status mca_get_trace(mca_handle* h, mca_trace_rec* dst, size_t cap, size_t* n);
+
+/* Test hook: decide trial tau[m] by accept[m] instead of by its loss change (tau strictly
+ * increasing, host arrays). Used to replay a reference trajectory through trials whose loss change
+ * is within rounding of zero. n = 0 clears the list. */
+mca_status mca_force_decisions(mca_handle* h, const uint64_t* tau, const uint8_t* accept,
+                               size_t n);
+
+/* Statistics accumulated over the handle's lifetime. */
+mca_status mca_get_stats(mca_handle* h, mca_run_stats* stats);
+
+/* Loss changes dS of n hypothetical single-weight changes, all against the current state, with
+ * no commit: weight flat_idx[m] set to the effective value new_w[m] (host arrays, n <= 128).
+ * Same kernels as mca_run's evaluation step. dS: [n] doubles (host). */
+mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
+                               size_t n, double* dS);
+
+void mca_destroy(mca_handle* h);
+
+/* Message of the last failed call on h (h may be NULL: then the last failed mca_create or
+ * mca_workspace_size of this thread). Never NULL. */
+const char* mca_last_error(mca_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MCA_H */

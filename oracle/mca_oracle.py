@@ -45,7 +45,8 @@ from scipy.special import erf as _erf
 
 __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
-    "forward", "total_loss", "run_full", "run_incremental", "Trace",
+    "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
+    "candidate_dS_two_layer",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -412,3 +413,45 @@ def run_incremental(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_tri
             S_full = total_loss(params, XT, y, loss)
             assert abs(S_full - S) <= 1e-9 * max(1.0, abs(S_full)), (t, S_full, S)
     return tr.arrays(), params, S
+
+
+# ------------------------------------------------------------------------------------------------
+# Single-candidate evaluation at large sizes (two-layer nets): the hidden layer is formed in row
+# blocks so that only the output fields are held for all samples.
+# ------------------------------------------------------------------------------------------------
+
+def output_fields_blocked(params: Params, XT: np.ndarray, block: int = 1024) -> np.ndarray:
+    """Output fields Z2 = W2 f(W1 X^T) of a two-layer net, [C, N], built over hidden-row blocks."""
+    L1 = params.layers[0]
+    W1 = params.eff64(0)
+    W2 = params.eff64(1)
+    Z2 = np.zeros((W2.shape[0], XT.shape[1]))
+    for j0 in range(0, W1.shape[0], block):
+        A = act_fn(L1.act, W1[j0:j0 + block] @ XT, L1.act_param)
+        Z2 += W2[:, j0:j0 + block] @ A
+    return Z2
+
+
+def candidate_dS_two_layer(params: Params, XT: np.ndarray, y: np.ndarray, loss: str,
+                           Z2: np.ndarray, idx: int, new_eff: float) -> float:
+    """S' - S when the flat weight idx takes the effective value new_eff (Section 2.4's update:
+    one hidden field row, then the output fields through one weight column)."""
+    L1, L2 = params.layers
+    W1 = params.eff64(0)
+    W2 = params.eff64(1)
+    P1 = L1.n_in * L1.n_out
+    ell = loss_per_sample(loss, act_fn(L2.act, Z2, L2.act_param), y)
+    if idx < P1:
+        j, i = divmod(idx, L1.n_in)
+        delta = float(new_eff) - W1[j, i]
+        z = W1[j] @ XT
+        da = act_fn(L1.act, z + delta * XT[i], L1.act_param) - act_fn(L1.act, z, L1.act_param)
+        Z2n = Z2 + np.outer(W2[:, j], da)
+    else:
+        o, j = divmod(idx - P1, L2.n_in)
+        delta = float(new_eff) - W2[o, j]
+        a = act_fn(L1.act, W1[j] @ XT, L1.act_param)
+        Z2n = Z2.copy()
+        Z2n[o] += delta * a
+    ell_new = loss_per_sample(loss, act_fn(L2.act, Z2n, L2.act_param), y)
+    return float((ell_new - ell).sum())

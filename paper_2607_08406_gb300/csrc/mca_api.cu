@@ -1,0 +1,717 @@
+// C ABI of the MCA trial loop (include/mca.h): argument checks, device memory layout, the
+// creation-time full forward pass, and the host side of mca_run.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "mca_device.cuh"
+#include "mca_internal.h"
+
+using mca::DevState;
+using mca::GridBarrier;
+
+namespace {
+
+thread_local std::string g_create_err;
+
+mca_status fail(mca_handle* h, mca_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  if (h)
+    h->err = buf;
+  else
+    g_create_err = buf;
+  return st;
+}
+
+void mark_broken(mca_handle* h, cudaError_t e) {
+  // An allocation failure leaves the context usable; any other CUDA error may be sticky.
+  if (h && e != cudaErrorMemoryAllocation) h->broken = true;
+}
+
+#define CUDA_TRY(h, expr)                                                                    \
+  do {                                                                                       \
+    cudaError_t e_ = (expr);                                                                 \
+    if (e_ != cudaSuccess) {                                                                 \
+      mark_broken((h), e_);                                                                  \
+      return fail((h), e_ == cudaErrorMemoryAllocation ? MCA_ERR_OOM : MCA_ERR_CUDA,         \
+                  "%s: %s (%s:%d)", #expr, cudaGetErrorString(e_), __FILE__, __LINE__);      \
+    }                                                                                        \
+  } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool is_device_ptr(const void* p) {
+  if (!p) return false;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+struct Layout {
+  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, z1, srec, partial, bar, st, trace, ex_idx, ex_new, ex_out,
+      scratch, total;
+  std::vector<size_t> w_eff, code, wfix;
+};
+
+int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
+
+Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long nnz, int trace_cap) {
+  Layout L;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align256(o + bytes);
+    return at;
+  };
+  const int Np = pad_n(N);
+  const int H = layers[0].n_out;
+  const int maxch = (int)((std::max<long long>(N, 1) + mca::kChunk - 1) / mca::kChunk);
+  L.XT = take(sizeof(float) * (size_t)D * Np);
+  L.y = take(sizeof(int) * (size_t)N);
+  L.xs_off = take(sizeof(int) * (size_t)(D + 1));
+  L.xs_n = take(sizeof(int) * (size_t)std::max<long long>(nnz, 1));
+  L.xs_v = take(sizeof(float) * (size_t)std::max<long long>(nnz, 1));
+  L.xs_sect = take(sizeof(int) * (size_t)D);
+  for (const auto& ly : layers) {
+    const size_t n = (size_t)ly.n_in * ly.n_out;
+    L.w_eff.push_back(take(sizeof(float) * n));
+    L.code.push_back(ly.wkind != MCA_W_FP32 ? take(n) : SIZE_MAX);
+    L.wfix.push_back(ly.wkind == MCA_W_MASKED_FP32 ? take(sizeof(float) * n) : SIZE_MAX);
+  }
+  L.z1 = take(sizeof(float) * (size_t)H * Np);
+  L.srec = take(sizeof(float) * (size_t)mca::kSR * N);
+  L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * maxch);
+  L.bar = take(sizeof(GridBarrier));
+  L.st = take(sizeof(DevState));
+  L.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
+  L.ex_idx = take(sizeof(unsigned int) * mca::kKmax);
+  L.ex_new = take(sizeof(float) * mca::kKmax);
+  L.ex_out = take(sizeof(double) * mca::kKmax);
+  L.scratch = take(sizeof(int) * (size_t)(D + 8));
+  L.total = o;
+  return L;
+}
+
+mca_status check_spec(const mca_layer* layers, int n_layers, int loss, const mca_dataset* data,
+                      std::vector<mca_layer>* out) {
+  if (!layers || n_layers < 2) return fail(nullptr, MCA_ERR_INVALID, "need n_layers >= 2");
+  if (!data || !data->x || !data->y || data->n <= 0 || data->d <= 0)
+    return fail(nullptr, MCA_ERR_INVALID, "empty or missing dataset");
+  if (data->n >= (1ll << 31) - 1024) return fail(nullptr, MCA_ERR_INVALID, "N too large");
+  if (loss != MCA_LOSS_MSE_ONEHOT && loss != MCA_LOSS_SOFTMAX_CE)
+    return fail(nullptr, MCA_ERR_INVALID, "unknown loss %d", loss);
+  unsigned long long P = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    const mca_layer& L = layers[l];
+    if (L.n_in <= 0 || L.n_out <= 0) return fail(nullptr, MCA_ERR_INVALID, "layer %d: bad size", l);
+    if (l == 0 && L.n_in != data->d)
+      return fail(nullptr, MCA_ERR_INVALID, "layer 0 n_in %d != data d %d", L.n_in, data->d);
+    if (l > 0 && L.n_in != layers[l - 1].n_out)
+      return fail(nullptr, MCA_ERR_INVALID, "layer %d n_in != layer %d n_out", l, l - 1);
+    if (L.act < MCA_ACT_IDENTITY || L.act > MCA_ACT_GELU)
+      return fail(nullptr, MCA_ERR_INVALID, "layer %d: unknown act %d", l, L.act);
+    if (L.wkind < MCA_W_FP32 || L.wkind > MCA_W_MASKED_FP32)
+      return fail(nullptr, MCA_ERR_INVALID, "layer %d: unknown wkind %d", l, L.wkind);
+    if (!std::isfinite(L.act_param) || !std::isfinite(L.scale))
+      return fail(nullptr, MCA_ERR_INVALID, "layer %d: non-finite parameter", l);
+    P += (unsigned long long)L.n_in * (unsigned long long)L.n_out;
+  }
+  if (P >= (1ull << 32)) return fail(nullptr, MCA_ERR_INVALID, "P = %llu >= 2^32", P);
+  const int C = layers[n_layers - 1].n_out;
+  if (C > mca::kMaxClasses)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "%d outputs > %d", C, mca::kMaxClasses);
+  if (n_layers != 2)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "this build runs single-hidden-layer nets only");
+  out->assign(layers, layers + n_layers);
+  return MCA_OK;
+}
+
+mca_options default_options() {
+  mca_options o;
+  std::memset(&o, 0, sizeof(o));
+  o.K = 32;
+  return o;
+}
+
+mca_domain default_domain() {
+  mca_domain d;
+  std::memset(&d, 0, sizeof(d));
+  d.op = MCA_OP_REPLACE;
+  d.lo = -1.0f;
+  d.hi = 1.0f;
+  d.delta = 0.01f;
+  return d;
+}
+
+long long host_nnz(const float* x, size_t n) {
+  long long c = 0;
+  for (size_t i = 0; i < n; ++i) c += x[i] != 0.0f;
+  return c;
+}
+
+__global__ void count_nonzero_kernel(const float* __restrict__ p, size_t n,
+                                     unsigned long long* out) {
+  unsigned int c = 0;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x)
+    c += p[i] != 0.0f;
+  c = __reduce_add_sync(0xffffffffu, c);
+  if ((threadIdx.x & 31) == 0) atomicAdd(out, (unsigned long long)c);
+}
+
+mca_status count_nnz(const mca_dataset* d, cudaStream_t s, long long* nnz) {
+  const size_t n = (size_t)d->n * (size_t)d->d;
+  if (!is_device_ptr(d->x)) {
+    *nnz = host_nnz(d->x, n);
+    return MCA_OK;
+  }
+  unsigned long long* dc = nullptr;
+  CUDA_TRY(nullptr, cudaMalloc(&dc, sizeof(unsigned long long)));
+  unsigned long long hc = 0;
+  cudaError_t e = cudaMemsetAsync(dc, 0, sizeof(unsigned long long), s);
+  if (e == cudaSuccess) {
+    const int grid = (int)std::min<size_t>(4096, (n + 255) / 256);
+    count_nonzero_kernel<<<grid, 256, 0, s>>>(d->x, n, dc);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&hc, dc, sizeof(hc), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  cudaFree(dc);
+  CUDA_TRY(nullptr, e);
+  *nnz = (long long)hc;
+  return MCA_OK;
+}
+
+mca::Mlp2Args mlp2_args(mca_handle* h) {
+  mca::Mlp2Args a;
+  std::memset(&a, 0, sizeof(a));
+  const mca_layer& L1 = h->layers[0];
+  const mca_layer& L2 = h->layers[1];
+  a.N = (int)h->N;
+  a.D = h->D;
+  a.H = L1.n_out;
+  a.C = h->C;
+  a.Np = h->Np;
+  a.CH = mca::kChunk;
+  a.maxch = h->maxch;
+  a.P = h->P;
+  a.P1 = (unsigned long long)L1.n_in * L1.n_out;
+  a.xs_off = h->xs_off;
+  a.xs_n = h->xs_n;
+  a.xs_v = h->xs_v;
+  a.xs_sect = h->xs_sect;
+  a.z1 = h->z1;
+  a.srec = h->srec;
+  a.w1 = h->w_eff[0];
+  a.w2 = h->w_eff[1];
+  a.code1 = h->code[0];
+  a.code2 = h->code[1];
+  a.wfix1 = h->wfix[0];
+  a.wfix2 = h->wfix[1];
+  a.wk1 = L1.wkind;
+  a.wk2 = L2.wkind;
+  a.sc1 = L1.scale;
+  a.sc2 = L2.scale;
+  a.act1 = L1.act;
+  a.act2 = L2.act;
+  a.g1 = L1.act_param;
+  a.g2 = L2.act_param;
+  a.loss = h->loss;
+  a.op = h->dom.op;
+  a.lo = h->dom.lo;
+  a.hi = h->dom.hi;
+  a.delta = h->dom.delta;
+  a.bound = h->dom.bound;
+  a.strict = h->dom.strict;
+  a.K = h->opt.K;
+  a.partial = h->partial;
+  a.bar = h->bar;
+  a.st = h->st;
+  a.trace = h->trace;
+  a.trace_cap = h->trace_cap;
+  a.ftau = h->ftau;
+  a.facc = h->facc;
+  a.nforce = h->nforce;
+  return a;
+}
+
+// Full forward pass: every cached field, every sample's loss, and S (Section 2.4's cache).
+mca_status resync(mca_handle* h) {
+  mca::Mlp2Args a = mlp2_args(h);
+  CUDA_TRY(h, mca::launch_sgemm_nn(a.H, h->Np, h->D, h->w_eff[0], h->D, h->XT, h->Np, h->z1,
+                                   h->Np, h->stream));
+  CUDA_TRY(h, mca::launch_mlp2_outputs(a, h->y, h->stream));
+  CUDA_TRY(h, mca::launch_sum_loss(h->srec, (int)h->N, h->st, h->stream));
+  h->launches += 3;
+  return MCA_OK;
+}
+
+// Load parameters in the init format into the per-layer weight arrays.
+mca_status load_params(mca_handle* h, const float* params, const signed char* codes) {
+  const bool pdev = is_device_ptr(params);
+  const bool cdev = codes && is_device_ptr(codes);
+  float* tmp = nullptr;
+  signed char* ctmp = nullptr;
+  const size_t P = h->P;
+  if (!pdev) {
+    CUDA_TRY(h, cudaMalloc(&tmp, sizeof(float) * P));
+    CUDA_TRY(h, cudaMemcpyAsync(tmp, params, sizeof(float) * P, cudaMemcpyHostToDevice, h->stream));
+  }
+  if (codes && !cdev) {
+    CUDA_TRY(h, cudaMalloc(&ctmp, P));
+    CUDA_TRY(h, cudaMemcpyAsync(ctmp, codes, P, cudaMemcpyHostToDevice, h->stream));
+  }
+  const float* src = pdev ? params : tmp;
+  const signed char* csrc = codes ? (cdev ? codes : ctmp) : nullptr;
+  mca_status rc = MCA_OK;
+  int* dflag = nullptr;
+  cudaError_t e = cudaMalloc(&dflag, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemsetAsync(dflag, 0, sizeof(int), h->stream);
+  if (e == cudaSuccess) e = mca::launch_count_nonfinite(src, P, dflag, h->stream);
+  for (size_t l = 0; e == cudaSuccess && l < h->layers.size(); ++l) {
+    const mca_layer& L = h->layers[l];
+    const size_t n = (size_t)L.n_in * L.n_out;
+    e = mca::launch_init_layer(L.wkind, L.scale, src + h->off[l], csrc ? csrc + h->off[l] : nullptr,
+                               n, h->w_eff[l], h->code[l], h->wfix[l], h->stream);
+    h->launches++;
+  }
+  int hflag = 0;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&hflag, dflag, sizeof(int), cudaMemcpyDeviceToHost,
+                                            h->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  cudaFree(dflag);
+  if (tmp) cudaFree(tmp);
+  if (ctmp) cudaFree(ctmp);
+  CUDA_TRY(h, e);
+  if (hflag) rc = fail(h, MCA_ERR_NUMERIC, "non-finite parameter value");
+  return rc;
+}
+
+mca_status read_state(mca_handle* h, DevState* out) {
+  CUDA_TRY(h, cudaMemcpyAsync(out, h->st, sizeof(DevState), cudaMemcpyDeviceToHost, h->stream));
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  return MCA_OK;
+}
+
+void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
+  s->trials = d.trials;
+  s->accepts = d.accepts;
+  s->candidates = d.candidates;
+  s->batches = d.batches;
+  s->wasted = d.wasted;
+  s->forced = d.forced;
+  s->resyncs = h->resyncs;
+  s->launches = h->launches;
+  s->tau = h->tau;
+  s->S = d.S;
+  s->alg_bytes = d.alg_bytes;
+}
+
+int auto_grid(mca_handle* h, int maxgrid) {
+  if (h->opt.grid > 0) return std::min(h->opt.grid, maxgrid);
+  const long long avg = h->nnz / std::max(1, h->D);
+  const long long per_cand = std::max<long long>(1, (avg + mca::kChunk - 1) / mca::kChunk);
+  long long g = (long long)h->opt.K * per_cand;
+  g = std::max<long long>(g, 1);
+  return (int)std::min<long long>(g, maxgrid);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* mca_last_error(mca_handle* h) {
+  return h ? h->err.c_str() : g_create_err.c_str();
+}
+
+mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t loss,
+                              const mca_dataset* data, const mca_options* opt, size_t* bytes) {
+  std::vector<mca_layer> ls;
+  mca_status rc = check_spec(layers, n_layers, loss, data, &ls);
+  if (rc != MCA_OK) return rc;
+  if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
+  const mca_options o = opt ? *opt : default_options();
+  long long nnz = 0;
+  rc = count_nnz(data, (cudaStream_t)o.stream, &nnz);
+  if (rc != MCA_OK) return rc;
+  *bytes = plan(ls, data->n, data->d, nnz, o.trace_cap).total;
+  return MCA_OK;
+}
+
+mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
+                      const mca_domain* dom, const mca_dataset* data, const float* init_params,
+                      const mca_options* opt, mca_handle** out) {
+  if (!out) return fail(nullptr, MCA_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  std::vector<mca_layer> ls;
+  mca_status rc = check_spec(layers, n_layers, loss, data, &ls);
+  if (rc != MCA_OK) return rc;
+  if (!init_params) return fail(nullptr, MCA_ERR_INVALID, "init_params is NULL");
+  const mca_options o = opt ? *opt : default_options();
+  if (o.K < 1 || o.K > mca::kKmax)
+    return fail(nullptr, MCA_ERR_INVALID, "K = %d outside 1..%d", o.K, mca::kKmax);
+  if (o.resync_period < 0 || o.trace_cap < 0 || o.grid < 0)
+    return fail(nullptr, MCA_ERR_INVALID, "negative option");
+  const mca_domain d = dom ? *dom : default_domain();
+  if (d.op != MCA_OP_REPLACE && d.op != MCA_OP_PERTURB)
+    return fail(nullptr, MCA_ERR_INVALID, "unknown op %d", d.op);
+  if (!std::isfinite(d.lo) || !std::isfinite(d.hi) || !std::isfinite(d.delta) || !(d.hi > d.lo))
+    return fail(nullptr, MCA_ERR_INVALID, "bad domain");
+
+  mca_handle* h = new (std::nothrow) mca_handle();
+  if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
+  h->layers = ls;
+  h->loss = loss;
+  h->dom = d;
+  h->opt = o;
+  h->N = data->n;
+  h->D = data->d;
+  h->C = ls.back().n_out;
+  h->Np = pad_n(h->N);
+  h->stream = (cudaStream_t)o.stream;
+  unsigned long long P = 0;
+  for (const auto& L : ls) {
+    h->off.push_back(P);
+    P += (unsigned long long)L.n_in * L.n_out;
+  }
+  h->P = P;
+  h->maxch = (int)((h->N + mca::kChunk - 1) / mca::kChunk);
+  h->trace_cap = o.trace_cap;
+
+  auto bail = [&](mca_status st) {
+    g_create_err = h->err;
+    mca_destroy(h);
+    return st;
+  };
+#define TRY(expr)                                   \
+  do {                                              \
+    mca_status s_ = (expr);                         \
+    if (s_ != MCA_OK) return bail(s_);              \
+  } while (0)
+#define CTRY(expr)                                                                             \
+  do {                                                                                         \
+    cudaError_t e_ = (expr);                                                                   \
+    if (e_ != cudaSuccess)                                                                     \
+      return bail(fail(h, e_ == cudaErrorMemoryAllocation ? MCA_ERR_OOM : MCA_ERR_CUDA,        \
+                       "%s: %s", #expr, cudaGetErrorString(e_)));                              \
+  } while (0)
+
+  CTRY(cudaGetDevice(&h->device));
+  CTRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
+  {
+    long long nnz = 0;
+    mca_status s = count_nnz(data, h->stream, &nnz);
+    if (s != MCA_OK) {
+      h->err = g_create_err;
+      return bail(s);
+    }
+    h->nnz = nnz;
+  }
+  const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap);
+  if (o.workspace) {
+    if (o.workspace_bytes < L.total)
+      return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
+                       L.total));
+    if (reinterpret_cast<uintptr_t>(o.workspace) % 256 != 0)
+      return bail(fail(h, MCA_ERR_INVALID, "workspace not 256-byte aligned"));
+    h->ws = o.workspace;
+    h->ws_bytes = o.workspace_bytes;
+  } else {
+    CTRY(cudaMalloc(&h->ws, L.total));
+    h->ws_owned = true;
+    h->ws_bytes = L.total;
+  }
+  char* base = static_cast<char*>(h->ws);
+  h->XT = reinterpret_cast<float*>(base + L.XT);
+  h->y = reinterpret_cast<int*>(base + L.y);
+  h->xs_off = reinterpret_cast<int*>(base + L.xs_off);
+  h->xs_n = reinterpret_cast<int*>(base + L.xs_n);
+  h->xs_v = reinterpret_cast<float*>(base + L.xs_v);
+  h->xs_sect = reinterpret_cast<int*>(base + L.xs_sect);
+  for (size_t l = 0; l < ls.size(); ++l) {
+    h->w_eff.push_back(reinterpret_cast<float*>(base + L.w_eff[l]));
+    h->code.push_back(L.code[l] == SIZE_MAX ? nullptr
+                                            : reinterpret_cast<signed char*>(base + L.code[l]));
+    h->wfix.push_back(L.wfix[l] == SIZE_MAX ? nullptr : reinterpret_cast<float*>(base + L.wfix[l]));
+  }
+  h->z1 = reinterpret_cast<float*>(base + L.z1);
+  h->srec = reinterpret_cast<float*>(base + L.srec);
+  h->partial = reinterpret_cast<float*>(base + L.partial);
+  h->bar = reinterpret_cast<GridBarrier*>(base + L.bar);
+  h->st = reinterpret_cast<DevState*>(base + L.st);
+  h->trace = o.trace_cap > 0 ? reinterpret_cast<mca_trace_rec*>(base + L.trace) : nullptr;
+  h->ex_idx = reinterpret_cast<unsigned int*>(base + L.ex_idx);
+  h->ex_new = reinterpret_cast<float*>(base + L.ex_new);
+  h->ex_out = reinterpret_cast<double*>(base + L.ex_out);
+  int* scratch = reinterpret_cast<int*>(base + L.scratch);
+  CTRY(cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream));
+  CTRY(cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
+  CTRY(cudaMemsetAsync(h->partial, 0, L.st - L.partial, h->stream));
+
+  // dataset: X -> XT (feature-major, zero-padded), CSR by feature, labels
+  const size_t nx = (size_t)h->N * h->D;
+  const float* Xd = data->x;
+  float* Xtmp = nullptr;
+  if (!is_device_ptr(data->x)) {
+    CTRY(cudaMalloc(&Xtmp, sizeof(float) * nx));
+    CTRY(cudaMemcpyAsync(Xtmp, data->x, sizeof(float) * nx, cudaMemcpyHostToDevice, h->stream));
+    Xd = Xtmp;
+  }
+  CTRY(cudaMemsetAsync(scratch, 0, sizeof(int), h->stream));
+  CTRY(mca::launch_count_nonfinite(Xd, nx, scratch, h->stream));
+  CTRY(mca::launch_transpose_pad(Xd, (int)h->N, h->D, h->XT, h->Np, h->stream));
+  CTRY(mca::launch_csr_count(h->XT, h->Np, (int)h->N, h->D, scratch + 8, h->stream));
+  h->launches += 3;
+  std::vector<int> cnt(h->D + 8);
+  CTRY(cudaMemcpyAsync(cnt.data(), scratch, sizeof(int) * (h->D + 8), cudaMemcpyDeviceToHost,
+                       h->stream));
+  CTRY(cudaStreamSynchronize(h->stream));
+  if (Xtmp) cudaFree(Xtmp);
+  if (cnt[0]) return bail(fail(h, MCA_ERR_NUMERIC, "non-finite value in x"));
+  std::vector<int> offs(h->D + 1, 0);
+  long long acc = 0;
+  for (int i = 0; i < h->D; ++i) {
+    offs[i] = (int)acc;
+    acc += cnt[8 + i];
+    h->max_nnz = std::max(h->max_nnz, cnt[8 + i]);
+  }
+  offs[h->D] = (int)acc;
+  if (acc != h->nnz) return bail(fail(h, MCA_ERR_INVALID, "nnz mismatch %lld vs %lld", acc, h->nnz));
+  CTRY(cudaMemcpyAsync(h->xs_off, offs.data(), sizeof(int) * (h->D + 1), cudaMemcpyHostToDevice,
+                       h->stream));
+  CTRY(mca::launch_csr_fill(h->XT, h->Np, (int)h->N, h->D, h->xs_off, h->xs_n, h->xs_v, h->stream));
+  CTRY(mca::launch_csr_sectors(h->xs_off, h->xs_n, h->D, h->xs_sect, h->stream));
+  h->launches += 2;
+  {
+    std::vector<int> yh(h->N);
+    CTRY(cudaMemcpyAsync(yh.data(), data->y, sizeof(int) * h->N, cudaMemcpyDefault, h->stream));
+    CTRY(cudaStreamSynchronize(h->stream));
+    for (long long n = 0; n < h->N; ++n)
+      if (yh[n] < 0 || yh[n] >= h->C)
+        return bail(fail(h, MCA_ERR_INVALID, "label %d of sample %lld outside [0, %d)", yh[n], n,
+                         h->C));
+    CTRY(cudaMemcpyAsync(h->y, yh.data(), sizeof(int) * h->N, cudaMemcpyHostToDevice, h->stream));
+    CTRY(cudaStreamSynchronize(h->stream));
+  }
+  TRY(load_params(h, init_params, nullptr));
+  TRY(resync(h));
+  DevState ds;
+  TRY(read_state(h, &ds));
+  if (!std::isfinite(ds.S)) return bail(fail(h, MCA_ERR_NUMERIC, "initial loss is not finite"));
+  {
+    mca::Mlp2Args a = mlp2_args(h);
+    const int maxgrid = mca::mlp2_loop_max_grid(a, h->num_sms);
+    if (maxgrid <= 0) return bail(fail(h, MCA_ERR_CUDA, "trial-loop kernel cannot be resident"));
+    h->grid = auto_grid(h, maxgrid);
+  }
+#undef TRY
+#undef CTRY
+  *out = h;
+  return MCA_OK;
+}
+
+mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stats* stats) {
+  if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  uint64_t remaining = n_trials;
+  while (remaining > 0) {
+    uint64_t seg = remaining;
+    const uint64_t R = (uint64_t)h->opt.resync_period;
+    if (R > 0) seg = std::min<uint64_t>(seg, R - h->tau % R);
+    mca::Mlp2Args a = mlp2_args(h);
+    a.seed = seed;
+    a.tau0 = h->tau;
+    a.n_trials = seg;
+    CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
+    CUDA_TRY(h, mca::launch_mlp2_loop(a, h->grid, h->stream));
+    h->launches++;
+    h->tau += seg;
+    remaining -= seg;
+    if (R > 0 && h->tau % R == 0) {
+      mca_status rc = resync(h);
+      if (rc != MCA_OK) return rc;
+      h->resyncs++;
+    }
+  }
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  if (stats) fill_stats(h, ds, stats);
+  if (ds.err != 0) {
+    h->broken = true;
+    return fail(h, (mca_status)ds.err, ds.err == MCA_ERR_TIMEOUT
+                                           ? "device-side wait timed out"
+                                           : "non-finite loss change");
+  }
+  return MCA_OK;
+}
+
+mca_status mca_loss(mca_handle* h, double* L) {
+  if (!h || !L) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  *L = ds.S / (double)h->N;
+  return MCA_OK;
+}
+
+mca_status mca_get_stats(mca_handle* h, mca_run_stats* stats) {
+  if (!h || !stats) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  fill_stats(h, ds, stats);
+  return MCA_OK;
+}
+
+mca_status mca_get_params(mca_handle* h, float* dst, size_t n) {
+  if (!h || !dst) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (n != h->P) return fail(h, MCA_ERR_INVALID, "n = %zu, P = %llu", n, h->P);
+  for (size_t l = 0; l < h->layers.size(); ++l) {
+    const size_t m = (size_t)h->layers[l].n_in * h->layers[l].n_out;
+    CUDA_TRY(h, cudaMemcpyAsync(dst + h->off[l], h->w_eff[l], sizeof(float) * m, cudaMemcpyDefault,
+                                h->stream));
+  }
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  return MCA_OK;
+}
+
+mca_status mca_get_codes(mca_handle* h, int8_t* dst, size_t n) {
+  if (!h || !dst) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (n != h->P) return fail(h, MCA_ERR_INVALID, "n = %zu, P = %llu", n, h->P);
+  const bool dev = is_device_ptr(dst);
+  for (size_t l = 0; l < h->layers.size(); ++l) {
+    const size_t m = (size_t)h->layers[l].n_in * h->layers[l].n_out;
+    if (h->code[l]) {
+      CUDA_TRY(h, cudaMemcpyAsync(dst + h->off[l], h->code[l], m, cudaMemcpyDefault, h->stream));
+    } else if (dev) {
+      CUDA_TRY(h, cudaMemsetAsync(dst + h->off[l], 0, m, h->stream));
+    } else {
+      CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+      std::memset(dst + h->off[l], 0, m);
+    }
+  }
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  return MCA_OK;
+}
+
+mca_status mca_set_params(mca_handle* h, const float* params, const int8_t* codes, size_t n,
+                          uint64_t tau) {
+  if (!h || !params) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (n != h->P) return fail(h, MCA_ERR_INVALID, "n = %zu, P = %llu", n, h->P);
+  mca_status rc = load_params(h, params, reinterpret_cast<const signed char*>(codes));
+  if (rc != MCA_OK) return rc;
+  rc = resync(h);
+  if (rc != MCA_OK) return rc;
+  h->tau = tau;
+  return MCA_OK;
+}
+
+mca_status mca_resync(mca_handle* h) {
+  if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  mca_status rc = resync(h);
+  if (rc != MCA_OK) return rc;
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  return MCA_OK;
+}
+
+mca_status mca_get_trace(mca_handle* h, mca_trace_rec* dst, size_t cap, size_t* n) {
+  if (!h || !n || (!dst && cap)) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (h->trace_cap <= 0) return fail(h, MCA_ERR_INVALID, "created without a trace");
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  const unsigned long long tc = (unsigned long long)h->trace_cap;
+  const unsigned long long have = std::min<unsigned long long>(ds.trace_written, tc);
+  const unsigned long long take = std::min<unsigned long long>(have, cap);
+  std::vector<mca_trace_rec> ring(tc);
+  CUDA_TRY(h, cudaMemcpyAsync(ring.data(), h->trace, sizeof(mca_trace_rec) * tc,
+                              cudaMemcpyDeviceToHost, h->stream));
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  const unsigned long long first = ds.trace_written - take;
+  for (unsigned long long m = 0; m < take; ++m) dst[m] = ring[(first + m) % tc];
+  *n = (size_t)take;
+  return MCA_OK;
+}
+
+mca_status mca_force_decisions(mca_handle* h, const uint64_t* tau, const uint8_t* accept,
+                               size_t n) {
+  if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  if (n && (!tau || !accept)) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  for (size_t m = 1; m < n; ++m)
+    if (tau[m] <= tau[m - 1]) return fail(h, MCA_ERR_INVALID, "tau not strictly increasing");
+  if (h->ftau) cudaFree(h->ftau);
+  if (h->facc) cudaFree(h->facc);
+  h->ftau = nullptr;
+  h->facc = nullptr;
+  h->nforce = 0;
+  if (n == 0) return MCA_OK;
+  CUDA_TRY(h, cudaMalloc(&h->ftau, sizeof(unsigned long long) * n));
+  CUDA_TRY(h, cudaMalloc(&h->facc, n));
+  CUDA_TRY(h, cudaMemcpyAsync(h->ftau, tau, sizeof(unsigned long long) * n, cudaMemcpyHostToDevice,
+                              h->stream));
+  CUDA_TRY(h, cudaMemcpyAsync(h->facc, accept, n, cudaMemcpyHostToDevice, h->stream));
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  h->nforce = (int)n;
+  return MCA_OK;
+}
+
+mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
+                               size_t n, double* dS) {
+  if (!h || (n && (!flat_idx || !new_w || !dS))) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (n > (size_t)mca::kKmax) return fail(h, MCA_ERR_INVALID, "n = %zu > %d", n, mca::kKmax);
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (n == 0) return MCA_OK;
+  for (size_t m = 0; m < n; ++m) {
+    if (flat_idx[m] >= h->P) return fail(h, MCA_ERR_INVALID, "flat_idx[%zu] >= P", m);
+    if (!std::isfinite(new_w[m])) return fail(h, MCA_ERR_INVALID, "new_w[%zu] not finite", m);
+  }
+  CUDA_TRY(h, cudaMemcpyAsync(h->ex_idx, flat_idx, sizeof(unsigned int) * n, cudaMemcpyHostToDevice,
+                              h->stream));
+  CUDA_TRY(h, cudaMemcpyAsync(h->ex_new, new_w, sizeof(float) * n, cudaMemcpyHostToDevice,
+                              h->stream));
+  mca::Mlp2Args a = mlp2_args(h);
+  a.n_explicit = (int)n;
+  a.ex_idx = h->ex_idx;
+  a.ex_new = h->ex_new;
+  a.ex_out = h->ex_out;
+  CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
+  CUDA_TRY(h, mca::launch_mlp2_loop(a, h->grid, h->stream));
+  h->launches++;
+  CUDA_TRY(h, cudaMemcpyAsync(dS, h->ex_out, sizeof(double) * n, cudaMemcpyDeviceToHost,
+                              h->stream));
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  if (ds.err == MCA_ERR_TIMEOUT) {
+    h->broken = true;
+    return fail(h, MCA_ERR_TIMEOUT, "device-side wait timed out");
+  }
+  return MCA_OK;
+}
+
+void mca_destroy(mca_handle* h) {
+  if (!h) return;
+  cudaStreamSynchronize(h->stream);
+  if (h->ws_owned && h->ws) cudaFree(h->ws);
+  if (h->ftau) cudaFree(h->ftau);
+  if (h->facc) cudaFree(h->facc);
+  delete h;
+}
+
+}  // extern "C"

@@ -1,0 +1,205 @@
+// Device building blocks of the MCA trial loop: the Philox proposal stream, transfer functions,
+// per-sample losses, deterministic block reductions and a bounded grid barrier.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/mca.h"
+
+namespace mca {
+
+// ------------------------------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11, Section 3.2): ten rounds of two 32x32->64
+// multiplies and xors over a 128-bit counter, the 64-bit key bumped by the Weyl constants between
+// rounds. Counter = (tau_lo, tau_hi, 0, 0), key = (seed_lo, seed_hi).
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k.x += 0x9E3779B9u;
+      k.y += 0xBB67AE85u;
+    }
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+  }
+  return c;
+}
+
+__device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
+  return philox4x32_10(make_uint4((uint32_t)tau, (uint32_t)(tau >> 32), 0u, 0u),
+                       make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+}
+
+// u = (r >> 8) * 2^-24: exact, in [0, 1)
+__device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >> 8) * 0x1p-24f; }
+
+// ------------------------------------------------------------------------------------------------
+// Transfer functions (Section 2) and losses (Eq. 2 with R = 0). ACT < 0 selects at run time.
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ float act_rt(int act, float z, float g) {
+  switch (act) {
+    case MCA_ACT_TANH: return tanhf(z);
+    case MCA_ACT_SIGMOID: return 1.0f / (1.0f + expf(-z));
+    case MCA_ACT_RELU: return fmaxf(z, 0.0f);
+    case MCA_ACT_GAUSSIAN: return expf(-g * z * z);
+    case MCA_ACT_GELU: return 0.5f * z * (1.0f + erff(z * 0.7071067811865476f));
+    default: return z;
+  }
+}
+
+template <int ACT>
+__device__ __forceinline__ float act(float z, float g, int act_runtime) {
+  if constexpr (ACT < 0) {
+    return act_rt(act_runtime, z, g);
+  } else {
+    return act_rt(ACT, z, g);
+  }
+}
+
+// Per-sample loss of the output fields z[0..C) with label y.
+template <int ACT2, int LOSS, int MAXC>
+__device__ __forceinline__ float sample_loss(const float (&z)[MAXC], int C, int y, float g2,
+                                             int act2_rt, int loss_rt) {
+  const int loss = LOSS < 0 ? loss_rt : LOSS;
+  if (loss == MCA_LOSS_MSE_ONEHOT) {
+    float s = 0.0f;
+#pragma unroll
+    for (int k = 0; k < MAXC; ++k) {
+      if (k < C) {
+        const float d = act<ACT2>(z[k], g2, act2_rt) - (k == y ? 1.0f : 0.0f);
+        s = fmaf(d, d, s);
+      }
+    }
+    return s;
+  }
+  float a[MAXC];
+  float m = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < MAXC; ++k) {
+    if (k < C) {
+      a[k] = act<ACT2>(z[k], g2, act2_rt);
+      m = fmaxf(m, a[k]);
+    }
+  }
+  float s = 0.0f, ay = 0.0f;
+#pragma unroll
+  for (int k = 0; k < MAXC; ++k) {
+    if (k < C) {
+      s += expf(a[k] - m);
+      if (k == y) ay = a[k];
+    }
+  }
+  return (logf(s) + m) - ay;
+}
+
+// ------------------------------------------------------------------------------------------------
+// Deterministic reductions (fixed shuffle tree, fixed warp order)
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over the block; the result is valid in every thread. red: >= 32 floats of shared memory.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = lane < nw ? red[lane] : 0.0f;
+  t = warp_sum(t);
+  return t;
+}
+
+__device__ __forceinline__ double block_sum_d(double v, double* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum_d(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  double t = lane < nw ? red[lane] : 0.0;
+  t = warp_sum_d(t);
+  return t;
+}
+
+// ------------------------------------------------------------------------------------------------
+// Grid barrier for a co-resident (cooperative) grid. Every wait is bounded: after kBarrierTimeoutNs
+// the waiting CTA records MCA_ERR_TIMEOUT in *err and returns false, and so does every CTA that
+// sees a non-zero *err while waiting; callers then leave the kernel.
+// ------------------------------------------------------------------------------------------------
+struct GridBarrier {
+  unsigned int count;
+  unsigned int gen;
+};
+
+constexpr unsigned long long kBarrierTimeoutNs = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int* p) {
+  unsigned int v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_gpu(unsigned int* p, unsigned int v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_volatile_int(const int* p) {
+  return *reinterpret_cast<const volatile int*>(p);
+}
+
+// gen_local: this CTA's copy of the barrier generation (same value in every CTA between barriers).
+__device__ __forceinline__ bool grid_sync(GridBarrier* bar, unsigned int nblocks,
+                                          unsigned int& gen_local, int* err, int* s_flag) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    const unsigned int g = gen_local;
+    __threadfence();
+    const unsigned int prev = atomicAdd(&bar->count, 1u);
+    if (prev == nblocks - 1) {
+      bar->count = 0u;
+      __threadfence();
+      st_release_gpu(&bar->gen, g + 1u);
+    } else {
+      const unsigned long long t0 = globaltimer_ns();
+      unsigned int spins = 0;
+      while (ld_acquire_gpu(&bar->gen) == g) {
+        if (ld_volatile_int(err) != 0) {
+          ok = 0;
+          break;
+        }
+        if ((++spins & 63u) == 0u && globaltimer_ns() - t0 > kBarrierTimeoutNs) {
+          atomicCAS(err, 0, (int)MCA_ERR_TIMEOUT);
+          ok = 0;
+          break;
+        }
+      }
+    }
+    __threadfence();
+    gen_local = g + 1u;
+    *s_flag = ok && ld_volatile_int(err) == 0;
+  }
+  __syncthreads();
+  const bool ok = *s_flag != 0;
+  return ok;
+}
+
+}  // namespace mca

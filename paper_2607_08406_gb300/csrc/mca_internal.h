@@ -1,0 +1,140 @@
+// Internal declarations shared by the C-ABI layer (mca_api.cu) and the kernels.
+#pragma once
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/mca.h"
+
+namespace mca {
+
+struct GridBarrier;
+
+constexpr int kKmax = 128;        // speculative candidates per batch
+constexpr int kMaxC = 16;         // register arrays of the output layer
+constexpr int kSR = 16;           // floats per sample record: fields [0, C), loss at 14, label at 15
+constexpr int kMaxClasses = kSR - 2;
+constexpr int kLoopThreads = 512; // threads per CTA of the trial-loop kernel
+constexpr int kPerThread = 4;     // entries per thread per chunk
+constexpr int kChunk = kLoopThreads * kPerThread;   // entries per work item (fixed partition)
+
+// Device-resident run state (one per handle).
+struct DevState {
+  double S;                  // loss sum of the cached state
+  unsigned long long trials, accepts, candidates, batches, wasted, forced, trace_written;
+  unsigned long long alg_bytes;  // compulsory DRAM bytes of the evaluated candidates and commits
+  int err;                   // first device-side error (mca_status), 0 = none
+  int pad;
+};
+
+// Arguments of the two-layer trial loop (input -> hidden -> output).
+struct Mlp2Args {
+  int N, D, H, C, Np, CH, maxch;
+  unsigned long long P, P1;
+  const int* xs_off;         // [D + 1] CSR of X by feature: entries of feature i in [off[i], off[i+1])
+  const int* xs_n;           // [nnz] sample index of each entry (ascending inside a feature)
+  const float* xs_v;         // [nnz] value x[n, i] != 0
+  const int* xs_sect;        // [D] 32-byte sectors of a z1 row that feature i's entries touch
+  float* z1;                 // [H x Np] hidden fields, feature-major
+  float* srec;               // [N x kSR] output fields, loss, label
+  float* w1;                 // [H x D] effective weights
+  float* w2;                 // [C x H]
+  signed char* code1;        // ternary codes / mask bits (nullable for fp32 layers)
+  signed char* code2;
+  const float* wfix1;        // masked layers: fixed weights
+  const float* wfix2;
+  int wk1, wk2;
+  float sc1, sc2;
+  int act1, act2;
+  float g1, g2;
+  int loss;
+  int op;
+  float lo, hi, delta, bound;
+  int strict;
+  unsigned long long seed, tau0, n_trials;
+  int K;
+  float* partial;            // [2 x kKmax x maxch]
+  GridBarrier* bar;
+  DevState* st;
+  mca_trace_rec* trace;
+  int trace_cap;
+  const unsigned long long* ftau;
+  const unsigned char* facc;
+  int nforce;
+  int n_explicit;            // > 0: evaluate these candidates once, no decision, no commit
+  const unsigned int* ex_idx;
+  const float* ex_new;
+  double* ex_out;
+};
+
+// Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
+cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
+cudaError_t launch_csr_count(const float* XT, int Np, int N, int D, int* cnt, cudaStream_t s);
+cudaError_t launch_csr_fill(const float* XT, int Np, int N, int D, const int* off, int* xs_n,
+                            float* xs_v, cudaStream_t s);
+cudaError_t launch_csr_sectors(const int* off, const int* xs_n, int D, int* sect, cudaStream_t s);
+cudaError_t launch_count_nonfinite(const float* p, size_t n, int* out, cudaStream_t s);
+cudaError_t launch_init_layer(int wkind, float scale, const float* src, const signed char* mask,
+                              size_t n, float* w_eff, signed char* code, float* wfix,
+                              cudaStream_t s);
+cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, const float* B,
+                            int ldb, float* C, int ldc, cudaStream_t s);
+cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s);
+cudaError_t launch_sum_loss(const float* srec, int N, DevState* st, cudaStream_t s);
+// Cooperative persistent trial loop; grid <= co-resident CTAs.
+cudaError_t launch_mlp2_loop(const Mlp2Args& a, int grid, cudaStream_t s);
+int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);
+
+}  // namespace mca
+
+struct mca_handle {
+  std::string err;
+  std::vector<mca_layer> layers;
+  int loss = 0;
+  mca_domain dom{};
+  mca_options opt{};
+  long long N = 0;
+  int D = 0, C = 0, Np = 0;
+  unsigned long long P = 0;
+  std::vector<unsigned long long> off;   // flat offset of each layer
+  cudaStream_t stream = nullptr;
+  int device = 0, num_sms = 0;
+  // memory
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  bool ws_owned = false;
+  float* XT = nullptr;                   // [D x Np]
+  int* y = nullptr;
+  int* xs_off = nullptr;
+  int* xs_n = nullptr;
+  float* xs_v = nullptr;
+  int* xs_sect = nullptr;
+  long long nnz = 0;
+  int max_nnz = 0;
+  std::vector<float*> w_eff;
+  std::vector<signed char*> code;
+  std::vector<float*> wfix;
+  float* z1 = nullptr;
+  float* srec = nullptr;
+  float* partial = nullptr;
+  int maxch = 0;
+  mca::GridBarrier* bar = nullptr;
+  mca::DevState* st = nullptr;
+  mca_trace_rec* trace = nullptr;
+  int trace_cap = 0;
+  unsigned int* ex_idx = nullptr;
+  float* ex_new = nullptr;
+  double* ex_out = nullptr;
+  // test hook
+  unsigned long long* ftau = nullptr;
+  unsigned char* facc = nullptr;
+  int nforce = 0;
+  // host-side counters
+  unsigned long long tau = 0;
+  unsigned long long launches = 0, resyncs = 0;
+  int grid = 0;
+  bool broken = false;                   // a sticky CUDA error or device timeout was seen
+};

@@ -1,0 +1,46 @@
+"""Helpers that compare the CUDA path's trial records with the oracle's (used by the -m gpu tests)."""
+import numpy as np
+
+from oracle import mca_oracle as O
+
+TIE_REL = 1e-5     # |dS| < 1e-5 * S: either decision is correct (candidate losses agree to 1e-5)
+
+
+def oracle_trace(wl, n_trials, seed=0, mode="incremental", domain=None):
+    run = O.run_incremental if mode == "incremental" else O.run_full
+    tr, params, S = run(wl.layers, wl.loss, wl.X, wl.y, wl.init, n_trials, seed,
+                        domain or wl.domain)
+    return tr, params, S
+
+
+def tie_band(tr):
+    """Trials where the oracle's |dS| < TIE_REL * S and dS != 0 (exact zeros must match)."""
+    d = np.abs(tr["dS"])
+    return tr["valid"] & (d < TIE_REL * np.abs(tr["S"])) & (tr["dS"] != 0.0)
+
+
+def forced_from_oracle(tr):
+    m = tie_band(tr)
+    return tr["tau"][m].astype(np.uint64), tr["accept"][m]
+
+
+def compare(gpu, ora, check_dS=True):
+    """gpu: structured array from mca_get_trace; ora: oracle trace dict. Proposals bit-exact,
+    decisions equal, dS within TIE_REL * S."""
+    n = len(ora["tau"])
+    assert len(gpu) == n, (len(gpu), n)
+    assert np.array_equal(gpu["tau"].astype(np.int64), ora["tau"])
+    assert np.array_equal(gpu["idx"].astype(np.int64), ora["idx"])
+    assert np.array_equal(gpu["new_w"], ora["new"].astype(np.float32))
+    assert np.array_equal(gpu["old_w"], ora["old"].astype(np.float32))
+    assert np.array_equal(gpu["valid"].astype(bool), ora["valid"])
+    bad = np.nonzero(gpu["accept"].astype(bool) != ora["accept"])[0]
+    assert len(bad) == 0, f"first decision mismatch at trial {bad[:5]}: gpu dS {gpu['dS'][bad[:5]]}, " \
+                          f"oracle dS {ora['dS'][bad[:5]]}, S {ora['S'][bad[:5]]}"
+    if check_dS:
+        v = ora["valid"]
+        err = np.abs(gpu["dS"][v] - ora["dS"][v])
+        tol = TIE_REL * np.abs(ora["S"][v])
+        worst = int(np.argmax(err / tol)) if v.any() else 0
+        assert np.all(err <= tol), f"dS error {err[worst]} > {tol[worst]}"
+        assert np.allclose(gpu["S"], ora["S"], rtol=TIE_REL, atol=0)

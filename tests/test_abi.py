@@ -1,0 +1,118 @@
+"""The C-ABI library loads, exports every entry point include/mca.h declares, and its structs match
+the Python binding's layout (CPU only: no compute calls)."""
+import ctypes
+import os
+import re
+import subprocess
+import tempfile
+
+import numpy as np
+import pytest
+
+from paper_2607_08406_gb300 import mca, build as B
+from paper_2607_08406_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mca.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return mca.load_library()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(mca_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for must in ("mca_create", "mca_run", "mca_loss", "mca_get_params", "mca_destroy"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    out = subprocess.run(["nm", "-D", "--defined-only", mca.LIB_PATH], capture_output=True,
+                         text=True).stdout
+    exported = set(re.findall(r"\sT\s(mca_\w+)", out))
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        assert hasattr(lib, n)
+    assert set(mca.SIGNATURES) == set(names)
+
+
+def test_struct_layouts_match_header(tmp_path):
+    """Compile a probe against include/mca.h with gcc and compare sizes/offsets with ctypes."""
+    structs = {"mca_layer": mca.mca_layer, "mca_domain": mca.mca_domain,
+               "mca_dataset": mca.mca_dataset, "mca_options": mca.mca_options,
+               "mca_run_stats": mca.mca_run_stats, "mca_trace_rec": mca.mca_trace_rec}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"', "int main(){"]
+    for s, cls in structs.items():
+        lines.append(f'printf("{s} %zu\\n", sizeof({s}));')
+        for f, _ in cls._fields_:
+            lines.append(f'printf("{s}.{f} %zu\\n", offsetof({s}, {f}));')
+    lines.append("return 0;}")
+    c = tmp_path / "probe.c"
+    c.write_text("\n".join(lines))
+    exe = tmp_path / "probe"
+    subprocess.run(["gcc", "-O0", str(c), "-o", str(exe)], check=True)
+    got = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                 check=True).stdout.splitlines())
+    for s, cls in structs.items():
+        assert int(got[s]) == ctypes.sizeof(cls), s
+        for f, _ in cls._fields_:
+            assert int(got[f"{s}.{f}"]) == getattr(cls, f).offset, (s, f)
+
+
+def _spec(n_layers=2):
+    wl = W.mlp_small(N=8, H=4)
+    layers = wl.layers if n_layers == 2 else wl.layers[:1]
+    return wl, mca._layers(layers), len(layers)
+
+
+def test_invalid_specs_rejected_without_gpu(lib):
+    """Argument checks run on the host before any CUDA call."""
+    wl, L, n = _spec()
+    ds = mca.mca_dataset(wl.X.ctypes.data, wl.y.ctypes.data, wl.N, 784)
+    h = ctypes.c_void_p(None)
+    # one layer
+    rc = lib.mca_create(L, 1, 0, None, ctypes.byref(ds), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_INVALID and h.value is None
+    assert b"n_layers" in lib.mca_last_error(None)
+    # mismatched input width
+    bad = mca.mca_dataset(wl.X.ctypes.data, wl.y.ctypes.data, wl.N, 783)
+    rc = lib.mca_create(L, n, 0, None, ctypes.byref(bad), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_INVALID
+    # unknown loss
+    rc = lib.mca_create(L, n, 7, None, ctypes.byref(ds), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_INVALID
+    # empty dataset
+    empty = mca.mca_dataset(wl.X.ctypes.data, wl.y.ctypes.data, 0, 784)
+    rc = lib.mca_create(L, n, 0, None, ctypes.byref(empty), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_INVALID
+    # too many classes for the sample record
+    big = (mca.mca_layer * 2)(mca.mca_layer(784, 4, 1, 0.0, 0, 1.0),
+                              mca.mca_layer(4, 40, 2, 0.0, 0, 1.0))
+    rc = lib.mca_create(big, 2, 0, None, ctypes.byref(ds), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_UNSUPPORTED
+    # NULL handle calls
+    assert lib.mca_run(None, 1, 0, None) == mca.MCA_ERR_INVALID
+    lib.mca_destroy(None)
+
+
+def test_binding_names_match_c_abi():
+    """The Python binding exposes each C entry point under the same name."""
+    for n in declared_functions():
+        if n == "mca_last_error":
+            continue
+        assert callable(getattr(mca, n)), n
