@@ -104,8 +104,10 @@ typedef struct {
                               crosses a multiple of this; 0: only at creation and set_params */
   void* stream;            /* cudaStream_t; NULL = legacy default stream */
   int32_t trace_cap;       /* > 0: keep the last trace_cap trial records (mca_get_trace) */
-  int32_t grid;            /* > 0: CTAs of the trial-loop kernel (capped at what is co-resident);
-                              0: automatic */
+  int32_t grid;            /* > 0: target number of sample ranges = CTAs of the trial-loop
+                              kernel (capped at what is co-resident); 0: automatic. The ranges
+                              fix the summation order of dS, so runs with different grids agree
+                              only to rounding */
   void* workspace;         /* NULL: the library allocates its device memory itself; otherwise a
                               caller-owned device buffer of >= mca_workspace_size() bytes,
                               256-byte aligned, that must outlive the handle */
@@ -128,6 +130,8 @@ typedef struct {
                               feature's non-zeros touch + 8 B per non-zero; per output-layer
                               candidate 4 B per sample (one hidden-field row); per accepted
                               first-layer candidate the sectors written back */
+  uint64_t phase_ns[4];    /* device time of the trial loop's first CTA in: propose + evaluate,
+                              grid barrier, reduce + decide, commit */
 } mca_run_stats;
 
 typedef struct {

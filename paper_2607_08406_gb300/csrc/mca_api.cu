@@ -60,14 +60,15 @@ bool is_device_ptr(const void* p) {
 }
 
 struct Layout {
-  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, z1, srec, partial, bar, st, trace, ex_idx, ex_new, ex_out,
+  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, bar, st, trace, ex_idx, ex_new, ex_out,
       scratch, total;
   std::vector<size_t> w_eff, code, wfix;
 };
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
 
-Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long nnz, int trace_cap) {
+Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long nnz, int trace_cap,
+            int NR) {
   Layout L;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -77,13 +78,13 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   };
   const int Np = pad_n(N);
   const int H = layers[0].n_out;
-  const int maxch = (int)((std::max<long long>(N, 1) + mca::kChunk - 1) / mca::kChunk);
   L.XT = take(sizeof(float) * (size_t)D * Np);
   L.y = take(sizeof(int) * (size_t)N);
   L.xs_off = take(sizeof(int) * (size_t)(D + 1));
   L.xs_n = take(sizeof(int) * (size_t)std::max<long long>(nnz, 1));
   L.xs_v = take(sizeof(float) * (size_t)std::max<long long>(nnz, 1));
   L.xs_sect = take(sizeof(int) * (size_t)D);
+  L.xs_roff = take(sizeof(int) * (size_t)D * (NR + 1));
   for (const auto& ly : layers) {
     const size_t n = (size_t)ly.n_in * ly.n_out;
     L.w_eff.push_back(take(sizeof(float) * n));
@@ -92,7 +93,7 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   }
   L.z1 = take(sizeof(float) * (size_t)H * Np);
   L.srec = take(sizeof(float) * (size_t)mca::kSR * N);
-  L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * maxch);
+  L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
   L.bar = take(sizeof(GridBarrier));
   L.st = take(sizeof(DevState));
   L.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
@@ -194,6 +195,48 @@ mca_status count_nnz(const mca_dataset* d, cudaStream_t s, long long* nnz) {
   return MCA_OK;
 }
 
+// Sample ranges of the trial loop: one CTA per range, all CTAs co-resident. Ranges hold a multiple
+// of 8 samples (whole 32-byte sectors of a hidden-field row) and at least about kRangeTarget.
+struct Ranges {
+  int NR, RS, SUB, smem_records;
+};
+
+mca_status choose_ranges(const std::vector<mca_layer>& layers, int loss, long long N, int grid_opt,
+                         Ranges* out) {
+  int dev = 0, sms = 0;
+  CUDA_TRY(nullptr, cudaGetDevice(&dev));
+  CUDA_TRY(nullptr, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  mca::Mlp2Args probe;
+  std::memset(&probe, 0, sizeof(probe));
+  probe.act1 = layers[0].act;
+  probe.act2 = layers[1].act;
+  probe.loss = loss;
+  for (int smem_records = 1; smem_records >= 0; --smem_records) {
+    probe.smem_records = 0;
+    const int maxgrid0 = mca::mlp2_loop_max_grid(probe, sms);
+    if (maxgrid0 <= 0) return fail(nullptr, MCA_ERR_CUDA, "trial-loop kernel cannot be resident");
+    long long target = grid_opt > 0 ? grid_opt : (N + mca::kRangeTarget - 1) / mca::kRangeTarget;
+    target = std::max<long long>(1, std::min<long long>(target, maxgrid0));
+    int RS = (int)((N + target - 1) / target);
+    RS = (RS + 7) / 8 * 8;
+    const int NR = (int)((N + RS - 1) / RS);
+    int SUB = (RS + mca::kMaxSubs - 1) / mca::kMaxSubs;
+    SUB = std::max(128, (SUB + 31) / 32 * 32);
+    Ranges R{NR, RS, SUB, 0};
+    if (smem_records && (size_t)RS * mca::kSR * sizeof(float) <= (size_t)mca::kSmemRecordBytes) {
+      probe.smem_records = 1;
+      probe.RS = RS;
+      if (mca::mlp2_loop_max_grid(probe, sms) < NR) continue;
+      R.smem_records = 1;
+    } else if (smem_records) {
+      continue;
+    }
+    *out = R;
+    return MCA_OK;
+  }
+  return fail(nullptr, MCA_ERR_CUDA, "no co-resident launch shape for the trial loop");
+}
+
 mca::Mlp2Args mlp2_args(mca_handle* h) {
   mca::Mlp2Args a;
   std::memset(&a, 0, sizeof(a));
@@ -204,14 +247,17 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.H = L1.n_out;
   a.C = h->C;
   a.Np = h->Np;
-  a.CH = mca::kChunk;
-  a.maxch = h->maxch;
+  a.NR = h->NR;
+  a.RS = h->RS;
+  a.SUB = h->SUB;
+  a.smem_records = h->smem_records;
   a.P = h->P;
   a.P1 = (unsigned long long)L1.n_in * L1.n_out;
   a.xs_off = h->xs_off;
   a.xs_n = h->xs_n;
   a.xs_v = h->xs_v;
   a.xs_sect = h->xs_sect;
+  a.xs_roff = h->xs_roff;
   a.z1 = h->z1;
   a.srec = h->srec;
   a.w1 = h->w_eff[0];
@@ -317,15 +363,7 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
   s->tau = h->tau;
   s->S = d.S;
   s->alg_bytes = d.alg_bytes;
-}
-
-int auto_grid(mca_handle* h, int maxgrid) {
-  if (h->opt.grid > 0) return std::min(h->opt.grid, maxgrid);
-  const long long avg = h->nnz / std::max(1, h->D);
-  const long long per_cand = std::max<long long>(1, (avg + mca::kChunk - 1) / mca::kChunk);
-  long long g = (long long)h->opt.K * per_cand;
-  g = std::max<long long>(g, 1);
-  return (int)std::min<long long>(g, maxgrid);
+  for (int q = 0; q < 4; ++q) s->phase_ns[q] = d.phase_ns[q];
 }
 
 }  // namespace
@@ -346,7 +384,10 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
   long long nnz = 0;
   rc = count_nnz(data, (cudaStream_t)o.stream, &nnz);
   if (rc != MCA_OK) return rc;
-  *bytes = plan(ls, data->n, data->d, nnz, o.trace_cap).total;
+  Ranges R;
+  rc = choose_ranges(ls, loss, data->n, o.grid, &R);
+  if (rc != MCA_OK) return rc;
+  *bytes = plan(ls, data->n, data->d, nnz, o.trace_cap, R.NR).total;
   return MCA_OK;
 }
 
@@ -387,7 +428,6 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     P += (unsigned long long)L.n_in * L.n_out;
   }
   h->P = P;
-  h->maxch = (int)((h->N + mca::kChunk - 1) / mca::kChunk);
   h->trace_cap = o.trace_cap;
 
   auto bail = [&](mca_status st) {
@@ -419,7 +459,19 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     }
     h->nnz = nnz;
   }
-  const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap);
+  {
+    Ranges R;
+    mca_status s = choose_ranges(ls, loss, h->N, o.grid, &R);
+    if (s != MCA_OK) {
+      h->err = g_create_err;
+      return bail(s);
+    }
+    h->NR = R.NR;
+    h->RS = R.RS;
+    h->SUB = R.SUB;
+    h->smem_records = R.smem_records;
+  }
+  const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap, h->NR);
   if (o.workspace) {
     if (o.workspace_bytes < L.total)
       return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
@@ -440,6 +492,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   h->xs_n = reinterpret_cast<int*>(base + L.xs_n);
   h->xs_v = reinterpret_cast<float*>(base + L.xs_v);
   h->xs_sect = reinterpret_cast<int*>(base + L.xs_sect);
+  h->xs_roff = reinterpret_cast<int*>(base + L.xs_roff);
   for (size_t l = 0; l < ls.size(); ++l) {
     h->w_eff.push_back(reinterpret_cast<float*>(base + L.w_eff[l]));
     h->code.push_back(L.code[l] == SIZE_MAX ? nullptr
@@ -493,7 +546,9 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
                        h->stream));
   CTRY(mca::launch_csr_fill(h->XT, h->Np, (int)h->N, h->D, h->xs_off, h->xs_n, h->xs_v, h->stream));
   CTRY(mca::launch_csr_sectors(h->xs_off, h->xs_n, h->D, h->xs_sect, h->stream));
-  h->launches += 2;
+  CTRY(mca::launch_csr_range_offsets(h->xs_off, h->xs_n, h->D, h->NR, h->RS, h->xs_roff,
+                                     h->stream));
+  h->launches += 3;
   {
     std::vector<int> yh(h->N);
     CTRY(cudaMemcpyAsync(yh.data(), data->y, sizeof(int) * h->N, cudaMemcpyDefault, h->stream));
@@ -510,12 +565,6 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   DevState ds;
   TRY(read_state(h, &ds));
   if (!std::isfinite(ds.S)) return bail(fail(h, MCA_ERR_NUMERIC, "initial loss is not finite"));
-  {
-    mca::Mlp2Args a = mlp2_args(h);
-    const int maxgrid = mca::mlp2_loop_max_grid(a, h->num_sms);
-    if (maxgrid <= 0) return bail(fail(h, MCA_ERR_CUDA, "trial-loop kernel cannot be resident"));
-    h->grid = auto_grid(h, maxgrid);
-  }
 #undef TRY
 #undef CTRY
   *out = h;
@@ -535,7 +584,7 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     a.tau0 = h->tau;
     a.n_trials = seg;
     CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
-    CUDA_TRY(h, mca::launch_mlp2_loop(a, h->grid, h->stream));
+    CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
     h->launches++;
     h->tau += seg;
     remaining -= seg;
@@ -690,7 +739,7 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
   a.ex_new = h->ex_new;
   a.ex_out = h->ex_out;
   CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
-  CUDA_TRY(h, mca::launch_mlp2_loop(a, h->grid, h->stream));
+  CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
   h->launches++;
   CUDA_TRY(h, cudaMemcpyAsync(dS, h->ex_out, sizeof(double) * n, cudaMemcpyDeviceToHost,
                               h->stream));

@@ -202,4 +202,37 @@ __device__ __forceinline__ bool grid_sync(GridBarrier* bar, unsigned int nblocks
   return ok;
 }
 
+// ------------------------------------------------------------------------------------------------
+// Sample records: 16 floats per sample -- output fields [0, C), the sample's loss at 14, its label
+// (int bits) at 15. Works on shared or global memory.
+// ------------------------------------------------------------------------------------------------
+// Load one sample record: fields into z[0..M), loss and label. Record slots M..13 are padding.
+template <int M>
+__device__ __forceinline__ void load_srec(const float* srec, int n, float (&z)[M], float& ell,
+                                          int& y) {
+  static_assert(M <= 14, "at most 14 output fields per sample record");
+  const float4* p = reinterpret_cast<const float4*>(srec + (size_t)n * 16);
+  const float4 v0 = p[0], v1 = p[1], v2 = p[2], v3 = p[3];
+  const float f[16] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w,
+                       v2.x, v2.y, v2.z, v2.w, v3.x, v3.y, v3.z, v3.w};
+#pragma unroll
+  for (int k = 0; k < M; ++k) z[k] = f[k];
+  ell = v3.z;
+  y = __float_as_int(v3.w);
+}
+
+template <int M>
+__device__ __forceinline__ void store_srec(float* srec, int n, const float (&z)[M], float ell,
+                                           int y) {
+  static_assert(M <= 14, "at most 14 output fields per sample record");
+  float f[16];
+#pragma unroll
+  for (int k = 0; k < 14; ++k) f[k] = k < M ? z[k] : 0.0f;
+  float4* p = reinterpret_cast<float4*>(srec + (size_t)n * 16);
+  p[0] = make_float4(f[0], f[1], f[2], f[3]);
+  p[1] = make_float4(f[4], f[5], f[6], f[7]);
+  p[2] = make_float4(f[8], f[9], f[10], f[11]);
+  p[3] = make_float4(f[12], f[13], ell, __int_as_float(y));
+}
+
 }  // namespace mca

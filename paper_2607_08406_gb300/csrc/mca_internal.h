@@ -14,30 +14,37 @@ namespace mca {
 struct GridBarrier;
 
 constexpr int kKmax = 128;        // speculative candidates per batch
-constexpr int kMaxC = 16;         // register arrays of the output layer
+constexpr int kMaxC = 14;         // output fields a sample record holds
 constexpr int kSR = 16;           // floats per sample record: fields [0, C), loss at 14, label at 15
 constexpr int kMaxClasses = kSR - 2;
 constexpr int kLoopThreads = 512; // threads per CTA of the trial-loop kernel
-constexpr int kPerThread = 4;     // entries per thread per chunk
-constexpr int kChunk = kLoopThreads * kPerThread;   // entries per work item (fixed partition)
+constexpr int kLoopWarps = kLoopThreads / 32;
+constexpr int kMaxSubs = 8;       // sub-chunks of one candidate inside one sample range
+constexpr int kRangeTarget = 64;  // samples per range below which fewer CTAs are used
+constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
 
 // Device-resident run state (one per handle).
 struct DevState {
   double S;                  // loss sum of the cached state
   unsigned long long trials, accepts, candidates, batches, wasted, forced, trace_written;
   unsigned long long alg_bytes;  // compulsory DRAM bytes of the evaluated candidates and commits
+  unsigned long long phase_ns[4];  // CTA 0: propose+evaluate, barrier, reduce+decide, commit
   int err;                   // first device-side error (mca_status), 0 = none
   int pad;
 };
 
-// Arguments of the two-layer trial loop (input -> hidden -> output).
+// Arguments of the two-layer trial loop (input -> hidden -> output). The samples are split into NR
+// contiguous ranges of RS samples (RS a multiple of 8); CTA r owns range r.
 struct Mlp2Args {
-  int N, D, H, C, Np, CH, maxch;
+  int N, D, H, C, Np;
+  int NR, RS, SUB;           // ranges, samples per range, entries per sub-chunk (multiple of 32)
+  int smem_records;          // 1: each CTA keeps its range's sample records in shared memory
   unsigned long long P, P1;
   const int* xs_off;         // [D + 1] CSR of X by feature: entries of feature i in [off[i], off[i+1])
   const int* xs_n;           // [nnz] sample index of each entry (ascending inside a feature)
   const float* xs_v;         // [nnz] value x[n, i] != 0
   const int* xs_sect;        // [D] 32-byte sectors of a z1 row that feature i's entries touch
+  const int* xs_roff;        // [D x (NR + 1)] first entry of feature i in range r
   float* z1;                 // [H x Np] hidden fields, feature-major
   float* srec;               // [N x kSR] output fields, loss, label
   float* w1;                 // [H x D] effective weights
@@ -56,7 +63,7 @@ struct Mlp2Args {
   int strict;
   unsigned long long seed, tau0, n_trials;
   int K;
-  float* partial;            // [2 x kKmax x maxch]
+  float* partial;            // [2 x kKmax x NR] per-candidate, per-range loss changes
   GridBarrier* bar;
   DevState* st;
   mca_trace_rec* trace;
@@ -76,6 +83,8 @@ cudaError_t launch_csr_count(const float* XT, int Np, int N, int D, int* cnt, cu
 cudaError_t launch_csr_fill(const float* XT, int Np, int N, int D, const int* off, int* xs_n,
                             float* xs_v, cudaStream_t s);
 cudaError_t launch_csr_sectors(const int* off, const int* xs_n, int D, int* sect, cudaStream_t s);
+cudaError_t launch_csr_range_offsets(const int* off, const int* xs_n, int D, int NR, int RS,
+                                     int* roff, cudaStream_t s);
 cudaError_t launch_count_nonfinite(const float* p, size_t n, int* out, cudaStream_t s);
 cudaError_t launch_init_layer(int wkind, float scale, const float* src, const signed char* mask,
                               size_t n, float* w_eff, signed char* code, float* wfix,
@@ -84,9 +93,10 @@ cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, con
                             int ldb, float* C, int ldc, cudaStream_t s);
 cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s);
 cudaError_t launch_sum_loss(const float* srec, int N, DevState* st, cudaStream_t s);
-// Cooperative persistent trial loop; grid <= co-resident CTAs.
-cudaError_t launch_mlp2_loop(const Mlp2Args& a, int grid, cudaStream_t s);
+// Cooperative persistent trial loop, one CTA per sample range (grid = NR).
+cudaError_t launch_mlp2_loop(const Mlp2Args& a, cudaStream_t s);
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);
+size_t mlp2_loop_smem_bytes(const Mlp2Args& a);
 
 }  // namespace mca
 
@@ -112,6 +122,7 @@ struct mca_handle {
   int* xs_n = nullptr;
   float* xs_v = nullptr;
   int* xs_sect = nullptr;
+  int* xs_roff = nullptr;
   long long nnz = 0;
   int max_nnz = 0;
   std::vector<float*> w_eff;
@@ -120,7 +131,7 @@ struct mca_handle {
   float* z1 = nullptr;
   float* srec = nullptr;
   float* partial = nullptr;
-  int maxch = 0;
+  int NR = 0, RS = 0, SUB = 0, smem_records = 0;
   mca::GridBarrier* bar = nullptr;
   mca::DevState* st = nullptr;
   mca_trace_rec* trace = nullptr;
@@ -135,6 +146,5 @@ struct mca_handle {
   // host-side counters
   unsigned long long tau = 0;
   unsigned long long launches = 0, resyncs = 0;
-  int grid = 0;
   bool broken = false;                   // a sticky CUDA error or device timeout was seen
 };

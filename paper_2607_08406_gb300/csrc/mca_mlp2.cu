@@ -1,24 +1,27 @@
-// Kernels of the single-hidden-layer MCA path (input -> hidden -> output), Section 2.4.
+// Trial loop of the single-hidden-layer MCA path (input -> hidden -> output), Section 2.4, as one
+// persistent cooperative kernel.
 //
-// Cached state (feature-major so that a mutated neuron's field row is contiguous):
+// Cached state (feature-major, so that a mutated neuron's field row is contiguous):
 //   z1   [H x Np]   hidden local fields z1[j, n] = sum_i W1[j, i] x[n, i]
 //   srec [N x 16]   per sample: output fields z2[0..C), the sample's loss, its label
-//   X    CSR by feature: the non-zero entries x[n, i] of each input feature i, ascending n
+//   X    CSR by input feature: the non-zero entries x[n, i] of feature i, ascending n
 //
-// One trial = one candidate (Eq. 1). A mutation of W1[j, i] changes z1[j, n] by delta * x[n, i]
-// only where x[n, i] != 0 (a rank-1 update restricted to feature i's non-zeros), and the output
-// fields by W2[:, j] times the hidden activation change (Section 2.4). A mutation of W2[o, j]
-// changes z2[o, n] by delta * f(z1[j, n]) for every sample.
+// A mutation of W1[j, i] changes z1[j, n] by delta * x[n, i] only where x[n, i] != 0 (a rank-1
+// update restricted to feature i's non-zeros) and the output fields by W2[:, j] times neuron j's
+// activation change. A mutation of W2[o, j] changes z2[o, n] by delta * f(z1[j, n]) for every n.
 //
-// The trial loop is one persistent cooperative kernel. Per batch of K candidates:
-//   propose   every CTA draws all K proposals itself (Philox, no communication)
-//   evaluate  work items = fixed chunks of kChunk entries of each candidate; each item's partial
-//             loss change goes to its own slot (no atomics), so dS_k does not depend on K or grid
-//   barrier
-//   decide    every CTA sums each candidate's chunk partials in the same fixed order and takes
-//             the lowest-index candidate with dS <= 0 (Eq. 6) -- the same answer everywhere
-//   commit    only if one was accepted: its chunks rewrite z1 row j and the touched sample
-//             records; CTA 0 writes the weight, S, statistics and trace; then a second barrier.
+// Work split: the samples are cut into NR contiguous ranges and CTA r owns range r for the whole
+// launch -- it is the only CTA that reads or writes z1[:, n] and srec[n] for n in its range, and it
+// keeps the range's sample records in shared memory. Per batch of K candidates:
+//   propose   every CTA draws all K proposals itself (Philox; no communication)
+//   evaluate  each CTA sums l' - l over its own samples for every candidate, in fixed sub-chunks
+//             (warp per sub-chunk, fixed lane order), and writes one partial per (candidate, range)
+//   barrier   the only grid-wide synchronisation of a batch
+//   decide    every CTA sums each candidate's NR partials in the same fixed order and takes the
+//             lowest-index candidate with dS <= 0 (Eq. 6): the same answer in every CTA
+//   commit    each CTA applies the accepted candidate to its own samples (no barrier needed: no
+//             other CTA reads them) and writes the new weight value (the same value from all CTAs)
+// Every partial depends only on (candidate, range), so dS and the trajectory do not depend on K.
 #include <algorithm>
 #include <cstdio>
 
@@ -28,16 +31,20 @@
 namespace mca {
 
 struct Cand {
+  unsigned long long bytes;  // compulsory DRAM bytes of evaluating this candidate (statistics)
   unsigned int idx;
   int layer, row, col;
   float oldw, neww, delta;
   int new_code;
   int valid;
-  int start, cnt, nch;
+  int gcnt;                  // entries over all samples; 0: nothing changes, dS = 0 exactly
+  int ebeg, ecnt;            // this CTA's segment (CSR entries, or samples of the range)
+  int sub0, nsub;            // this CTA's sub-chunks
 };
 
 __device__ __forceinline__ void fill_candidate(const Mlp2Args& a, unsigned int idx, uint32_t r1,
-                                               bool explicit_value, float ex_new, Cand& c) {
+                                               bool explicit_value, float ex_new, int r, int s0,
+                                               int s1, Cand& c) {
   const int layer = (unsigned long long)idx >= a.P1 ? 1 : 0;
   const unsigned long long off = idx - (layer ? a.P1 : 0ull);
   const int n_in = layer ? a.H : a.D;
@@ -79,608 +86,443 @@ __device__ __forceinline__ void fill_candidate(const Mlp2Args& a, unsigned int i
     if (a.bound > 0.0f && !(fabsf(c.neww) < a.bound)) c.valid = 0;
   }
   c.delta = __fsub_rn(c.neww, c.oldw);
-  if (layer == 0) {
-    c.start = a.xs_off[c.col];
-    c.cnt = a.xs_off[c.col + 1] - c.start;
-  } else {
-    c.start = 0;
-    c.cnt = a.N;
-  }
+  const int all = layer == 0 ? a.xs_off[c.col + 1] - a.xs_off[c.col] : a.N;
   // A zero change leaves every field bit-identical: dS = 0 exactly, nothing to evaluate.
-  c.nch = (c.valid && c.delta != 0.0f) ? (c.cnt + a.CH - 1) / a.CH : 0;
-}
-
-// Load one sample record: fields into z[0..C), loss and label.
-__device__ __forceinline__ void load_srec(const float* srec, int n, float (&z)[kMaxC], float& ell,
-                                          int& y) {
-  const float4* p = reinterpret_cast<const float4*>(srec + (size_t)n * kSR);
-  const float4 v0 = p[0], v1 = p[1], v2 = p[2], v3 = p[3];
-  z[0] = v0.x; z[1] = v0.y; z[2] = v0.z; z[3] = v0.w;
-  z[4] = v1.x; z[5] = v1.y; z[6] = v1.z; z[7] = v1.w;
-  z[8] = v2.x; z[9] = v2.y; z[10] = v2.z; z[11] = v2.w;
-  z[12] = v3.x; z[13] = v3.y;
-  z[14] = 0.0f; z[15] = 0.0f;
-  ell = v3.z;
-  y = __float_as_int(v3.w);
-}
-
-__device__ __forceinline__ void store_srec(float* srec, int n, const float (&z)[kMaxC], float ell,
-                                           int y) {
-  float4* p = reinterpret_cast<float4*>(srec + (size_t)n * kSR);
-  p[0] = make_float4(z[0], z[1], z[2], z[3]);
-  p[1] = make_float4(z[4], z[5], z[6], z[7]);
-  p[2] = make_float4(z[8], z[9], z[10], z[11]);
-  p[3] = make_float4(z[12], z[13], ell, __int_as_float(y));
-}
-
-// Chunk `chunk` of a first-layer candidate: entries [start + chunk*CH, ...) of feature col.
-// Returns this thread's share of sum(l' - l). COMMIT: also write the new fields and losses.
-template <int ACT1, int ACT2, int LOSS, bool COMMIT>
-__device__ __forceinline__ float l1_chunk(const Mlp2Args& a, const Cand& c, const float* w2c,
-                                          int chunk) {
-  const int e0 = c.start + chunk * a.CH;
-  const int e1 = min(e0 + a.CH, c.start + c.cnt);
-  float* zrow = a.z1 + (size_t)c.row * a.Np;
-  int nn[kPerThread];
-  float xv[kPerThread], zv[kPerThread];
-#pragma unroll
-  for (int r = 0; r < kPerThread; ++r) {
-    const int e = e0 + threadIdx.x + r * kLoopThreads;
-    nn[r] = -1;
-    if (e < e1) {
-      nn[r] = __ldg(a.xs_n + e);
-      xv[r] = __ldg(a.xs_v + e);
+  c.gcnt = (c.valid && c.delta != 0.0f) ? all : 0;
+  c.bytes = 0ull;
+  c.ebeg = 0;
+  c.ecnt = 0;
+  if (c.gcnt > 0) {
+    if (layer == 0) {
+      const int* ro = a.xs_roff + (size_t)c.col * (a.NR + 1) + r;
+      c.ebeg = ro[0];
+      c.ecnt = ro[1] - ro[0];
+      c.bytes = 32ull * (unsigned long long)a.xs_sect[c.col] + 8ull * (unsigned long long)all;
+    } else {
+      c.ecnt = s1 - s0;
+      c.bytes = 4ull * (unsigned long long)a.N;
     }
   }
+  c.nsub = (c.ecnt + a.SUB - 1) / a.SUB;
+}
+
+// One entry of a first-layer candidate: range-local sample nl with input value x and cached field
+// z. Returns l' - l; COMMIT also writes the new hidden field (*zp) and sample record.
+template <int ACT1, int ACT2, int LOSS, int NC, bool COMMIT>
+__device__ __forceinline__ float entry_l1(const Mlp2Args& a, float* sr, const Cand& c,
+                                          const float* w2c, int nl, float x, float z, float* zp) {
+  const float zn = fmaf(c.delta, x, z);
+  const float da = act<ACT1>(zn, a.g1, a.act1) - act<ACT1>(z, a.g1, a.act1);
+  if (COMMIT) *zp = zn;
+  if (da == 0.0f) return 0.0f;
+  constexpr int M = NC > 0 ? NC : kMaxC;
+  const int C = NC > 0 ? NC : a.C;
+  float zz[M];
+  float ell;
+  int y;
+  load_srec(sr, nl, zz, ell, y);
 #pragma unroll
-  for (int r = 0; r < kPerThread; ++r) zv[r] = nn[r] >= 0 ? zrow[nn[r]] : 0.0f;
+  for (int k = 0; k < M; ++k)
+    if (k < C) zz[k] = fmaf(w2c[k], da, zz[k]);
+  const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
+  if (COMMIT) store_srec(sr, nl, zz, ln, y);
+  return ln - ell;
+}
+
+// One sample of an output-layer candidate W2[o, j] (o = c.row, j = c.col), cached field z1[j, n].
+template <int ACT1, int ACT2, int LOSS, int NC, bool COMMIT>
+__device__ __forceinline__ float entry_l2(const Mlp2Args& a, float* sr, const Cand& c, int nl,
+                                          float z) {
+  constexpr int M = NC > 0 ? NC : kMaxC;
+  const int C = NC > 0 ? NC : a.C;
+  const float av = act<ACT1>(z, a.g1, a.act1);
+  float zz[M];
+  float ell;
+  int y;
+  load_srec(sr, nl, zz, ell, y);
+  float zo = 0.0f;
+#pragma unroll
+  for (int k = 0; k < M; ++k)
+    if (k == c.row) zo = zz[k];
+  const float zon = fmaf(c.delta, av, zo);
+  if (zon == zo) return 0.0f;
+#pragma unroll
+  for (int k = 0; k < M; ++k)
+    if (k == c.row) zz[k] = zon;
+  const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
+  if (COMMIT) store_srec(sr, nl, zz, ln, y);
+  return ln - ell;
+}
+
+// Warp-level sum of l' - l over sub-chunk q of candidate c's segment in this CTA's range. Lane l
+// takes entries l, l + 32, ... of the sub-chunk in ascending order (four at a time, loads first).
+template <int ACT1, int ACT2, int LOSS, int NC>
+__device__ __forceinline__ float eval_sub(const Mlp2Args& a, float* sr, int s0, const Cand& c,
+                                          const float* w2c, int q) {
+  const int lane = threadIdx.x & 31;
+  const int e_lo = q * a.SUB;
+  const int e_hi = min(e_lo + a.SUB, c.ecnt);
+  const float* zrow = a.z1 + (size_t)(c.layer == 0 ? c.row : c.col) * a.Np;
   float acc = 0.0f;
+  for (int g = e_lo; g < e_hi; g += 128) {
+    int nn[4];
+    float xv[4], zv[4];
 #pragma unroll
-  for (int r = 0; r < kPerThread; ++r) {
-    if (nn[r] < 0) continue;
-    const float zn = fmaf(c.delta, xv[r], zv[r]);
-    const float da = act<ACT1>(zn, a.g1, a.act1) - act<ACT1>(zv[r], a.g1, a.act1);
-    if (COMMIT) zrow[nn[r]] = zn;
-    if (da != 0.0f) {
-      float z[kMaxC];
-      float ell;
-      int y;
-      load_srec(a.srec, nn[r], z, ell, y);
+    for (int t = 0; t < 4; ++t) {
+      const int e = g + t * 32 + lane;
+      nn[t] = -1;
+      xv[t] = 0.0f;
+      if (e < e_hi) {
+        if (c.layer == 0) {
+          nn[t] = __ldg(a.xs_n + c.ebeg + e);
+          xv[t] = __ldg(a.xs_v + c.ebeg + e);
+        } else {
+          nn[t] = s0 + e;
+        }
+      }
+    }
 #pragma unroll
-      for (int k = 0; k < kMaxC; ++k)
-        if (k < a.C) z[k] = fmaf(w2c[k], da, z[k]);
-      const float ln = sample_loss<ACT2, LOSS, kMaxC>(z, a.C, y, a.g2, a.act2, a.loss);
-      acc += ln - ell;
-      if (COMMIT) store_srec(a.srec, nn[r], z, ln, y);
+    for (int t = 0; t < 4; ++t) zv[t] = nn[t] >= 0 ? zrow[nn[t]] : 0.0f;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      if (nn[t] < 0) continue;
+      if (c.layer == 0)
+        acc += entry_l1<ACT1, ACT2, LOSS, NC, false>(a, sr, c, w2c, nn[t] - s0, xv[t], zv[t],
+                                                     nullptr);
+      else
+        acc += entry_l2<ACT1, ACT2, LOSS, NC, false>(a, sr, c, nn[t] - s0, zv[t]);
     }
   }
-  return acc;
+  return warp_sum(acc);
 }
 
-// Chunk of an output-layer candidate W2[o, j]: samples [chunk*CH, ...).
-template <int ACT1, int ACT2, int LOSS, bool COMMIT>
-__device__ __forceinline__ float l2_chunk(const Mlp2Args& a, const Cand& c, int chunk) {
-  const int n0 = chunk * a.CH;
-  const int n1 = min(n0 + a.CH, a.N);
-  const float* zrow = a.z1 + (size_t)c.col * a.Np;
-  const int o = c.row;
-  float zv[kPerThread];
-#pragma unroll
-  for (int r = 0; r < kPerThread; ++r) {
-    const int n = n0 + threadIdx.x + r * kLoopThreads;
-    zv[r] = n < n1 ? zrow[n] : 0.0f;
-  }
-  float acc = 0.0f;
-#pragma unroll
-  for (int r = 0; r < kPerThread; ++r) {
-    const int n = n0 + threadIdx.x + r * kLoopThreads;
-    if (n >= n1) continue;
-    const float av = act<ACT1>(zv[r], a.g1, a.act1);
-    float z[kMaxC];
-    float ell;
-    int y;
-    load_srec(a.srec, n, z, ell, y);
-    float zo = 0.0f;
-#pragma unroll
-    for (int k = 0; k < kMaxC; ++k)
-      if (k == o) zo = z[k];
-    const float zon = fmaf(c.delta, av, zo);
-    if (zon != zo) {
-#pragma unroll
-      for (int k = 0; k < kMaxC; ++k)
-        if (k == o) z[k] = zon;
-      const float ln = sample_loss<ACT2, LOSS, kMaxC>(z, a.C, y, a.g2, a.act2, a.loss);
-      acc += ln - ell;
-      if (COMMIT) store_srec(a.srec, n, z, ln, y);
-    }
-  }
-  return acc;
-}
-
-template <int ACT1, int ACT2, int LOSS>
+template <int ACT1, int ACT2, int LOSS, int NC>
 __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
+  extern __shared__ __align__(16) float s_records[];
   __shared__ Cand s_c[kKmax];
   __shared__ float s_w2c[kKmax][kMaxC];
-  __shared__ int s_pre[kKmax + 1];
+  __shared__ float s_sub[kKmax * kMaxSubs];
   __shared__ double s_dS[kKmax];
-  __shared__ float s_red[32];
-  __shared__ int s_flag, s_kstar;
+  __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
+  __shared__ int s_flag, s_kstar, s_total;
 
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int r = blockIdx.x;
+  const int s0 = min(r * a.RS, a.N), s1 = min(s0 + a.RS, a.N);
+  const bool explicit_mode = a.n_explicit > 0;
+  float* sr = a.smem_records ? s_records : a.srec + (size_t)s0 * kSR;
+  if (a.smem_records) {
+    const float4* src = reinterpret_cast<const float4*>(a.srec + (size_t)s0 * kSR);
+    float4* dst = reinterpret_cast<float4*>(s_records);
+    for (int t = tid; t < (s1 - s0) * (kSR / 4); t += kLoopThreads) dst[t] = src[t];
+  }
+
+  // CTA 0, thread 0 carries the run statistics in registers for the whole launch.
+  DevState* st = a.st;
+  const bool stats_thread = r == 0 && tid == 0;
+  double S = 0.0;
+  unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
+                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0;
+  if (stats_thread) {
+    S = st->S;
+    n_trace = st->trace_written;
+  }
   unsigned int gen = 0;
   unsigned long long tau = a.tau0;
   const unsigned long long end = a.tau0 + a.n_trials;
-  const bool explicit_mode = a.n_explicit > 0;
-  int fcur = 0;
-  if (threadIdx.x == 0)
-    while (fcur < a.nforce && a.ftau[fcur] < tau) ++fcur;
   int buf = 0;
-  const size_t pstride = (size_t)kKmax * a.maxch;
+  __syncthreads();
 
   while (explicit_mode || tau < end) {
+    const unsigned long long t_a = stats_thread ? globaltimer_ns() : 0ull;
     const int Kb = explicit_mode ? a.n_explicit
                                  : (int)((end - tau) < (unsigned long long)a.K ? (end - tau) : a.K);
-    // ---- propose (every CTA, redundantly)
-    for (int k = threadIdx.x; k < Kb; k += blockDim.x) {
+    // ---- propose: every CTA draws every candidate
+    for (int k = tid; k < Kb; k += kLoopThreads) {
       Cand c;
       if (explicit_mode) {
-        fill_candidate(a, a.ex_idx[k], 0u, true, a.ex_new[k], c);
+        fill_candidate(a, a.ex_idx[k], 0u, true, a.ex_new[k], r, s0, s1, c);
       } else {
-        const uint4 r = trial_words(a.seed, tau + (unsigned long long)k);
-        const unsigned int idx = (unsigned int)(((unsigned long long)r.x * a.P) >> 32);
-        fill_candidate(a, idx, r.y, false, 0.0f, c);
+        const uint4 w = trial_words(a.seed, tau + (unsigned long long)k);
+        const unsigned int idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
+        fill_candidate(a, idx, w.y, false, 0.0f, r, s0, s1, c);
       }
-      s_c[k] = c;
-      if (c.layer == 0) {
+      if (c.layer == 0 && c.gcnt > 0) {
 #pragma unroll
         for (int q = 0; q < kMaxC; ++q)
           s_w2c[k][q] = q < a.C ? a.w2[(size_t)q * a.H + c.row] : 0.0f;
       }
+      s_c[k] = c;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int t = 0;
-      for (int k = 0; k < Kb; ++k) {
-        s_pre[k] = t;
-        t += s_c[k].nch;
+    if (warp == 0) {                 // exclusive scan of the sub-chunk counts
+      int v[4], loc = 0;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int k = lane * 4 + t;
+        v[t] = k < Kb ? s_c[k].nsub : 0;
+        loc += v[t];
       }
-      s_pre[Kb] = t;
+      int inc = loc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      int ex = inc - loc;
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int k = lane * 4 + t;
+        if (k < Kb) s_c[k].sub0 = ex;
+        ex += v[t];
+      }
+      if (lane == 31) s_total = inc;
     }
     __syncthreads();
-    const int total = s_pre[Kb];
-    float* part = a.partial + (size_t)buf * pstride;
 
-    // ---- evaluate: items blockIdx.x, blockIdx.x + gridDim.x, ...
-    int k = 0;
-    for (int it = blockIdx.x; it < total; it += gridDim.x) {
-      while (s_pre[k + 1] <= it) ++k;
-      const int ch = it - s_pre[k];
-      const Cand& c = s_c[k];
-      float v = c.layer == 0 ? l1_chunk<ACT1, ACT2, LOSS, false>(a, c, s_w2c[k], ch)
-                             : l2_chunk<ACT1, ACT2, LOSS, false>(a, c, ch);
-      v = block_sum(v, s_red);
-      if (threadIdx.x == 0) part[(size_t)k * a.maxch + ch] = v;
+    // ---- evaluate this CTA's samples: warp per sub-chunk
+    {
+      const int total = s_total;
+      int k = 0;
+      for (int it = warp; it < total; it += kLoopWarps) {
+        while (s_c[k].sub0 + s_c[k].nsub <= it) ++k;
+        const float v =
+            eval_sub<ACT1, ACT2, LOSS, NC>(a, sr, s0, s_c[k], s_w2c[k], it - s_c[k].sub0);
+        if (lane == 0) s_sub[it] = v;
+      }
     }
-    if (!grid_sync(a.bar, gridDim.x, gen, &a.st->err, &s_flag)) return;
+    __syncthreads();
+    float* part = a.partial + (size_t)buf * kKmax * a.NR;
+    for (int k = tid; k < Kb; k += kLoopThreads) {
+      float s = 0.0f;
+      const int b = s_c[k].sub0, nb = s_c[k].nsub;
+      for (int q = 0; q < nb; ++q) s += s_sub[b + q];
+      part[(size_t)k * a.NR + r] = s;
+    }
+    const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
+    if (!grid_sync(a.bar, gridDim.x, gen, &st->err, &s_flag)) break;
+    const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
 
-    // ---- per-candidate loss change, fixed order over chunks
-    for (int kk = threadIdx.x; kk < Kb; kk += blockDim.x) {
-      double s = 0.0;
-      const int nch = s_c[kk].nch;
-      for (int ch = 0; ch < nch; ++ch) s += (double)part[(size_t)kk * a.maxch + ch];
-      s_dS[kk] = s_c[kk].valid ? s : __longlong_as_double(0x7ff8000000000000ll);
+    // ---- dS of every candidate: the NR partials in a fixed order (lane-strided, fp64)
+    for (int k = warp; k < Kb; k += kLoopWarps) {
+      double d = 0.0;
+      if (s_c[k].gcnt > 0)
+        for (int q = lane; q < a.NR; q += 32) d += (double)part[(size_t)k * a.NR + q];
+      d = warp_sum_d(d);
+      if (lane == 0) s_dS[k] = s_c[k].valid ? d : __longlong_as_double(0x7ff8000000000000ll);
     }
     __syncthreads();
     if (explicit_mode) {
-      if (blockIdx.x == 0)
-        for (int kk = threadIdx.x; kk < Kb; kk += blockDim.x) a.ex_out[kk] = s_dS[kk];
-      return;
+      if (r == 0)
+        for (int k = tid; k < Kb; k += kLoopThreads) a.ex_out[k] = s_dS[k];
+      break;
     }
 
-    // ---- decide (identical in every CTA): lowest-index candidate with dS <= 0 (Eq. 6)
-    if (threadIdx.x == 0) {
-      int kstar = -1, nonfinite = 0, forced_here = 0;
-      for (int kk = 0; kk < Kb; ++kk) {
-        const unsigned long long tk = tau + (unsigned long long)kk;
-        while (fcur < a.nforce && a.ftau[fcur] < tk) ++fcur;
-        const bool forced = fcur < a.nforce && a.ftau[fcur] == tk;
-        const double d = s_dS[kk];
-        bool acc;
-        if (!s_c[kk].valid) {
-          acc = false;
-        } else if (forced) {
-          acc = a.facc[fcur] != 0;
-          forced_here++;
+    // ---- decide (the same in every CTA): lowest-index candidate with dS <= 0 (Eq. 6)
+    if (warp < kKmax / 32) {
+      bool acc = false, bad = false, forced = false;
+      const int k = tid;
+      if (k < Kb && s_c[k].valid) {
+        const unsigned long long tk = tau + (unsigned long long)k;
+        bool facc = false;
+        if (a.nforce > 0) {          // binary search of the forced-decision list
+          int lo = 0, hi = a.nforce;
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (a.ftau[mid] < tk)
+              lo = mid + 1;
+            else
+              hi = mid;
+          }
+          if (lo < a.nforce && a.ftau[lo] == tk) {
+            forced = true;
+            facc = a.facc[lo] != 0;
+          }
+        }
+        const double d = s_dS[k];
+        if (forced) {
+          acc = facc;
         } else {
-          if (!isfinite(d)) nonfinite = 1;
+          bad = !isfinite(d);
           acc = a.strict ? (d < 0.0) : (d <= 0.0);
         }
-        if (blockIdx.x == 0 && a.trace_cap > 0) {
-          const unsigned long long slot = a.st->trace_written % (unsigned long long)a.trace_cap;
-          mca_trace_rec rec;
-          rec.tau = tk;
-          rec.idx = s_c[kk].idx;
-          rec.accept = acc ? 1 : 0;
-          rec.old_w = s_c[kk].oldw;
-          rec.new_w = s_c[kk].neww;
-          rec.valid = s_c[kk].valid;
-          rec.forced = forced ? 1 : 0;
-          rec.dS = d;
-          rec.S = a.st->S;
-          a.trace[slot] = rec;
-          a.st->trace_written += 1ull;
-        }
-        if (acc) {
-          kstar = kk;
-          break;
-        }
       }
-      s_kstar = nonfinite ? -2 : kstar;
-      if (blockIdx.x == 0) {
-        DevState* st = a.st;
-        st->batches += 1ull;
-        st->forced += (unsigned long long)forced_here;
-        // compulsory DRAM bytes: per evaluated first-layer candidate the z1 sectors its feature's
-        // entries touch plus the entries (index + value); per output-layer candidate one z1 row
-        unsigned long long bytes = 0ull;
-        for (int kk = 0; kk < Kb; ++kk) {
-          const Cand& c = s_c[kk];
-          st->candidates += c.valid ? 1ull : 0ull;
-          if (c.nch > 0)
-            bytes += c.layer == 0 ? 32ull * (unsigned long long)a.xs_sect[c.col] + 8ull * c.cnt
-                                  : 4ull * (unsigned long long)a.N;
+      const unsigned int ma = __ballot_sync(0xffffffffu, acc);
+      const unsigned int mb = __ballot_sync(0xffffffffu, bad);
+      const unsigned int mf = __ballot_sync(0xffffffffu, forced);
+      if (lane == 0) {
+        s_macc[warp] = ma;
+        s_mbad[warp] = mb;
+        s_mforced[warp] = mf;
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int kstar = -1, kbad = -1;
+      for (int w = 0; w < kKmax / 32 && kstar < 0; ++w)
+        if (s_macc[w]) kstar = w * 32 + __ffs(s_macc[w]) - 1;
+      for (int w = 0; w < kKmax / 32 && kbad < 0; ++w)
+        if (s_mbad[w]) kbad = w * 32 + __ffs(s_mbad[w]) - 1;
+      if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
+      s_kstar = kstar;
+      if (stats_thread) {
+        const int last = kstar >= 0 ? kstar : Kb - 1;
+        if (a.trace_cap > 0) {
+          for (int k = 0; k <= last; ++k) {
+            mca_trace_rec rec;
+            rec.tau = tau + (unsigned long long)k;
+            rec.idx = s_c[k].idx;
+            rec.accept = k == kstar ? 1 : 0;
+            rec.old_w = s_c[k].oldw;
+            rec.new_w = s_c[k].neww;
+            rec.valid = s_c[k].valid;
+            rec.forced = (int)((s_mforced[k >> 5] >> (k & 31)) & 1u);
+            rec.dS = s_dS[k];
+            rec.S = S;
+            a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
+            ++n_trace;
+          }
         }
-        if (kstar >= 0 && s_c[kstar].nch > 0 && s_c[kstar].layer == 0)
-          bytes += 32ull * (unsigned long long)a.xs_sect[s_c[kstar].col];   // z1 write-back
-        st->alg_bytes += bytes;
+        for (int w = 0; w < kKmax / 32; ++w) {
+          unsigned int m = s_mforced[w];
+          const int hi = last - w * 32;
+          if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
+          n_forced += (unsigned long long)__popc(m);
+        }
+        for (int k = 0; k < Kb; ++k) {
+          n_cand += s_c[k].valid ? 1ull : 0ull;
+          n_bytes += s_c[k].bytes;
+        }
+        ++n_batch;
         if (kstar >= 0) {
-          st->trials += (unsigned long long)(kstar + 1);
-          st->accepts += 1ull;
-          st->wasted += (unsigned long long)(Kb - kstar - 1);
-          st->S += s_dS[kstar] == s_dS[kstar] ? s_dS[kstar] : 0.0;
-        } else {
-          st->trials += (unsigned long long)Kb;
+          n_trials += (unsigned long long)(kstar + 1);
+          ++n_acc;
+          n_waste += (unsigned long long)(Kb - kstar - 1);
+          S += s_dS[kstar];
+          if (s_c[kstar].layer == 0 && s_c[kstar].gcnt > 0)
+            n_bytes += 32ull * (unsigned long long)a.xs_sect[s_c[kstar].col];
+        } else if (kstar == -1) {
+          n_trials += (unsigned long long)Kb;
         }
-        if (nonfinite) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
       }
     }
     __syncthreads();
     const int kstar = s_kstar;
-    if (kstar == -2) return;       // every CTA sees the same non-finite candidate and leaves
+    const unsigned long long t_d = stats_thread ? globaltimer_ns() : 0ull;
+    if (kstar == -2) {                // the same non-finite candidate in every CTA
+      if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
+      break;
+    }
 
-    // ---- commit the accepted candidate (no writes at all on a reject)
+    // ---- commit the accepted candidate to this CTA's samples (no writes on a reject)
     if (kstar >= 0) {
       const Cand& c = s_c[kstar];
-      for (int ch = blockIdx.x; ch < c.nch; ch += gridDim.x) {
-        if (c.layer == 0)
-          (void)l1_chunk<ACT1, ACT2, LOSS, true>(a, c, s_w2c[kstar], ch);
-        else
-          (void)l2_chunk<ACT1, ACT2, LOSS, true>(a, c, ch);
+      if (c.gcnt > 0) {
+        if (c.layer == 0) {
+          float* zrow = a.z1 + (size_t)c.row * a.Np;
+          for (int e = tid; e < c.ecnt; e += kLoopThreads) {
+            const int n = __ldg(a.xs_n + c.ebeg + e);
+            const float x = __ldg(a.xs_v + c.ebeg + e);
+            (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, sr, c, s_w2c[kstar], n - s0, x, zrow[n],
+                                                      zrow + n);
+          }
+        } else {
+          const float* zrow = a.z1 + (size_t)c.col * a.Np;
+          for (int e = tid; e < c.ecnt; e += kLoopThreads)
+            (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, sr, c, e, zrow[s0 + e]);
+        }
       }
-      if (blockIdx.x == 0 && threadIdx.x == 0) {
+      if (tid == 0) {                 // every CTA writes the same value
         const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
-        float* weff = c.layer ? a.w2 : a.w1;
-        weff[off] = c.neww;
+        (c.layer ? a.w2 : a.w1)[off] = c.neww;
         const int wk = c.layer ? a.wk2 : a.wk1;
         if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
       }
-      if (!grid_sync(a.bar, gridDim.x, gen, &a.st->err, &s_flag)) return;
+      __syncthreads();
       tau += (unsigned long long)(kstar + 1);
     } else {
       tau += (unsigned long long)Kb;
     }
+    if (stats_thread) {
+      const unsigned long long t_e = globaltimer_ns();
+      ph0 += t_b - t_a;
+      ph1 += t_c - t_b;
+      ph2 += t_d - t_c;
+      ph3 += t_e - t_d;
+    }
     buf ^= 1;
   }
-}
 
-// ------------------------------------------------------------------------------------------------
-// Full forward pass (resync): z1 = W1 X^T (SGEMM), then output fields, losses and S.
-// ------------------------------------------------------------------------------------------------
-
-// XT[i, n] = X[n, i] for n < N, 0 in the padding columns.
-__global__ void transpose_pad_kernel(const float* __restrict__ X, int N, int D,
-                                     float* __restrict__ XT, int Np) {
-  __shared__ float tile[32][33];
-  const int n0 = blockIdx.x * 32, i0 = blockIdx.y * 32;
-  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
-    const int n = n0 + r, i = i0 + threadIdx.x;
-    tile[r][threadIdx.x] = (n < N && i < D) ? X[(size_t)n * D + i] : 0.0f;
-  }
-  __syncthreads();
-  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
-    const int i = i0 + r, n = n0 + threadIdx.x;
-    if (i < D && n < Np) XT[(size_t)i * Np + n] = tile[threadIdx.x][r];
-  }
-}
-
-__global__ void csr_count_kernel(const float* __restrict__ XT, int Np, int N, int* cnt) {
-  const float* row = XT + (size_t)blockIdx.x * Np;
-  int c = 0;
-  for (int n0 = 0; n0 < N; n0 += blockDim.x) {
-    const int n = n0 + threadIdx.x;
-    c += __syncthreads_count(n < N && row[n] != 0.0f);
-  }
-  if (threadIdx.x == 0) cnt[blockIdx.x] = c;
-}
-
-// One CTA per feature; block-wide compaction keeps entries in ascending sample order.
-__global__ void csr_fill_kernel(const float* __restrict__ XT, int Np, int N, const int* off,
-                                int* xs_n, float* xs_v) {
-  __shared__ int wcount[32];
-  __shared__ int s_base;
-  const float* row = XT + (size_t)blockIdx.x * Np;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  if (threadIdx.x == 0) s_base = off[blockIdx.x];
-  __syncthreads();
-  for (int n0 = 0; n0 < N; n0 += blockDim.x) {
-    const int n = n0 + threadIdx.x;
-    const float v = n < N ? row[n] : 0.0f;
-    const bool nz = v != 0.0f;
-    const unsigned int m = __ballot_sync(0xffffffffu, nz);
-    if (lane == 0) wcount[warp] = __popc(m);
+  // ---- epilogue: sample records back to global memory, statistics to the device state
+  if (a.smem_records && !explicit_mode) {
     __syncthreads();
-    int before = 0, tot = 0;
-    for (int w = 0; w < nw; ++w) {
-      if (w < warp) before += wcount[w];
-      tot += wcount[w];
-    }
-    const int pos = s_base + before + __popc(m & ((1u << lane) - 1u));
-    if (nz) {
-      xs_n[pos] = n;
-      xs_v[pos] = v;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) s_base += tot;
-    __syncthreads();
+    const float4* src = reinterpret_cast<const float4*>(s_records);
+    float4* dst = reinterpret_cast<float4*>(a.srec + (size_t)s0 * kSR);
+    for (int t = tid; t < (s1 - s0) * (kSR / 4); t += kLoopThreads) dst[t] = src[t];
+  }
+  if (stats_thread && !explicit_mode) {
+    st->S = S;
+    st->trials += n_trials;
+    st->accepts += n_acc;
+    st->candidates += n_cand;
+    st->batches += n_batch;
+    st->wasted += n_waste;
+    st->forced += n_forced;
+    st->alg_bytes += n_bytes;
+    st->trace_written = n_trace;
+    st->phase_ns[0] += ph0;
+    st->phase_ns[1] += ph1;
+    st->phase_ns[2] += ph2;
+    st->phase_ns[3] += ph3;
   }
 }
 
-// Distinct 32-byte sectors (8 samples) of a z1 row holding feature i's entries.
-__global__ void csr_sectors_kernel(const int* __restrict__ off, const int* __restrict__ xs_n,
-                                   int* sect) {
-  const int s = off[blockIdx.x], e = off[blockIdx.x + 1];
-  int c = 0;
-  for (int p0 = s; p0 < e; p0 += blockDim.x) {
-    const int p = p0 + threadIdx.x;
-    c += __syncthreads_count(p < e && (p == s || (xs_n[p] >> 3) != (xs_n[p - 1] >> 3)));
-  }
-  if (threadIdx.x == 0) sect[blockIdx.x] = c;
-}
-
-__global__ void count_nonfinite_kernel(const float* __restrict__ p, size_t n, int* out) {
-  int bad = 0;
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
-       i += (size_t)gridDim.x * blockDim.x)
-    bad |= !isfinite(p[i]);
-  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(out, 1);
-}
-
-__global__ void init_layer_kernel(int wkind, float scale, const float* __restrict__ src,
-                                  const signed char* __restrict__ mask, size_t n, float* w_eff,
-                                  signed char* code, float* wfix) {
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
-       i += (size_t)gridDim.x * blockDim.x) {
-    const float v = src[i];
-    if (wkind == MCA_W_TERNARY_I8) {
-      const int t = (int)v;
-      code[i] = (signed char)t;
-      w_eff[i] = __fmul_rn(scale, (float)t);
-    } else if (wkind == MCA_W_MASKED_FP32) {
-      const int m = mask ? (mask[i] != 0) : 1;
-      wfix[i] = v;
-      code[i] = (signed char)m;
-      w_eff[i] = m ? v : 0.0f;
-    } else {
-      w_eff[i] = v;
-    }
-  }
-}
-
-// C[M x Ncol] = A[M x K] * B[K x Ncol], row-major, fp32 FMA in ascending k. Ncol % 128 == 0,
-// ldb and ldc multiples of 4. 128x128 tile per CTA, 256 threads, 8x8 outputs per thread.
-__global__ void __launch_bounds__(256) sgemm_nn_kernel(int M, int Ncol, int K,
-                                                       const float* __restrict__ A, int lda,
-                                                       const float* __restrict__ B, int ldb,
-                                                       float* __restrict__ C, int ldc) {
-  constexpr int BM = 128, BN = 128, BK = 8;
-  __shared__ __align__(16) float As[BK][BM];
-  __shared__ __align__(16) float Bs[BK][BN];
-  const int tid = threadIdx.x;
-  const int bm = blockIdx.y * BM, bn = blockIdx.x * BN;
-  const int tr = tid / 16, tc = tid % 16;
-  float acc[8][8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
-  const int arow = tid / 2, akk = (tid % 2) * 4;
-  const int bkk = tid / 32, bcol = (tid % 32) * 4;
-  for (int k0 = 0; k0 < K; k0 += BK) {
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int m = bm + arow, kk = k0 + akk + q;
-      As[akk + q][arow] = (m < M && kk < K) ? A[(size_t)m * lda + kk] : 0.0f;
-    }
-    {
-      const int kk = k0 + bkk;
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (kk < K) v = *reinterpret_cast<const float4*>(B + (size_t)kk * ldb + bn + bcol);
-      *reinterpret_cast<float4*>(&Bs[bkk][bcol]) = v;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < BK; ++kk) {
-      float ra[8], rb[8];
-      const float4 a0 = *reinterpret_cast<const float4*>(&As[kk][tr * 4]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&As[kk][64 + tr * 4]);
-      const float4 b0 = *reinterpret_cast<const float4*>(&Bs[kk][tc * 4]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&Bs[kk][64 + tc * 4]);
-      ra[0] = a0.x; ra[1] = a0.y; ra[2] = a0.z; ra[3] = a0.w;
-      ra[4] = a1.x; ra[5] = a1.y; ra[6] = a1.z; ra[7] = a1.w;
-      rb[0] = b0.x; rb[1] = b0.y; rb[2] = b0.z; rb[3] = b0.w;
-      rb[4] = b1.x; rb[5] = b1.y; rb[6] = b1.z; rb[7] = b1.w;
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(ra[i], rb[j], acc[i][j]);
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int m = bm + (i < 4 ? tr * 4 + i : 64 + tr * 4 + (i - 4));
-    if (m >= M) continue;
-    float* crow = C + (size_t)m * ldc + bn;
-    *reinterpret_cast<float4*>(crow + tc * 4) =
-        make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-    *reinterpret_cast<float4*>(crow + 64 + tc * 4) =
-        make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
-  }
-}
-
-// Output fields z2[:, n] = W2 f(z1[:, n]) (ascending j), the sample's loss, and its label.
-template <int ACT1, int ACT2, int LOSS>
-__global__ void __launch_bounds__(128) mlp2_outputs_kernel(Mlp2Args a, const int* __restrict__ y) {
-  constexpr int TJ = 64;
-  __shared__ float w2s[kMaxC][TJ];
-  const int n = blockIdx.x * blockDim.x + threadIdx.x;
-  float acc[kMaxC];
-#pragma unroll
-  for (int k = 0; k < kMaxC; ++k) acc[k] = 0.0f;
-  for (int j0 = 0; j0 < a.H; j0 += TJ) {
-    __syncthreads();
-    for (int t = threadIdx.x; t < kMaxC * TJ; t += blockDim.x) {
-      const int k = t / TJ, jj = t % TJ;
-      w2s[k][jj] = (k < a.C && j0 + jj < a.H) ? a.w2[(size_t)k * a.H + j0 + jj] : 0.0f;
-    }
-    __syncthreads();
-    if (n < a.N) {
-      const int jn = min(TJ, a.H - j0);
-      for (int jj = 0; jj < jn; ++jj) {
-        const float av = act<ACT1>(a.z1[(size_t)(j0 + jj) * a.Np + n], a.g1, a.act1);
-#pragma unroll
-        for (int k = 0; k < kMaxC; ++k)
-          if (k < a.C) acc[k] = fmaf(w2s[k][jj], av, acc[k]);
-      }
-    }
-  }
-  if (n < a.N) {
-    const int yn = y[n];
-    const float ln = sample_loss<ACT2, LOSS, kMaxC>(acc, a.C, yn, a.g2, a.act2, a.loss);
-    store_srec(a.srec, n, acc, ln, yn);
-  }
-}
-
-// S = sum_n loss_n in fp64, one CTA, fixed order.
-__global__ void __launch_bounds__(1024) sum_loss_kernel(const float* __restrict__ srec, int N,
-                                                        DevState* st) {
-  __shared__ double red[32];
-  double s = 0.0;
-  for (int n = threadIdx.x; n < N; n += blockDim.x) s += (double)srec[(size_t)n * kSR + kSR - 2];
-  s = block_sum_d(s, red);
-  if (threadIdx.x == 0) st->S = s;
-}
-
-// ------------------------------------------------------------------------------------------------
-// Launchers
-// ------------------------------------------------------------------------------------------------
-cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s) {
-  dim3 grid((Np + 31) / 32, (D + 31) / 32), block(32, 8);
-  transpose_pad_kernel<<<grid, block, 0, s>>>(X, N, D, XT, Np);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_csr_count(const float* XT, int Np, int N, int D, int* cnt, cudaStream_t s) {
-  csr_count_kernel<<<D, 256, 0, s>>>(XT, Np, N, cnt);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_csr_fill(const float* XT, int Np, int N, int D, const int* off, int* xs_n,
-                            float* xs_v, cudaStream_t s) {
-  csr_fill_kernel<<<D, 1024, 0, s>>>(XT, Np, N, off, xs_n, xs_v);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_csr_sectors(const int* off, const int* xs_n, int D, int* sect, cudaStream_t s) {
-  csr_sectors_kernel<<<D, 256, 0, s>>>(off, xs_n, sect);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_count_nonfinite(const float* p, size_t n, int* out, cudaStream_t s) {
-  if (n == 0) return cudaSuccess;
-  const int grid = (int)std::min<size_t>(4096, (n + 255) / 256);
-  count_nonfinite_kernel<<<grid, 256, 0, s>>>(p, n, out);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_init_layer(int wkind, float scale, const float* src, const signed char* mask,
-                              size_t n, float* w_eff, signed char* code, float* wfix,
-                              cudaStream_t s) {
-  const int grid = (int)std::min<size_t>(4096, (n + 255) / 256);
-  init_layer_kernel<<<grid, 256, 0, s>>>(wkind, scale, src, mask, n, w_eff, code, wfix);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, const float* B,
-                            int ldb, float* C, int ldc, cudaStream_t s) {
-  dim3 grid(Ncol / 128, (M + 127) / 128);
-  sgemm_nn_kernel<<<grid, 256, 0, s>>>(M, Ncol, K, A, lda, B, ldb, C, ldc);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_sum_loss(const float* srec, int N, DevState* st, cudaStream_t s) {
-  sum_loss_kernel<<<1, 1024, 0, s>>>(srec, N, st);
-  return cudaGetLastError();
-}
-
-// Kernel variants: (tanh, sigmoid, MSE), (tanh, identity, CE), (Gaussian, sigmoid, MSE), and a
-// generic one that switches on the transfer functions and loss at run time.
+// Kernel variants with 10 classes: (tanh, sigmoid, MSE), (tanh, identity, CE), (Gaussian, sigmoid,
+// MSE); and a generic one that switches on transfer functions, loss and class count at run time.
 using LoopFn = void (*)(Mlp2Args);
-using OutFn = void (*)(Mlp2Args, const int*);
 
-static void pick(const Mlp2Args& a, LoopFn* loop, OutFn* out) {
-  if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_SIGMOID && a.loss == MCA_LOSS_MSE_ONEHOT) {
-    *loop = mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT>;
-    *out = mlp2_outputs_kernel<MCA_ACT_TANH, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT>;
-  } else if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_IDENTITY &&
-             a.loss == MCA_LOSS_SOFTMAX_CE) {
-    *loop = mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_IDENTITY, MCA_LOSS_SOFTMAX_CE>;
-    *out = mlp2_outputs_kernel<MCA_ACT_TANH, MCA_ACT_IDENTITY, MCA_LOSS_SOFTMAX_CE>;
-  } else if (a.act1 == MCA_ACT_GAUSSIAN && a.act2 == MCA_ACT_SIGMOID &&
-             a.loss == MCA_LOSS_MSE_ONEHOT) {
-    *loop = mlp2_trial_loop<MCA_ACT_GAUSSIAN, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT>;
-    *out = mlp2_outputs_kernel<MCA_ACT_GAUSSIAN, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT>;
-  } else {
-    *loop = mlp2_trial_loop<-1, -1, -1>;
-    *out = mlp2_outputs_kernel<-1, -1, -1>;
+static LoopFn pick_loop(const Mlp2Args& a) {
+  if (a.C == 10) {
+    if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_SIGMOID && a.loss == MCA_LOSS_MSE_ONEHOT)
+      return mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>;
+    if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_IDENTITY && a.loss == MCA_LOSS_SOFTMAX_CE)
+      return mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_IDENTITY, MCA_LOSS_SOFTMAX_CE, 10>;
+    if (a.act1 == MCA_ACT_GAUSSIAN && a.act2 == MCA_ACT_SIGMOID && a.loss == MCA_LOSS_MSE_ONEHOT)
+      return mlp2_trial_loop<MCA_ACT_GAUSSIAN, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>;
   }
+  return mlp2_trial_loop<-1, -1, -1, -1>;
 }
 
-cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s) {
-  LoopFn loop;
-  OutFn out;
-  pick(a, &loop, &out);
-  out<<<(a.N + 127) / 128, 128, 0, s>>>(a, y);
-  return cudaGetLastError();
+size_t mlp2_loop_smem_bytes(const Mlp2Args& a) {
+  return a.smem_records ? (size_t)a.RS * kSR * sizeof(float) : 0;
 }
 
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms) {
-  LoopFn loop;
-  OutFn out;
-  pick(a, &loop, &out);
+  const LoopFn loop = pick_loop(a);
+  const size_t smem = mlp2_loop_smem_bytes(a);
+  if (smem > 0 && cudaFuncSetAttribute((const void*)loop,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem) != cudaSuccess)
+    return 0;
   int occ = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, loop, kLoopThreads, 0) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, loop, kLoopThreads, smem) !=
+      cudaSuccess)
     return 0;
   return occ * num_sms;
 }
 
-cudaError_t launch_mlp2_loop(const Mlp2Args& a, int grid, cudaStream_t s) {
-  LoopFn loop;
-  OutFn out;
-  pick(a, &loop, &out);
+cudaError_t launch_mlp2_loop(const Mlp2Args& a, cudaStream_t s) {
+  const LoopFn loop = pick_loop(a);
+  const size_t smem = mlp2_loop_smem_bytes(a);
+  if (smem > 0) {
+    cudaError_t e = cudaFuncSetAttribute((const void*)loop,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
   Mlp2Args args = a;
   void* params[] = {&args};
-  return cudaLaunchCooperativeKernel((const void*)loop, dim3(grid), dim3(kLoopThreads), params, 0,
-                                     s);
+  return cudaLaunchCooperativeKernel((const void*)loop, dim3(a.NR), dim3(kLoopThreads), params,
+                                     smem, s);
 }
 
 }  // namespace mca
