@@ -299,6 +299,10 @@ def run_ours(args):
                        "l2": "no flush: cached hidden fields (3.9 GB) exceed L2",
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
                        "accepts_timed": st1["accepts"] - st0["accepts"],
+                       "batches_timed": st1["batches"] - st0["batches"],
+                       "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
+                                    for q, nm in enumerate(["propose_eval", "barrier",
+                                                            "reduce_decide", "commit"])},
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

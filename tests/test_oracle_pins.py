@@ -415,3 +415,23 @@ def test_planted_dropped_rank1_term_is_caught(monkeypatch):
     monkeypatch.setattr(O.np, "outer", lambda a, b: np.zeros_like(real_outer(a, b)))
     with pytest.raises(AssertionError):
         test_incremental_equals_full("mlp_small", dict(N=60, H=6))
+
+
+def test_blocked_single_candidate_helpers_match_full_recompute():
+    """output_fields_blocked equals the full forward's output fields, and candidate_dS_two_layer
+    equals S(W') - S(W) from two full forward passes, for first- and output-layer weights."""
+    wl = W.mlp_wide(N=400, H=37)
+    p = O.Params(wl.layers, wl.init)
+    XT = wl.X.T.astype(np.float64)
+    Z2 = O.output_fields_blocked(p, XT, block=8)
+    Zs, _ = O.forward(p, XT)
+    assert np.allclose(Z2, Zs[1], rtol=0, atol=1e-13)
+    S = O.total_loss(p, XT, wl.y, wl.loss)
+    P1 = 784 * 37
+    for idx, v in ((5, 0.37), (P1 - 1, -0.8), (P1 + 3, 0.9), (wl.n_params - 1, -0.2)):
+        q = p.copy()
+        l, off = (0, idx) if idx < P1 else (1, idx - P1)
+        q.vals[l].reshape(-1)[off] = np.float32(v)
+        want = O.total_loss(q, XT, wl.y, wl.loss) - S
+        got = O.candidate_dS_two_layer(p, XT, wl.y, wl.loss, Z2, idx, float(np.float32(v)))
+        assert got == pytest.approx(want, rel=1e-9, abs=1e-10)
