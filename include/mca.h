@@ -206,6 +206,22 @@ mca_status mca_get_stats(mca_handle* h, mca_run_stats* stats);
 mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
                                size_t n, double* dS);
 
+/* The same evaluation as mca_eval_candidates, for callers that cannot allocate device memory:
+ * a caller whose device memory is entirely reserved by another allocator (a framework's caching
+ * allocator, a fixed arena), or a latency-critical loop that cannot afford the device-wide
+ * synchronisation a cudaMalloc or cudaFree may cause. The paper has no counterpart; this is an
+ * interface convenience. flat_idx [n] (uint32), new_w [n] (fp32) and dS [n] (fp64) are DEVICE
+ * arrays owned by the caller. The evaluation's scratch (one partial per candidate and sample
+ * range, plus a grid barrier) lives in a fixed 128 KB + 256 B device array inside the library,
+ * which every GPU that loads the library holds until the process exits; nothing is allocated per
+ * call. Limits: n <= 128 candidates and a handle of at most 256 sample ranges, else
+ * MCA_ERR_INVALID with a message. The first call on a device looks up the array's device address
+ * (once per device), so make that first call before any stream capture. All calls share the
+ * array: calls whose work overlaps on the GPU (two handles on different streams, or two threads)
+ * race and must be serialised by the caller. Blocks until the results are in dS. */
+mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t* flat_idx,
+                                       const float* new_w, size_t n, double* dS);
+
 void mca_destroy(mca_handle* h);
 
 /* Message of the last failed call on h (h may be NULL: then the last failed mca_create or

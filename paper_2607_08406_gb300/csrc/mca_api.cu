@@ -368,6 +368,10 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
 
 }  // namespace
 
+namespace mca {
+Mlp2Args handle_mlp2_args(mca_handle* h) { return mlp2_args(h); }
+}  // namespace mca
+
 extern "C" {
 
 const char* mca_last_error(mca_handle* h) {

@@ -100,6 +100,14 @@ size_t mlp2_loop_smem_bytes(const Mlp2Args& a);
 
 }  // namespace mca
 
+struct mca_handle;
+
+namespace mca {
+// Kernel arguments of a handle's trial loop (its state and workspace scratch).
+Mlp2Args handle_mlp2_args(mca_handle* h);
+
+}  // namespace mca
+
 struct mca_handle {
   std::string err;
   std::vector<mca_layer> layers;

@@ -85,6 +85,7 @@ SIGNATURES = {
     "mca_force_decisions": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t]),
     "mca_get_stats": (c_int32, [c_void_p, POINTER(mca_run_stats)]),
     "mca_eval_candidates": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "mca_eval_candidates_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "mca_destroy": (None, [c_void_p]),
     "mca_last_error": (c_char_p, [c_void_p]),
 }
@@ -262,6 +263,15 @@ def mca_eval_candidates(h: Handle, flat_idx, new_w) -> np.ndarray:
     _check(load_library().mca_eval_candidates(h.ptr, idx.ctypes.data, nw.ctypes.data, len(idx),
                                               out.ctypes.data), h.ptr)
     return out
+
+
+def mca_eval_candidates_noalloc(h: Handle, flat_idx, new_w, dS):
+    """flat_idx (int32/uint32 bits), new_w (float32) and dS (float64): CUDA tensors of equal length
+    owned by the caller; the library allocates nothing for this call."""
+    n = int(flat_idx.numel())
+    _check(load_library().mca_eval_candidates_noalloc(h.ptr, flat_idx.data_ptr(), new_w.data_ptr(),
+                                                      n, dS.data_ptr()), h.ptr)
+    return dS
 
 
 def mca_destroy(h: Handle):
