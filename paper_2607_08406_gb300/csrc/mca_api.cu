@@ -92,7 +92,7 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
     L.wfix.push_back(ly.wkind == MCA_W_MASKED_FP32 ? take(sizeof(float) * n) : SIZE_MAX);
   }
   L.z1 = take(sizeof(float) * (size_t)H * Np);
-  L.srec = take(sizeof(float) * (size_t)mca::kSR * N);
+  L.srec = take(sizeof(float) * (size_t)mca::kSR * Np);
   L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
   L.bar = take(sizeof(GridBarrier));
   L.st = take(sizeof(DevState));
@@ -299,7 +299,7 @@ mca_status resync(mca_handle* h) {
   CUDA_TRY(h, mca::launch_sgemm_nn(a.H, h->Np, h->D, h->w_eff[0], h->D, h->XT, h->Np, h->z1,
                                    h->Np, h->stream));
   CUDA_TRY(h, mca::launch_mlp2_outputs(a, h->y, h->stream));
-  CUDA_TRY(h, mca::launch_sum_loss(h->srec, (int)h->N, h->st, h->stream));
+  CUDA_TRY(h, mca::launch_sum_loss(h->srec, (int)h->N, h->Np, h->st, h->stream));
   h->launches += 3;
   return MCA_OK;
 }

@@ -38,13 +38,24 @@ __device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >
 
 // ------------------------------------------------------------------------------------------------
 // Transfer functions (Section 2) and losses (Eq. 2 with R = 0). ACT < 0 selects at run time.
+//
+// exp and log use the hardware base-2 units (__expf, __logf: a few ulp). tanh is its exponential
+// form tanh|x| = (1 - e^{-2|x|}) / (1 + e^{-2|x|}) with the sign restored: absolute error below
+// ~2e-7, far inside the 1e-5 relative tolerance on the loss sum. Exactness where it matters does not
+// depend on accuracy: an unchanged field gives f(z) - f(z) = 0 exactly because both sides go through
+// the same function.
 // ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ float tanh_exp(float x) {
+  const float t = __expf(-2.0f * fabsf(x));
+  return copysignf(__fdividef(1.0f - t, 1.0f + t), x);
+}
+
 __device__ __forceinline__ float act_rt(int act, float z, float g) {
   switch (act) {
-    case MCA_ACT_TANH: return tanhf(z);
-    case MCA_ACT_SIGMOID: return 1.0f / (1.0f + expf(-z));
+    case MCA_ACT_TANH: return tanh_exp(z);
+    case MCA_ACT_SIGMOID: return __fdividef(1.0f, 1.0f + __expf(-z));
     case MCA_ACT_RELU: return fmaxf(z, 0.0f);
-    case MCA_ACT_GAUSSIAN: return expf(-g * z * z);
+    case MCA_ACT_GAUSSIAN: return __expf(-g * z * z);
     case MCA_ACT_GELU: return 0.5f * z * (1.0f + erff(z * 0.7071067811865476f));
     default: return z;
   }
@@ -88,11 +99,11 @@ __device__ __forceinline__ float sample_loss(const float (&z)[MAXC], int C, int 
 #pragma unroll
   for (int k = 0; k < MAXC; ++k) {
     if (k < C) {
-      s += expf(a[k] - m);
+      s += __expf(a[k] - m);
       if (k == y) ay = a[k];
     }
   }
-  return (logf(s) + m) - ay;
+  return (__logf(s) + m) - ay;
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -203,36 +214,56 @@ __device__ __forceinline__ bool grid_sync(GridBarrier* bar, unsigned int nblocks
 }
 
 // ------------------------------------------------------------------------------------------------
-// Sample records: 16 floats per sample -- output fields [0, C), the sample's loss at 14, its label
-// (int bits) at 15. Works on shared or global memory.
+// Sample records, field-major: field f of sample n at base[f * pitch + n]; fields [0, M) are the
+// output fields, 14 the sample's loss, 15 its label (int bits). Field-major keeps the lanes of a warp,
+// which read different samples, in different shared-memory banks.
 // ------------------------------------------------------------------------------------------------
-// Load one sample record: fields into z[0..M), loss and label. Record slots M..13 are padding.
+constexpr int kRecFields = 16;
+constexpr int kRecLoss = 14;
+constexpr int kRecLabel = 15;
+
 template <int M>
-__device__ __forceinline__ void load_srec(const float* srec, int n, float (&z)[M], float& ell,
-                                          int& y) {
-  static_assert(M <= 14, "at most 14 output fields per sample record");
-  const float4* p = reinterpret_cast<const float4*>(srec + (size_t)n * 16);
-  const float4 v0 = p[0], v1 = p[1], v2 = p[2], v3 = p[3];
-  const float f[16] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w,
-                       v2.x, v2.y, v2.z, v2.w, v3.x, v3.y, v3.z, v3.w};
+__device__ __forceinline__ void load_srec(const float* base, int pitch, int n, float (&z)[M],
+                                          float& ell, int& y) {
+  static_assert(M <= kRecLoss, "at most 14 output fields per sample record");
 #pragma unroll
-  for (int k = 0; k < M; ++k) z[k] = f[k];
-  ell = v3.z;
-  y = __float_as_int(v3.w);
+  for (int k = 0; k < M; ++k) z[k] = base[k * pitch + n];
+  ell = base[kRecLoss * pitch + n];
+  y = __float_as_int(base[kRecLabel * pitch + n]);
 }
 
 template <int M>
-__device__ __forceinline__ void store_srec(float* srec, int n, const float (&z)[M], float ell,
-                                           int y) {
-  static_assert(M <= 14, "at most 14 output fields per sample record");
-  float f[16];
+__device__ __forceinline__ void store_srec(float* base, int pitch, int n, const float (&z)[M],
+                                           float ell, int y) {
+  static_assert(M <= kRecLoss, "at most 14 output fields per sample record");
 #pragma unroll
-  for (int k = 0; k < 14; ++k) f[k] = k < M ? z[k] : 0.0f;
-  float4* p = reinterpret_cast<float4*>(srec + (size_t)n * 16);
-  p[0] = make_float4(f[0], f[1], f[2], f[3]);
-  p[1] = make_float4(f[4], f[5], f[6], f[7]);
-  p[2] = make_float4(f[8], f[9], f[10], f[11]);
-  p[3] = make_float4(f[12], f[13], ell, __int_as_float(y));
+  for (int k = 0; k < M; ++k) base[k * pitch + n] = z[k];
+  base[kRecLoss * pitch + n] = ell;
+  base[kRecLabel * pitch + n] = __int_as_float(y);
+}
+
+// ------------------------------------------------------------------------------------------------
+// Compensated fp32 summation (Knuth's TwoSum): hi + lo carries the sum with the rounding error of
+// every addition kept in lo. Fixed order in, fixed result out; no fp64 (which is slow on this GPU).
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
+  const float s = hi + x;
+  const float bb = s - hi;
+  const float err = (hi - (s - bb)) + (x - bb);
+  hi = s;
+  lo += err;
+}
+
+// Lane 0 receives the compensated sum of the warp's (hi, lo) pairs (fixed xor tree).
+__device__ __forceinline__ float warp_sum_comp(float hi, float lo) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float h2 = __shfl_xor_sync(0xffffffffu, hi, o);
+    const float l2 = __shfl_xor_sync(0xffffffffu, lo, o);
+    two_sum_add(hi, lo, h2);
+    lo += l2;
+  }
+  return hi + lo;
 }
 
 }  // namespace mca

@@ -227,16 +227,17 @@ __global__ void __launch_bounds__(128) mlp2_outputs_kernel(Mlp2Args a, const int
   if (n < a.N) {
     const int yn = y[n];
     const float ln = sample_loss<ACT2, LOSS, kMaxC>(acc, a.C, yn, a.g2, a.act2, a.loss);
-    store_srec(a.srec, n, acc, ln, yn);
+    store_srec(a.srec, a.Np, n, acc, ln, yn);
   }
 }
 
 // S = sum_n loss_n in fp64, one CTA, fixed order.
 __global__ void __launch_bounds__(1024) sum_loss_kernel(const float* __restrict__ srec, int N,
-                                                        DevState* st) {
+                                                        int Np, DevState* st) {
   __shared__ double red[32];
   double s = 0.0;
-  for (int n = threadIdx.x; n < N; n += blockDim.x) s += (double)srec[(size_t)n * kSR + kSR - 2];
+  const float* ell = srec + (size_t)kRecLoss * Np;
+  for (int n = threadIdx.x; n < N; n += blockDim.x) s += (double)ell[n];
   s = block_sum_d(s, red);
   if (threadIdx.x == 0) st->S = s;
 }
@@ -294,8 +295,8 @@ cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, con
   return cudaGetLastError();
 }
 
-cudaError_t launch_sum_loss(const float* srec, int N, DevState* st, cudaStream_t s) {
-  sum_loss_kernel<<<1, 1024, 0, s>>>(srec, N, st);
+cudaError_t launch_sum_loss(const float* srec, int N, int Np, DevState* st, cudaStream_t s) {
+  sum_loss_kernel<<<1, 1024, 0, s>>>(srec, N, Np, st);
   return cudaGetLastError();
 }
 

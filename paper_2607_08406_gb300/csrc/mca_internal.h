@@ -15,7 +15,7 @@ struct GridBarrier;
 
 constexpr int kKmax = 128;        // speculative candidates per batch
 constexpr int kMaxC = 14;         // output fields a sample record holds
-constexpr int kSR = 16;           // floats per sample record: fields [0, C), loss at 14, label at 15
+constexpr int kSR = 16;           // fields per sample record: outputs [0, C), loss 14, label 15
 constexpr int kMaxClasses = kSR - 2;
 constexpr int kLoopThreads = 512; // threads per CTA of the trial-loop kernel
 constexpr int kLoopWarps = kLoopThreads / 32;
@@ -46,7 +46,7 @@ struct Mlp2Args {
   const int* xs_sect;        // [D] 32-byte sectors of a z1 row that feature i's entries touch
   const int* xs_roff;        // [D x (NR + 1)] first entry of feature i in range r
   float* z1;                 // [H x Np] hidden fields, feature-major
-  float* srec;               // [N x kSR] output fields, loss, label
+  float* srec;               // [kSR x Np] field-major: output fields, loss, label
   float* w1;                 // [H x D] effective weights
   float* w2;                 // [C x H]
   signed char* code1;        // ternary codes / mask bits (nullable for fp32 layers)
@@ -92,7 +92,7 @@ cudaError_t launch_init_layer(int wkind, float scale, const float* src, const si
 cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, const float* B,
                             int ldb, float* C, int ldc, cudaStream_t s);
 cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s);
-cudaError_t launch_sum_loss(const float* srec, int N, DevState* st, cudaStream_t s);
+cudaError_t launch_sum_loss(const float* srec, int N, int Np, DevState* st, cudaStream_t s);
 // Cooperative persistent trial loop, one CTA per sample range (grid = NR).
 cudaError_t launch_mlp2_loop(const Mlp2Args& a, cudaStream_t s);
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);

@@ -106,12 +106,19 @@ __device__ __forceinline__ void fill_candidate(const Mlp2Args& a, unsigned int i
   c.nsub = (c.ecnt + a.SUB - 1) / a.SUB;
 }
 
+// Sample records of this CTA's range: field f of range-local sample nl at rec[f * pitch + nl].
+struct Recs {
+  float* rec;
+  int pitch;
+};
+
 // One entry of a first-layer candidate: range-local sample nl with input value x and cached field
-// z. Returns l' - l; COMMIT also writes the new hidden field (*zp) and sample record.
+// z; w holds W2[:, j]. Returns l' - l; COMMIT also writes the new hidden field (*zp) and record.
 template <int ACT1, int ACT2, int LOSS, int NC, bool COMMIT>
-__device__ __forceinline__ float entry_l1(const Mlp2Args& a, float* sr, const Cand& c,
-                                          const float* w2c, int nl, float x, float z, float* zp) {
-  const float zn = fmaf(c.delta, x, z);
+__device__ __forceinline__ float entry_l1(const Mlp2Args& a, Recs R, float delta,
+                                          const float (&w)[NC > 0 ? NC : kMaxC], int nl, float x,
+                                          float z, float* zp) {
+  const float zn = fmaf(delta, x, z);
   const float da = act<ACT1>(zn, a.g1, a.act1) - act<ACT1>(z, a.g1, a.act1);
   if (COMMIT) *zp = zn;
   if (da == 0.0f) return 0.0f;
@@ -120,18 +127,18 @@ __device__ __forceinline__ float entry_l1(const Mlp2Args& a, float* sr, const Ca
   float zz[M];
   float ell;
   int y;
-  load_srec(sr, nl, zz, ell, y);
+  load_srec(R.rec, R.pitch, nl, zz, ell, y);
 #pragma unroll
   for (int k = 0; k < M; ++k)
-    if (k < C) zz[k] = fmaf(w2c[k], da, zz[k]);
+    if (k < C) zz[k] = fmaf(w[k], da, zz[k]);
   const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
-  if (COMMIT) store_srec(sr, nl, zz, ln, y);
+  if (COMMIT) store_srec(R.rec, R.pitch, nl, zz, ln, y);
   return ln - ell;
 }
 
-// One sample of an output-layer candidate W2[o, j] (o = c.row, j = c.col), cached field z1[j, n].
+// One sample of an output-layer candidate W2[o, j] (o = row, j's cached field z1[j, n] = z).
 template <int ACT1, int ACT2, int LOSS, int NC, bool COMMIT>
-__device__ __forceinline__ float entry_l2(const Mlp2Args& a, float* sr, const Cand& c, int nl,
+__device__ __forceinline__ float entry_l2(const Mlp2Args& a, Recs R, float delta, int o, int nl,
                                           float z) {
   constexpr int M = NC > 0 ? NC : kMaxC;
   const int C = NC > 0 ? NC : a.C;
@@ -139,30 +146,41 @@ __device__ __forceinline__ float entry_l2(const Mlp2Args& a, float* sr, const Ca
   float zz[M];
   float ell;
   int y;
-  load_srec(sr, nl, zz, ell, y);
+  load_srec(R.rec, R.pitch, nl, zz, ell, y);
   float zo = 0.0f;
 #pragma unroll
   for (int k = 0; k < M; ++k)
-    if (k == c.row) zo = zz[k];
-  const float zon = fmaf(c.delta, av, zo);
+    if (k == o) zo = zz[k];
+  const float zon = fmaf(delta, av, zo);
   if (zon == zo) return 0.0f;
 #pragma unroll
   for (int k = 0; k < M; ++k)
-    if (k == c.row) zz[k] = zon;
+    if (k == o) zz[k] = zon;
   const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
-  if (COMMIT) store_srec(sr, nl, zz, ln, y);
+  if (COMMIT) store_srec(R.rec, R.pitch, nl, zz, ln, y);
   return ln - ell;
+}
+
+template <int NC>
+__device__ __forceinline__ void load_w2c(const float* src, int C, float (&w)[NC > 0 ? NC : kMaxC]) {
+  constexpr int M = NC > 0 ? NC : kMaxC;
+#pragma unroll
+  for (int k = 0; k < M; ++k) w[k] = (NC > 0 || k < C) ? src[k] : 0.0f;
 }
 
 // Warp-level sum of l' - l over sub-chunk q of candidate c's segment in this CTA's range. Lane l
 // takes entries l, l + 32, ... of the sub-chunk in ascending order (four at a time, loads first).
 template <int ACT1, int ACT2, int LOSS, int NC>
-__device__ __forceinline__ float eval_sub(const Mlp2Args& a, float* sr, int s0, const Cand& c,
+__device__ __forceinline__ float eval_sub(const Mlp2Args& a, Recs R, int s0, const Cand& c,
                                           const float* w2c, int q) {
   const int lane = threadIdx.x & 31;
   const int e_lo = q * a.SUB;
   const int e_hi = min(e_lo + a.SUB, c.ecnt);
   const float* zrow = a.z1 + (size_t)(c.layer == 0 ? c.row : c.col) * a.Np;
+  const float delta = c.delta;
+  const int layer = c.layer, o = c.row, ebeg = c.ebeg;
+  float w[NC > 0 ? NC : kMaxC];
+  load_w2c<NC>(w2c, a.C, w);
   float acc = 0.0f;
   for (int g = e_lo; g < e_hi; g += 128) {
     int nn[4];
@@ -173,9 +191,9 @@ __device__ __forceinline__ float eval_sub(const Mlp2Args& a, float* sr, int s0, 
       nn[t] = -1;
       xv[t] = 0.0f;
       if (e < e_hi) {
-        if (c.layer == 0) {
-          nn[t] = __ldg(a.xs_n + c.ebeg + e);
-          xv[t] = __ldg(a.xs_v + c.ebeg + e);
+        if (layer == 0) {
+          nn[t] = __ldg(a.xs_n + ebeg + e);
+          xv[t] = __ldg(a.xs_v + ebeg + e);
         } else {
           nn[t] = s0 + e;
         }
@@ -186,14 +204,77 @@ __device__ __forceinline__ float eval_sub(const Mlp2Args& a, float* sr, int s0, 
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       if (nn[t] < 0) continue;
-      if (c.layer == 0)
-        acc += entry_l1<ACT1, ACT2, LOSS, NC, false>(a, sr, c, w2c, nn[t] - s0, xv[t], zv[t],
+      if (layer == 0)
+        acc += entry_l1<ACT1, ACT2, LOSS, NC, false>(a, R, delta, w, nn[t] - s0, xv[t], zv[t],
                                                      nullptr);
       else
-        acc += entry_l2<ACT1, ACT2, LOSS, NC, false>(a, sr, c, nn[t] - s0, zv[t]);
+        acc += entry_l2<ACT1, ACT2, LOSS, NC, false>(a, R, delta, o, nn[t] - s0, zv[t]);
     }
   }
   return warp_sum(acc);
+}
+
+// Up to four sub-chunks of at most 128 entries each (the common case SUB == 128) at once: every lane
+// issues the loads of all its entries (up to 16) before computing any, so one warp keeps up to 512
+// gathers in flight. The per-sub-chunk lane order is the same as eval_sub's.
+template <int ACT1, int ACT2, int LOSS, int NC>
+__device__ __forceinline__ void eval_quad(const Mlp2Args& a, Recs R, int s0, const Cand* cs,
+                                          const float (*w2c)[kMaxC], const int (&ks)[4],
+                                          const int (&qs)[4], int nq, float (&out)[4]) {
+  const int lane = threadIdx.x & 31;
+  int nn[16];
+  float xv[16], zv[16];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const Cand& c = cs[ks[u]];
+    const int e_lo = qs[u] * 128;
+    const int e_hi = u < nq ? min(e_lo + 128, c.ecnt) : 0;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int e = e_lo + t * 32 + lane;
+      const int sidx = u * 4 + t;
+      nn[sidx] = -1;
+      xv[sidx] = 0.0f;
+      if (e < e_hi) {
+        if (c.layer == 0) {
+          nn[sidx] = __ldg(a.xs_n + c.ebeg + e);
+          xv[sidx] = __ldg(a.xs_v + c.ebeg + e);
+        } else {
+          nn[sidx] = s0 + e;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const Cand& c = cs[ks[u]];
+    const float* zrow = a.z1 + (size_t)(c.layer == 0 ? c.row : c.col) * a.Np;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int sidx = u * 4 + t;
+      zv[sidx] = nn[sidx] >= 0 ? zrow[nn[sidx]] : 0.0f;
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const Cand& c = cs[ks[u]];
+    const float delta = c.delta;
+    const int layer = c.layer, o = c.row;
+    float w[NC > 0 ? NC : kMaxC];
+    load_w2c<NC>(w2c[ks[u]], a.C, w);
+    float acc = 0.0f;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int sidx = u * 4 + t;
+      if (nn[sidx] < 0) continue;
+      if (layer == 0)
+        acc += entry_l1<ACT1, ACT2, LOSS, NC, false>(a, R, delta, w, nn[sidx] - s0, xv[sidx],
+                                                     zv[sidx], nullptr);
+      else
+        acc += entry_l2<ACT1, ACT2, LOSS, NC, false>(a, R, delta, o, nn[sidx] - s0, zv[sidx]);
+    }
+    out[u] = warp_sum(acc);
+  }
 }
 
 template <int ACT1, int ACT2, int LOSS, int NC>
@@ -202,19 +283,22 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   __shared__ Cand s_c[kKmax];
   __shared__ float s_w2c[kKmax][kMaxC];
   __shared__ float s_sub[kKmax * kMaxSubs];
-  __shared__ double s_dS[kKmax];
+  __shared__ float s_dS[kKmax];
   __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
-  __shared__ int s_flag, s_kstar, s_total;
+  __shared__ int s_flag, s_kstar, s_total, s_bvalid;
+  __shared__ unsigned long long s_bbytes;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int r = blockIdx.x;
   const int s0 = min(r * a.RS, a.N), s1 = min(s0 + a.RS, a.N);
   const bool explicit_mode = a.n_explicit > 0;
-  float* sr = a.smem_records ? s_records : a.srec + (size_t)s0 * kSR;
+  const Recs R = a.smem_records ? Recs{s_records, a.RS} : Recs{a.srec + s0, a.Np};
   if (a.smem_records) {
-    const float4* src = reinterpret_cast<const float4*>(a.srec + (size_t)s0 * kSR);
-    float4* dst = reinterpret_cast<float4*>(s_records);
-    for (int t = tid; t < (s1 - s0) * (kSR / 4); t += kLoopThreads) dst[t] = src[t];
+    const int ns = s1 - s0;
+    for (int t = tid; t < kRecFields * ns; t += kLoopThreads) {
+      const int f = t / ns, nl = t - f * ns;
+      s_records[f * a.RS + nl] = a.srec[(size_t)f * a.Np + s0 + nl];
+    }
   }
 
   // CTA 0, thread 0 carries the run statistics in registers for the whole launch.
@@ -255,13 +339,28 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
       s_c[k] = c;
     }
     __syncthreads();
-    if (warp == 0) {                 // exclusive scan of the sub-chunk counts
+    if (warp == 0) {                 // exclusive scan of the sub-chunk counts; batch statistics
       int v[4], loc = 0;
+      unsigned long long bytes = 0ull;
+      int valid = 0;
 #pragma unroll
       for (int t = 0; t < 4; ++t) {
         const int k = lane * 4 + t;
         v[t] = k < Kb ? s_c[k].nsub : 0;
         loc += v[t];
+        if (k < Kb) {
+          bytes += s_c[k].bytes;
+          valid += s_c[k].valid;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
+        valid += __shfl_xor_sync(0xffffffffu, valid, o);
+      }
+      if (lane == 0) {
+        s_bbytes = bytes;
+        s_bvalid = valid;
       }
       int inc = loc;
 #pragma unroll
@@ -280,15 +379,40 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
     }
     __syncthreads();
 
-    // ---- evaluate this CTA's samples: warp per sub-chunk
+    // ---- evaluate this CTA's samples: warp per sub-chunk (four at a time when SUB == 128)
     {
       const int total = s_total;
       int k = 0;
-      for (int it = warp; it < total; it += kLoopWarps) {
-        while (s_c[k].sub0 + s_c[k].nsub <= it) ++k;
-        const float v =
-            eval_sub<ACT1, ACT2, LOSS, NC>(a, sr, s0, s_c[k], s_w2c[k], it - s_c[k].sub0);
-        if (lane == 0) s_sub[it] = v;
+      if (a.SUB == 128) {
+        for (int it0 = warp; it0 < total; it0 += 4 * kLoopWarps) {
+          int ks[4], qs[4], nq = 0;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int it = it0 + u * kLoopWarps;
+            ks[u] = k;
+            qs[u] = 0;
+            if (it < total) {
+              while (s_c[k].sub0 + s_c[k].nsub <= it) ++k;
+              ks[u] = k;
+              qs[u] = it - s_c[k].sub0;
+              nq = u + 1;
+            }
+          }
+          float v[4];
+          eval_quad<ACT1, ACT2, LOSS, NC>(a, R, s0, s_c, s_w2c, ks, qs, nq, v);
+          if (lane == 0) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+              if (u < nq) s_sub[it0 + u * kLoopWarps] = v[u];
+          }
+        }
+      } else {
+        for (int it = warp; it < total; it += kLoopWarps) {
+          while (s_c[k].sub0 + s_c[k].nsub <= it) ++k;
+          const float v =
+              eval_sub<ACT1, ACT2, LOSS, NC>(a, R, s0, s_c[k], s_w2c[k], it - s_c[k].sub0);
+          if (lane == 0) s_sub[it] = v;
+        }
       }
     }
     __syncthreads();
@@ -303,18 +427,38 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
     if (!grid_sync(a.bar, gridDim.x, gen, &st->err, &s_flag)) break;
     const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
 
-    // ---- dS of every candidate: the NR partials in a fixed order (lane-strided, fp64)
-    for (int k = warp; k < Kb; k += kLoopWarps) {
-      double d = 0.0;
-      if (s_c[k].gcnt > 0)
-        for (int q = lane; q < a.NR; q += 32) d += (double)part[(size_t)k * a.NR + q];
-      d = warp_sum_d(d);
-      if (lane == 0) s_dS[k] = s_c[k].valid ? d : __longlong_as_double(0x7ff8000000000000ll);
+    // ---- dS of every candidate: the NR partials in a fixed order (lane-strided, compensated
+    // fp32). A warp takes candidates warp, warp + 16, warp + 32, warp + 48 together, loads first.
+    for (int k0 = warp; k0 < Kb; k0 += 4 * kLoopWarps) {
+      float hi[4] = {0.0f, 0.0f, 0.0f, 0.0f}, lo[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      for (int q0 = 0; q0 < a.NR; q0 += 32 * 8) {
+        float v[4][8];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int k = k0 + u * kLoopWarps;
+          const bool live = k < Kb && s_c[k].gcnt > 0;
+#pragma unroll
+          for (int m = 0; m < 8; ++m) {
+            const int q = q0 + m * 32 + lane;
+            v[u][m] = (live && q < a.NR) ? part[(size_t)k * a.NR + q] : 0.0f;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int m = 0; m < 8; ++m) two_sum_add(hi[u], lo[u], v[u][m]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = k0 + u * kLoopWarps;
+        const float t = warp_sum_comp(hi[u], lo[u]);
+        if (lane == 0 && k < Kb) s_dS[k] = s_c[k].valid ? t : __int_as_float(0x7fc00000);
+      }
     }
     __syncthreads();
     if (explicit_mode) {
       if (r == 0)
-        for (int k = tid; k < Kb; k += kLoopThreads) a.ex_out[k] = s_dS[k];
+        for (int k = tid; k < Kb; k += kLoopThreads) a.ex_out[k] = (double)s_dS[k];
       break;
     }
 
@@ -339,12 +483,12 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
             facc = a.facc[lo] != 0;
           }
         }
-        const double d = s_dS[k];
+        const float d = s_dS[k];
         if (forced) {
           acc = facc;
         } else {
           bad = !isfinite(d);
-          acc = a.strict ? (d < 0.0) : (d <= 0.0);
+          acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
         }
       }
       const unsigned int ma = __ballot_sync(0xffffffffu, acc);
@@ -377,7 +521,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
             rec.new_w = s_c[k].neww;
             rec.valid = s_c[k].valid;
             rec.forced = (int)((s_mforced[k >> 5] >> (k & 31)) & 1u);
-            rec.dS = s_dS[k];
+            rec.dS = (double)s_dS[k];
             rec.S = S;
             a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
             ++n_trace;
@@ -389,16 +533,14 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
           if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
           n_forced += (unsigned long long)__popc(m);
         }
-        for (int k = 0; k < Kb; ++k) {
-          n_cand += s_c[k].valid ? 1ull : 0ull;
-          n_bytes += s_c[k].bytes;
-        }
+        n_cand += (unsigned long long)s_bvalid;
+        n_bytes += s_bbytes;
         ++n_batch;
         if (kstar >= 0) {
           n_trials += (unsigned long long)(kstar + 1);
           ++n_acc;
           n_waste += (unsigned long long)(Kb - kstar - 1);
-          S += s_dS[kstar];
+          S += (double)s_dS[kstar];
           if (s_c[kstar].layer == 0 && s_c[kstar].gcnt > 0)
             n_bytes += 32ull * (unsigned long long)a.xs_sect[s_c[kstar].col];
         } else if (kstar == -1) {
@@ -420,16 +562,18 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
       if (c.gcnt > 0) {
         if (c.layer == 0) {
           float* zrow = a.z1 + (size_t)c.row * a.Np;
+          float w[NC > 0 ? NC : kMaxC];
+          load_w2c<NC>(s_w2c[kstar], a.C, w);
           for (int e = tid; e < c.ecnt; e += kLoopThreads) {
             const int n = __ldg(a.xs_n + c.ebeg + e);
             const float x = __ldg(a.xs_v + c.ebeg + e);
-            (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, sr, c, s_w2c[kstar], n - s0, x, zrow[n],
+            (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
                                                       zrow + n);
           }
         } else {
           const float* zrow = a.z1 + (size_t)c.col * a.Np;
           for (int e = tid; e < c.ecnt; e += kLoopThreads)
-            (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, sr, c, e, zrow[s0 + e]);
+            (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
         }
       }
       if (tid == 0) {                 // every CTA writes the same value
@@ -456,9 +600,11 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   // ---- epilogue: sample records back to global memory, statistics to the device state
   if (a.smem_records && !explicit_mode) {
     __syncthreads();
-    const float4* src = reinterpret_cast<const float4*>(s_records);
-    float4* dst = reinterpret_cast<float4*>(a.srec + (size_t)s0 * kSR);
-    for (int t = tid; t < (s1 - s0) * (kSR / 4); t += kLoopThreads) dst[t] = src[t];
+    const int ns = s1 - s0;
+    for (int t = tid; t < kRecFields * ns; t += kLoopThreads) {
+      const int f = t / ns, nl = t - f * ns;
+      a.srec[(size_t)f * a.Np + s0 + nl] = s_records[f * a.RS + nl];
+    }
   }
   if (stats_thread && !explicit_mode) {
     st->S = S;
@@ -494,7 +640,7 @@ static LoopFn pick_loop(const Mlp2Args& a) {
 }
 
 size_t mlp2_loop_smem_bytes(const Mlp2Args& a) {
-  return a.smem_records ? (size_t)a.RS * kSR * sizeof(float) : 0;
+  return a.smem_records ? (size_t)a.RS * kRecFields * sizeof(float) : 0;
 }
 
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms) {
