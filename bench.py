@@ -29,6 +29,22 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roofline"
+
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the trial-loop kernel per trial,
+# from the ncu launch list of `python bench.py --steps 3 --warmup 3 --no-e2e --no-cpu` summarised in
+# profiles/. It is only valid for the kernel source it was measured on; any other source hash
+# reports null.
+LOOP_TRAFFIC = {"source_sha1": None, "bytes_per_trial": None}
+LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
+
+
+def loop_source_sha1() -> str:
+    import hashlib
+    h = hashlib.sha1()
+    for rel in LOOP_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 UNIT = "trials/s"
 JOB_TRIALS = 1_000_000
 
@@ -238,6 +254,9 @@ def run_ours(args):
     bytes_timed = st1["alg_bytes"] - st0["alg_bytes"]
     loop_launches = K
     achieved = bytes_timed / loop_launches / (total_ms / K / 1e3) / 1e9
+    traffic = None
+    if LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and LOOP_TRAFFIC["bytes_per_trial"]:
+        traffic = LOOP_TRAFFIC["bytes_per_trial"] * (st1["trials"] - st0["trials"]) / K
     loss_end = mca.mca_loss(h)
     h.close()
 
@@ -306,9 +325,10 @@ def run_ours(args):
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
+                         "frac": achieved / peak, "traffic": traffic,
                          "kernel": "mlp2_trial_loop", "peak_kind": peak_kind,
-                         "bytes": "compulsory DRAM bytes counted by the kernel per candidate"},
+                         "bytes": "compulsory DRAM bytes of the distinct candidates evaluated, "
+                                  "counted by the kernel (per launch)"},
             "cpu_baseline": cpu,
             "e2e": e2e,
             "clocks": clk.summary(),

@@ -125,8 +125,9 @@ typedef struct {
   uint64_t launches;       /* kernels this handle launched */
   uint64_t tau;            /* next trial counter */
   double S;                /* current loss sum */
-  uint64_t alg_bytes;      /* compulsory DRAM bytes of the evaluated candidates and commits: per
-                              first-layer candidate 32 B per hidden-field sector its input
+  uint64_t alg_bytes;      /* compulsory DRAM bytes of the distinct candidates evaluated (each
+                              trial counted once, the first time it is evaluated) and commits:
+                              per first-layer candidate 32 B per hidden-field sector its input
                               feature's non-zeros touch + 8 B per non-zero; per output-layer
                               candidate 4 B per sample (one hidden-field row); per accepted
                               first-layer candidate the sectors written back */

@@ -286,7 +286,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   __shared__ float s_dS[kKmax];
   __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
   __shared__ int s_flag, s_kstar, s_total, s_bvalid;
-  __shared__ unsigned long long s_bbytes;
+  __shared__ unsigned long long s_bbytes, s_tau_hi;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int r = blockIdx.x;
@@ -313,6 +313,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   }
   unsigned int gen = 0;
   unsigned long long tau = a.tau0;
+  if (tid == 0) s_tau_hi = a.tau0;
   const unsigned long long end = a.tau0 + a.n_trials;
   int buf = 0;
   __syncthreads();
@@ -349,7 +350,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
         v[t] = k < Kb ? s_c[k].nsub : 0;
         loc += v[t];
         if (k < Kb) {
-          bytes += s_c[k].bytes;
+          // bytes of candidates not evaluated before in this launch (a candidate re-evaluated in
+          // the next batch finds its data on chip)
+          if (tau + (unsigned long long)k >= s_tau_hi) bytes += s_c[k].bytes;
           valid += s_c[k].valid;
         }
       }
@@ -583,8 +586,10 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
         if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
       }
       __syncthreads();
+      if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
       tau += (unsigned long long)(kstar + 1);
     } else {
+      if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
       tau += (unsigned long long)Kb;
     }
     if (stats_thread) {
