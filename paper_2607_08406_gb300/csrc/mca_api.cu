@@ -60,15 +60,21 @@ bool is_device_ptr(const void* p) {
 }
 
 struct Layout {
-  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, bar, st, trace, ex_idx, ex_new, ex_out,
-      scratch, total;
-  std::vector<size_t> w_eff, code, wfix;
+  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, bar, st, trace, ex_idx,
+      ex_new, ex_out, scratch, ell, ctl, total;
+  std::vector<size_t> w_eff, code, wfix, Z;
 };
+
+bool is_deep(const std::vector<mca_layer>& layers) { return layers.size() > 2; }
+int deep_tiles(long long N) { return (int)((N + mca::kDeepTS - 1) / mca::kDeepTS); }
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
 
+// Device memory of a handle. Single hidden layer: feature CSR of X, z1, sample records, per-range
+// partials. Deep: the fields of every layer, per-sample losses, per-tile partials.
 Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long nnz, int trace_cap,
             int NR) {
+  const bool deep = is_deep(layers);
   Layout L;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -80,6 +86,7 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   const int H = layers[0].n_out;
   L.XT = take(sizeof(float) * (size_t)D * Np);
   L.y = take(sizeof(int) * (size_t)N);
+  if (deep) nnz = 0;
   L.xs_off = take(sizeof(int) * (size_t)(D + 1));
   L.xs_n = take(sizeof(int) * (size_t)std::max<long long>(nnz, 1));
   L.xs_v = take(sizeof(float) * (size_t)std::max<long long>(nnz, 1));
@@ -91,9 +98,18 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
     L.code.push_back(ly.wkind != MCA_W_FP32 ? take(n) : SIZE_MAX);
     L.wfix.push_back(ly.wkind == MCA_W_MASKED_FP32 ? take(sizeof(float) * n) : SIZE_MAX);
   }
-  L.z1 = take(sizeof(float) * (size_t)H * Np);
-  L.srec = take(sizeof(float) * (size_t)mca::kSR * Np);
-  L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
+  if (deep) {
+    for (const auto& ly : layers) L.Z.push_back(take(sizeof(float) * (size_t)ly.n_out * Np));
+    L.ell = take(sizeof(float) * (size_t)Np);
+    L.ctl = take(sizeof(mca::DeepCtl));
+    L.z1 = L.srec = SIZE_MAX;
+    L.partial = take(sizeof(float) * (size_t)mca::kKmax * deep_tiles(N));
+  } else {
+    L.ell = L.ctl = SIZE_MAX;
+    L.z1 = take(sizeof(float) * (size_t)H * Np);
+    L.srec = take(sizeof(float) * (size_t)mca::kSR * Np);
+    L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
+  }
   L.bar = take(sizeof(GridBarrier));
   L.st = take(sizeof(DevState));
   L.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
@@ -133,8 +149,13 @@ mca_status check_spec(const mca_layer* layers, int n_layers, int loss, const mca
   const int C = layers[n_layers - 1].n_out;
   if (C > mca::kMaxClasses)
     return fail(nullptr, MCA_ERR_UNSUPPORTED, "%d outputs > %d", C, mca::kMaxClasses);
-  if (n_layers != 2)
-    return fail(nullptr, MCA_ERR_UNSUPPORTED, "this build runs single-hidden-layer nets only");
+  if (n_layers > mca::kMaxLayers)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "%d layers > %d", n_layers, mca::kMaxLayers);
+  if (n_layers > 2)
+    for (int l = 0; l + 1 < n_layers; ++l)
+      if (layers[l].n_out > mca::kDeepMaxWidth)
+        return fail(nullptr, MCA_ERR_UNSUPPORTED, "deep nets: hidden width %d > %d",
+                    layers[l].n_out, mca::kDeepMaxWidth);
   out->assign(layers, layers + n_layers);
   return MCA_OK;
 }
@@ -293,13 +314,67 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   return a;
 }
 
+mca::DeepArgs deep_args(mca_handle* h) {
+  mca::DeepArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.L = (int)h->layers.size();
+  a.N = (int)h->N;
+  a.Np = h->Np;
+  a.D = h->D;
+  a.C = h->C;
+  a.ntiles = h->ntiles;
+  for (int l = 0; l < a.L; ++l) {
+    const mca_layer& L = h->layers[l];
+    a.n_in[l] = L.n_in;
+    a.n_out[l] = L.n_out;
+    a.act[l] = L.act;
+    a.g[l] = L.act_param;
+    a.wk[l] = L.wkind;
+    a.sc[l] = L.scale;
+    a.off[l] = h->off[l];
+    a.w[l] = h->w_eff[l];
+    a.code[l] = h->code[l];
+    a.wfix[l] = h->wfix[l];
+    a.Z[l] = h->Z[l];
+  }
+  a.off[a.L] = h->P;
+  a.XT = h->XT;
+  a.ell = h->ell;
+  a.y = h->y;
+  a.loss = h->loss;
+  a.op = h->dom.op;
+  a.lo = h->dom.lo;
+  a.hi = h->dom.hi;
+  a.delta = h->dom.delta;
+  a.bound = h->dom.bound;
+  a.strict = h->dom.strict;
+  a.partial = h->partial;
+  a.st = h->st;
+  a.ctl = h->ctl;
+  a.trace = h->trace;
+  a.trace_cap = h->trace_cap;
+  a.ftau = h->ftau;
+  a.facc = h->facc;
+  a.nforce = h->nforce;
+  return a;
+}
+
 // Full forward pass: every cached field, every sample's loss, and S (Section 2.4's cache).
 mca_status resync(mca_handle* h) {
+  if (h->deep) {
+    const mca::DeepArgs a = deep_args(h);
+    for (int l = 0; l < a.L; ++l) CUDA_TRY(h, mca::launch_deep_forward_layer(a, l, h->stream));
+    CUDA_TRY(h, mca::launch_deep_losses(a, h->stream));
+    CUDA_TRY(h, mca::launch_sum_loss(h->ell, (int)h->N, h->st, h->stream));
+    h->launches += a.L + 2;
+    return MCA_OK;
+  }
   mca::Mlp2Args a = mlp2_args(h);
   CUDA_TRY(h, mca::launch_sgemm_nn(a.H, h->Np, h->D, h->w_eff[0], h->D, h->XT, h->Np, h->z1,
                                    h->Np, h->stream));
   CUDA_TRY(h, mca::launch_mlp2_outputs(a, h->y, h->stream));
-  CUDA_TRY(h, mca::launch_sum_loss(h->srec, (int)h->N, h->Np, h->st, h->stream));
+  CUDA_TRY(h, mca::launch_sum_loss(h->srec + (size_t)mca::kRecLoss * h->Np, (int)h->N, h->st,
+                                    h->stream));
   h->launches += 3;
   return MCA_OK;
 }
@@ -385,6 +460,10 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
   if (rc != MCA_OK) return rc;
   if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
   const mca_options o = opt ? *opt : default_options();
+  if (is_deep(ls)) {
+    *bytes = plan(ls, data->n, data->d, 0, o.trace_cap, 0).total;
+    return MCA_OK;
+  }
   long long nnz = 0;
   rc = count_nnz(data, (cudaStream_t)o.stream, &nnz);
   if (rc != MCA_OK) return rc;
@@ -454,7 +533,9 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
 
   CTRY(cudaGetDevice(&h->device));
   CTRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
-  {
+  h->deep = is_deep(ls);
+  h->ntiles = deep_tiles(h->N);
+  if (!h->deep) {
     long long nnz = 0;
     mca_status s = count_nnz(data, h->stream, &nnz);
     if (s != MCA_OK) {
@@ -463,7 +544,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     }
     h->nnz = nnz;
   }
-  {
+  if (!h->deep) {
     Ranges R;
     mca_status s = choose_ranges(ls, loss, h->N, o.grid, &R);
     if (s != MCA_OK) {
@@ -503,8 +584,15 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
                                             : reinterpret_cast<signed char*>(base + L.code[l]));
     h->wfix.push_back(L.wfix[l] == SIZE_MAX ? nullptr : reinterpret_cast<float*>(base + L.wfix[l]));
   }
-  h->z1 = reinterpret_cast<float*>(base + L.z1);
-  h->srec = reinterpret_cast<float*>(base + L.srec);
+  if (h->deep) {
+    for (size_t l = 0; l < ls.size(); ++l) h->Z.push_back(reinterpret_cast<float*>(base + L.Z[l]));
+    h->ell = reinterpret_cast<float*>(base + L.ell);
+    h->ctl = reinterpret_cast<mca::DeepCtl*>(base + L.ctl);
+    CTRY(cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream));
+  } else {
+    h->z1 = reinterpret_cast<float*>(base + L.z1);
+    h->srec = reinterpret_cast<float*>(base + L.srec);
+  }
   h->partial = reinterpret_cast<float*>(base + L.partial);
   h->bar = reinterpret_cast<GridBarrier*>(base + L.bar);
   h->st = reinterpret_cast<DevState*>(base + L.st);
@@ -529,14 +617,18 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   CTRY(cudaMemsetAsync(scratch, 0, sizeof(int), h->stream));
   CTRY(mca::launch_count_nonfinite(Xd, nx, scratch, h->stream));
   CTRY(mca::launch_transpose_pad(Xd, (int)h->N, h->D, h->XT, h->Np, h->stream));
-  CTRY(mca::launch_csr_count(h->XT, h->Np, (int)h->N, h->D, scratch + 8, h->stream));
-  h->launches += 3;
+  if (!h->deep) {
+    CTRY(mca::launch_csr_count(h->XT, h->Np, (int)h->N, h->D, scratch + 8, h->stream));
+    h->launches++;
+  }
+  h->launches += 2;
   std::vector<int> cnt(h->D + 8);
   CTRY(cudaMemcpyAsync(cnt.data(), scratch, sizeof(int) * (h->D + 8), cudaMemcpyDeviceToHost,
                        h->stream));
   CTRY(cudaStreamSynchronize(h->stream));
   if (Xtmp) cudaFree(Xtmp);
   if (cnt[0]) return bail(fail(h, MCA_ERR_NUMERIC, "non-finite value in x"));
+  if (!h->deep) {
   std::vector<int> offs(h->D + 1, 0);
   long long acc = 0;
   for (int i = 0; i < h->D; ++i) {
@@ -553,6 +645,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   CTRY(mca::launch_csr_range_offsets(h->xs_off, h->xs_n, h->D, h->NR, h->RS, h->xs_roff,
                                      h->stream));
   h->launches += 3;
+  }
   {
     std::vector<int> yh(h->N);
     CTRY(cudaMemcpyAsync(yh.data(), data->y, sizeof(int) * h->N, cudaMemcpyDefault, h->stream));
@@ -579,6 +672,36 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
   if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
   if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
   uint64_t remaining = n_trials;
+  if (h->deep) {
+    // one batch per round trip: evaluate, decide, commit, then read how many trials it consumed
+    mca::DeepArgs a = deep_args(h);
+    a.seed = seed;
+    const uint64_t R = (uint64_t)h->opt.resync_period;
+    while (remaining > 0) {
+      uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)h->opt.K);
+      if (R > 0) kb = std::min<uint64_t>(kb, R - h->tau % R);
+      a.tau = h->tau;
+      a.Kb = (int)kb;
+      CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
+      CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
+      CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+      h->launches += 3;
+      mca::DeepCtl ctl;
+      CUDA_TRY(h, cudaMemcpyAsync(&ctl, h->ctl, sizeof(ctl), cudaMemcpyDeviceToHost, h->stream));
+      CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+      if (ctl.kstar == -2 || ctl.consumed <= 0) {
+        h->broken = true;
+        return fail(h, MCA_ERR_NUMERIC, "non-finite loss change");
+      }
+      h->tau += (uint64_t)ctl.consumed;
+      remaining -= (uint64_t)ctl.consumed;
+      if (R > 0 && h->tau % R == 0) {
+        mca_status rc = resync(h);
+        if (rc != MCA_OK) return rc;
+        h->resyncs++;
+      }
+    }
+  }
   while (remaining > 0) {
     uint64_t seg = remaining;
     const uint64_t R = (uint64_t)h->opt.resync_period;
@@ -737,14 +860,25 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
                               h->stream));
   CUDA_TRY(h, cudaMemcpyAsync(h->ex_new, new_w, sizeof(float) * n, cudaMemcpyHostToDevice,
                               h->stream));
-  mca::Mlp2Args a = mlp2_args(h);
-  a.n_explicit = (int)n;
-  a.ex_idx = h->ex_idx;
-  a.ex_new = h->ex_new;
-  a.ex_out = h->ex_out;
-  CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
-  CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
-  h->launches++;
+  if (h->deep) {
+    mca::DeepArgs a = deep_args(h);
+    a.n_explicit = (int)n;
+    a.ex_idx = h->ex_idx;
+    a.ex_new = h->ex_new;
+    a.ex_out = h->ex_out;
+    CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
+    CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
+    h->launches += 2;
+  } else {
+    mca::Mlp2Args a = mlp2_args(h);
+    a.n_explicit = (int)n;
+    a.ex_idx = h->ex_idx;
+    a.ex_new = h->ex_new;
+    a.ex_out = h->ex_out;
+    CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
+    CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
+    h->launches++;
+  }
   CUDA_TRY(h, cudaMemcpyAsync(dS, h->ex_out, sizeof(double) * n, cudaMemcpyDeviceToHost,
                               h->stream));
   CUDA_TRY(h, cudaStreamSynchronize(h->stream));

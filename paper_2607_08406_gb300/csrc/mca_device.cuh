@@ -37,6 +37,58 @@ __device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
 __device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >> 8) * 0x1p-24f; }
 
 // ------------------------------------------------------------------------------------------------
+// The new value of one weight (Eq. 1). wk: storage kind; weff / code / wfix: the layer's arrays;
+// off: the weight's offset in its layer; r1: the trial's second Philox word.
+//   FP32:    replace by lo + (hi - lo) u, or perturb by delta (2u - 1); u = (r1 >> 8) 2^-24; the
+//            domain |w'| < bound (bound > 0) rejects without evaluation
+//   TERNARY: new code floor(r1 * 3 / 2^32) - 1, effective weight scale * code
+//   MASKED:  toggle the mask bit of the fixed weight
+// explicit_value: take ex_new as the new effective value instead (evaluation of given candidates).
+// ------------------------------------------------------------------------------------------------
+struct Mutation {
+  float oldw, neww;
+  int new_code;
+  int valid;
+};
+
+__device__ __forceinline__ Mutation draw_mutation(int wk, const float* weff,
+                                                  const signed char* code, const float* wfix,
+                                                  float sc, unsigned long long off, int op, float lo,
+                                                  float hi, float delta, float bound, uint32_t r1,
+                                                  bool explicit_value, float ex_new) {
+  Mutation m;
+  m.valid = 1;
+  m.new_code = 0;
+  m.oldw = weff[off];
+  if (explicit_value) {
+    m.neww = ex_new;
+  } else if (wk == MCA_W_TERNARY_I8) {
+    const int oc = code[off];
+    const int nc = (int)(((unsigned long long)r1 * 3ull) >> 32) - 1;
+    m.oldw = __fmul_rn(sc, (float)oc);
+    m.neww = __fmul_rn(sc, (float)nc);
+    m.new_code = nc;
+  } else if (wk == MCA_W_MASKED_FP32) {
+    const int om = code[off];
+    const int nm = 1 - om;
+    const float w = wfix[off];
+    m.oldw = om ? w : 0.0f;
+    m.neww = nm ? w : 0.0f;
+    m.new_code = nm;
+  } else {
+    const float u = __uint2float_rn(r1 >> 8) * 0x1p-24f;
+    if (op == MCA_OP_PERTURB) {
+      const float rr = __fsub_rn(__fmul_rn(2.0f, u), 1.0f);
+      m.neww = __fadd_rn(m.oldw, __fmul_rn(delta, rr));
+    } else {
+      m.neww = __fadd_rn(lo, __fmul_rn(__fsub_rn(hi, lo), u));
+    }
+    if (bound > 0.0f && !(fabsf(m.neww) < bound)) m.valid = 0;
+  }
+  return m;
+}
+
+// ------------------------------------------------------------------------------------------------
 // Transfer functions (Section 2) and losses (Eq. 2 with R = 0). ACT < 0 selects at run time.
 //
 // exp and log use the hardware base-2 units (__expf, __logf: a few ulp). tanh is its exponential

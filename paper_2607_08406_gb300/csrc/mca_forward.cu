@@ -138,10 +138,13 @@ __global__ void init_layer_kernel(int wkind, float scale, const float* __restric
 
 // C[M x Ncol] = A[M x K] * B[K x Ncol], row-major, fp32 FMA in ascending k. Ncol % 128 == 0,
 // ldb and ldc multiples of 4. 128x128 tile per CTA, 256 threads, 8x8 outputs per thread.
+// ACTB: the B operand enters as act(B) (the previous layer's activations from its fields).
+template <bool ACTB>
 __global__ void __launch_bounds__(256) sgemm_nn_kernel(int M, int Ncol, int K,
                                                        const float* __restrict__ A, int lda,
                                                        const float* __restrict__ B, int ldb,
-                                                       float* __restrict__ C, int ldc) {
+                                                       float* __restrict__ C, int ldc, int bact,
+                                                       float bg) {
   constexpr int BM = 128, BN = 128, BK = 8;
   __shared__ __align__(16) float As[BK][BM];
   __shared__ __align__(16) float Bs[BK][BN];
@@ -164,7 +167,15 @@ __global__ void __launch_bounds__(256) sgemm_nn_kernel(int M, int Ncol, int K,
     {
       const int kk = k0 + bkk;
       float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (kk < K) v = *reinterpret_cast<const float4*>(B + (size_t)kk * ldb + bn + bcol);
+      if (kk < K) {
+        v = *reinterpret_cast<const float4*>(B + (size_t)kk * ldb + bn + bcol);
+        if (ACTB) {
+          v.x = act_rt(bact, v.x, bg);
+          v.y = act_rt(bact, v.y, bg);
+          v.z = act_rt(bact, v.z, bg);
+          v.w = act_rt(bact, v.w, bg);
+        }
+      }
       *reinterpret_cast<float4*>(&Bs[bkk][bcol]) = v;
     }
     __syncthreads();
@@ -232,11 +243,10 @@ __global__ void __launch_bounds__(128) mlp2_outputs_kernel(Mlp2Args a, const int
 }
 
 // S = sum_n loss_n in fp64, one CTA, fixed order.
-__global__ void __launch_bounds__(1024) sum_loss_kernel(const float* __restrict__ srec, int N,
-                                                        int Np, DevState* st) {
+__global__ void __launch_bounds__(1024) sum_loss_kernel(const float* __restrict__ ell, int N,
+                                                        DevState* st) {
   __shared__ double red[32];
   double s = 0.0;
-  const float* ell = srec + (size_t)kRecLoss * Np;
   for (int n = threadIdx.x; n < N; n += blockDim.x) s += (double)ell[n];
   s = block_sum_d(s, red);
   if (threadIdx.x == 0) st->S = s;
@@ -291,12 +301,25 @@ cudaError_t launch_init_layer(int wkind, float scale, const float* src, const si
 cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, const float* B,
                             int ldb, float* C, int ldc, cudaStream_t s) {
   dim3 grid(Ncol / 128, (M + 127) / 128);
-  sgemm_nn_kernel<<<grid, 256, 0, s>>>(M, Ncol, K, A, lda, B, ldb, C, ldc);
+  sgemm_nn_kernel<false><<<grid, 256, 0, s>>>(M, Ncol, K, A, lda, B, ldb, C, ldc, 0, 0.0f);
   return cudaGetLastError();
 }
 
-cudaError_t launch_sum_loss(const float* srec, int N, int Np, DevState* st, cudaStream_t s) {
-  sum_loss_kernel<<<1, 1024, 0, s>>>(srec, N, Np, st);
+// Fields of deep layer l from the previous layer (or X for l = 0): Z_l = W_l act_{l-1}(Z_{l-1}).
+cudaError_t launch_deep_forward_layer(const DeepArgs& a, int l, cudaStream_t s) {
+  const int M = a.n_out[l], K = a.n_in[l];
+  dim3 grid(a.Np / 128, (M + 127) / 128);
+  if (l == 0)
+    sgemm_nn_kernel<false><<<grid, 256, 0, s>>>(M, a.Np, K, a.w[0], K, a.XT, a.Np, a.Z[0], a.Np, 0,
+                                                0.0f);
+  else
+    sgemm_nn_kernel<true><<<grid, 256, 0, s>>>(M, a.Np, K, a.w[l], K, a.Z[l - 1], a.Np, a.Z[l],
+                                               a.Np, a.act[l - 1], a.g[l - 1]);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sum_loss(const float* ell, int N, DevState* st, cudaStream_t s) {
+  sum_loss_kernel<<<1, 1024, 0, s>>>(ell, N, st);
   return cudaGetLastError();
 }
 

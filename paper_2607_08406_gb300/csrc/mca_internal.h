@@ -77,6 +77,69 @@ struct Mlp2Args {
   double* ex_out;
 };
 
+// ------------------------------------------------------------------------------------------------
+// Deep MLP path (three or more weight layers): every layer's fields are cached; a candidate in layer
+// l updates row j of layer l, then layer l+1 by one weight column (rank-1), then recomputes the layers
+// from l+2 on as  Z'_m = Z_m + W_m (f(Z'_{m-1}) - f(Z_{m-1}))  over tiles of kDeepTS samples.
+// ------------------------------------------------------------------------------------------------
+constexpr int kMaxLayers = 32;
+constexpr int kDeepTS = 64;        // samples per tile
+constexpr int kDeepThreads = 256;
+constexpr int kDeepMaxWidth = 256; // widths of the layers inside the dense chain
+constexpr int kDeepKC = 16;        // weight-tile depth of the chain GEMM
+
+struct DeepCand {
+  unsigned int idx;
+  int layer, row, col;
+  float oldw, neww, delta;
+  int new_code, valid;
+};
+
+// Decision of the last batch, written by the decide kernel and read by the commit kernel and host.
+struct DeepCtl {
+  int kstar;                 // accepted candidate, -1 none, -2 non-finite loss change
+  int consumed;              // trials consumed by the batch
+  DeepCand acc;              // the accepted candidate
+};
+
+struct DeepArgs {
+  int L, N, Np, D, C, ntiles;
+  int n_in[kMaxLayers], n_out[kMaxLayers], act[kMaxLayers], wk[kMaxLayers];
+  float g[kMaxLayers], sc[kMaxLayers];
+  unsigned long long off[kMaxLayers + 1];
+  float* w[kMaxLayers];
+  signed char* code[kMaxLayers];
+  const float* wfix[kMaxLayers];
+  float* Z[kMaxLayers];      // [n_out[l] x Np] fields of layer l; Z[L-1] are the output fields
+  const float* XT;           // [D x Np]
+  float* ell;                // [Np] per-sample loss
+  const int* y;
+  int loss;
+  int op;
+  float lo, hi, delta, bound;
+  int strict;
+  unsigned long long seed, tau;
+  int Kb;
+  float* partial;            // [kKmax x ntiles]
+  DevState* st;
+  DeepCtl* ctl;
+  mca_trace_rec* trace;
+  int trace_cap;
+  const unsigned long long* ftau;
+  const unsigned char* facc;
+  int nforce;
+  int n_explicit;
+  const unsigned int* ex_idx;
+  const float* ex_new;
+  double* ex_out;
+};
+
+cudaError_t launch_deep_eval(const DeepArgs& a, cudaStream_t s);    // grid (Kb, ntiles)
+cudaError_t launch_deep_decide(const DeepArgs& a, cudaStream_t s);  // one CTA
+cudaError_t launch_deep_commit(const DeepArgs& a, cudaStream_t s);  // grid ntiles
+cudaError_t launch_deep_forward_layer(const DeepArgs& a, int l, cudaStream_t s);
+cudaError_t launch_deep_losses(const DeepArgs& a, cudaStream_t s);
+
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
 cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
 cudaError_t launch_csr_count(const float* XT, int Np, int N, int D, int* cnt, cudaStream_t s);
@@ -92,7 +155,8 @@ cudaError_t launch_init_layer(int wkind, float scale, const float* src, const si
 cudaError_t launch_sgemm_nn(int M, int Ncol, int K, const float* A, int lda, const float* B,
                             int ldb, float* C, int ldc, cudaStream_t s);
 cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s);
-cudaError_t launch_sum_loss(const float* srec, int N, int Np, DevState* st, cudaStream_t s);
+// S = sum of ell[0 .. N) in fp64 (fixed order) into st->S.
+cudaError_t launch_sum_loss(const float* ell, int N, DevState* st, cudaStream_t s);
 // Cooperative persistent trial loop, one CTA per sample range (grid = NR).
 cudaError_t launch_mlp2_loop(const Mlp2Args& a, cudaStream_t s);
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);
@@ -138,6 +202,12 @@ struct mca_handle {
   std::vector<float*> wfix;
   float* z1 = nullptr;
   float* srec = nullptr;
+  // deep path
+  bool deep = false;
+  std::vector<float*> Z;
+  float* ell = nullptr;
+  mca::DeepCtl* ctl = nullptr;
+  int ntiles = 0;
   float* partial = nullptr;
   int NR = 0, RS = 0, SUB = 0, smem_records = 0;
   mca::GridBarrier* bar = nullptr;

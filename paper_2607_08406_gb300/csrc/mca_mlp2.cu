@@ -52,39 +52,14 @@ __device__ __forceinline__ void fill_candidate(const Mlp2Args& a, unsigned int i
   c.layer = layer;
   c.row = (int)(off / (unsigned long long)n_in);
   c.col = (int)(off % (unsigned long long)n_in);
-  const int wk = layer ? a.wk2 : a.wk1;
-  const float* weff = layer ? a.w2 : a.w1;
-  const signed char* code = layer ? a.code2 : a.code1;
-  const float* wfix = layer ? a.wfix2 : a.wfix1;
-  const float sc = layer ? a.sc2 : a.sc1;
-  c.valid = 1;
-  c.new_code = 0;
-  c.oldw = weff[off];
-  if (explicit_value) {
-    c.neww = ex_new;
-  } else if (wk == MCA_W_TERNARY_I8) {
-    const int oc = code[off];
-    const int nc = (int)(((unsigned long long)r1 * 3ull) >> 32) - 1;
-    c.oldw = __fmul_rn(sc, (float)oc);
-    c.neww = __fmul_rn(sc, (float)nc);
-    c.new_code = nc;
-  } else if (wk == MCA_W_MASKED_FP32) {
-    const int om = code[off];
-    const int nm = 1 - om;
-    const float w = wfix[off];
-    c.oldw = om ? w : 0.0f;
-    c.neww = nm ? w : 0.0f;
-    c.new_code = nm;
-  } else {
-    const float u = unit24(r1);
-    if (a.op == MCA_OP_PERTURB) {
-      const float rr = __fsub_rn(__fmul_rn(2.0f, u), 1.0f);
-      c.neww = __fadd_rn(c.oldw, __fmul_rn(a.delta, rr));
-    } else {
-      c.neww = __fadd_rn(a.lo, __fmul_rn(__fsub_rn(a.hi, a.lo), u));
-    }
-    if (a.bound > 0.0f && !(fabsf(c.neww) < a.bound)) c.valid = 0;
-  }
+  const Mutation mu = draw_mutation(layer ? a.wk2 : a.wk1, layer ? a.w2 : a.w1,
+                                    layer ? a.code2 : a.code1, layer ? a.wfix2 : a.wfix1,
+                                    layer ? a.sc2 : a.sc1, off, a.op, a.lo, a.hi, a.delta, a.bound,
+                                    r1, explicit_value, ex_new);
+  c.oldw = mu.oldw;
+  c.neww = mu.neww;
+  c.new_code = mu.new_code;
+  c.valid = mu.valid;
   c.delta = __fsub_rn(c.neww, c.oldw);
   const int all = layer == 0 ? a.xs_off[c.col + 1] - a.xs_off[c.col] : a.N;
   // A zero change leaves every field bit-identical: dS = 0 exactly, nothing to evaluate.

@@ -64,6 +64,9 @@ extern "C" mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t*
   if (!flat_idx || !new_w || !dS) return set_err(h, MCA_ERR_INVALID, "NULL argument");
   if (h->broken)
     return set_err(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (h->deep)
+    return set_err(h, MCA_ERR_UNSUPPORTED,
+                   "the no-allocation evaluation runs single-hidden-layer handles only");
   if (n > (size_t)kNoAllocMaxCandidates)
     return set_err(h, MCA_ERR_INVALID,
                    "n = " + std::to_string(n) + " candidates exceeds the no-allocation maximum of " +
