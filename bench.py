@@ -249,14 +249,36 @@ def run_ours(args):
     trials_timed = (st1["trials"] - st0["trials"]) * world
     value = trials_timed / (total_ms / 1e3)
     launches = st1["launches"] - st0["launches"]
-    # dominant kernel: the trial loop (one launch per step when no resync falls in the step)
+    # dominant kernel: single hidden layer -- the trial loop (one launch per step when no resync
+    # falls in the step), HBM-bound; deep nets -- the candidate chains (SIMT fp32 FMA), whose
+    # FLOPs are divided by the whole step time (a lower bound: the step also holds the decide and
+    # commit kernels and one host round trip per batch)
+    deep = len(wl.layers) > 2
     peak, peak_kind = load_peaks()
-    bytes_timed = st1["alg_bytes"] - st0["alg_bytes"]
-    loop_launches = K
-    achieved = bytes_timed / loop_launches / (total_ms / K / 1e3) / 1e9
     traffic = None
-    if LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and LOOP_TRAFFIC["bytes_per_trial"]:
-        traffic = LOOP_TRAFFIC["bytes_per_trial"] * (st1["trials"] - st0["trials"]) / K
+    if deep:
+        sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
+        sm_max = float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["sm_max_mhz"]) \
+            if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else 2070.0
+        peak = sms * 128 * 2 * sm_max * 1e6 / 1e12        # fp32 FMA lanes x 2 FLOP x clock
+        peak_kind = f"derived: {sms} SMs x 128 fp32 lanes x 2 FLOP x {sm_max:.0f} MHz"
+        flops_timed = st1["alg_flops"] - st0["alg_flops"]
+        achieved = flops_timed / (total_ms / 1e3) / 1e12
+        roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "traffic": None, "kernel": "deep_chain_kernel",
+                    "peak_kind": peak_kind,
+                    "flops": "FLOPs of the evaluated candidates' recomputation, counted by the "
+                             "library, over the whole step time"}
+    else:
+        bytes_timed = st1["alg_bytes"] - st0["alg_bytes"]
+        achieved = bytes_timed / K / (total_ms / K / 1e3) / 1e9
+        if LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and LOOP_TRAFFIC["bytes_per_trial"]:
+            traffic = LOOP_TRAFFIC["bytes_per_trial"] * (st1["trials"] - st0["trials"]) / K
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                    "frac": achieved / peak, "traffic": traffic, "kernel": "mlp2_trial_loop",
+                    "peak_kind": peak_kind,
+                    "bytes": "compulsory DRAM bytes of the distinct candidates evaluated, "
+                             "counted by the kernel (per launch)"}
     loss_end = mca.mca_loss(h)
     h.close()
 
@@ -312,10 +334,12 @@ def run_ours(args):
             "warmup": W_, "ms_per_step": total_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": wl.name, "N": wl.N, "hidden": wl.layers[0].n_out,
+                       "layers": len(wl.layers),
                        "K": wl.K, "trials_per_step": T,
                        "trial_range": [W_ * T, (W_ + K) * T], "seed": args.seed,
                        "resync_period": args.resync, "resync_ms": resync_ms,
-                       "l2": "no flush: cached hidden fields (3.9 GB) exceed L2",
+                       "l2": "no flush: the cached fields exceed L2" if not deep else
+                             "no flush: the cached fields of all layers (256 MB) exceed L2",
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
@@ -324,11 +348,7 @@ def run_ours(args):
                                                             "reduce_decide", "commit"])},
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": traffic,
-                         "kernel": "mlp2_trial_loop", "peak_kind": peak_kind,
-                         "bytes": "compulsory DRAM bytes of the distinct candidates evaluated, "
-                                  "counted by the kernel (per launch)"},
+            "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
             "clocks": clk.summary(),

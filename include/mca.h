@@ -112,6 +112,10 @@ typedef struct {
                               caller-owned device buffer of >= mca_workspace_size() bytes,
                               256-byte aligned, that must outlive the handle */
   size_t workspace_bytes;
+  int32_t fixed_K;         /* 0: each batch evaluates ceil(c / p) candidates, at most K, where p is
+                              the recently observed acceptance rate per trial (fewer discarded
+                              candidates while many are accepted; the trajectory is the same);
+                              1: every batch evaluates K candidates */
 } mca_options;
 
 typedef struct {
@@ -133,6 +137,8 @@ typedef struct {
                               first-layer candidate the sectors written back */
   uint64_t phase_ns[4];    /* device time of the trial loop's first CTA in: propose + evaluate,
                               grid barrier, reduce + decide, commit */
+  uint64_t alg_flops;      /* deep nets: FLOPs of the evaluated candidates' recomputation (2 per
+                              multiply-add: the row update, the rank-1 layer, the dense layers) */
 } mca_run_stats;
 
 typedef struct {

@@ -303,6 +303,7 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.bound = h->dom.bound;
   a.strict = h->dom.strict;
   a.K = h->opt.K;
+  a.fixed_K = h->opt.fixed_K;
   a.partial = h->partial;
   a.bar = h->bar;
   a.st = h->st;
@@ -439,6 +440,7 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
   s->S = d.S;
   s->alg_bytes = d.alg_bytes;
   for (int q = 0; q < 4; ++q) s->phase_ns[q] = d.phase_ns[q];
+  s->alg_flops = d.alg_flops;
 }
 
 }  // namespace
@@ -678,7 +680,10 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     a.seed = seed;
     const uint64_t R = (uint64_t)h->opt.resync_period;
     while (remaining > 0) {
-      uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)h->opt.K);
+      const int Kw = h->opt.fixed_K ? h->opt.K
+                                    : mca::batch_width(h->rate_acc, h->rate_trials,
+                                                       mca::kWidthDeep, h->opt.K);
+      uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)Kw);
       if (R > 0) kb = std::min<uint64_t>(kb, R - h->tau % R);
       a.tau = h->tau;
       a.Kb = (int)kb;
@@ -695,6 +700,8 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
       }
       h->tau += (uint64_t)ctl.consumed;
       remaining -= (uint64_t)ctl.consumed;
+      h->rate_acc = h->rate_acc * mca::kRateDecay + (ctl.kstar >= 0 ? 1.0f : 0.0f);
+      h->rate_trials = h->rate_trials * mca::kRateDecay + (float)ctl.consumed;
       if (R > 0 && h->tau % R == 0) {
         mca_status rc = resync(h);
         if (rc != MCA_OK) return rc;

@@ -373,9 +373,21 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
     if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
     st->forced += (unsigned long long)__popc(m);
   }
-  unsigned long long ncand = 0;
-  for (int q = 0; q < Kb; ++q) ncand += s_c[q].valid ? 1ull : 0ull;
+  // FLOPs of the evaluated chains: row update (2 per sample), rank-1 into layer l+1
+  // (2 n_out[l+1] per sample), dense layers m = l+2 .. L-1 (2 n_out[m] n_in[m] per sample)
+  unsigned long long ncand = 0, flops = 0;
+  for (int q = 0; q < Kb; ++q) {
+    const DeepCand& c = s_c[q];
+    ncand += c.valid ? 1ull : 0ull;
+    if (!c.valid || c.delta == 0.0f) continue;
+    unsigned long long per = 2ull;
+    if (c.layer + 1 < a.L) per += 2ull * (unsigned long long)a.n_out[c.layer + 1];
+    for (int m = c.layer + 2; m < a.L; ++m)
+      per += 2ull * (unsigned long long)a.n_out[m] * (unsigned long long)a.n_in[m];
+    flops += per * (unsigned long long)a.N;
+  }
   st->candidates += ncand;
+  st->alg_flops += flops;
   st->batches += 1ull;
   if (kstar >= 0) {
     const DeepCand& c = s_c[kstar];

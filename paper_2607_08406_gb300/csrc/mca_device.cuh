@@ -88,6 +88,14 @@ __device__ __forceinline__ Mutation draw_mutation(int wk, const float* weff,
   return m;
 }
 
+// Batch width from the decayed acceptance counts (the same arithmetic wherever it is evaluated, so
+// every CTA of a launch, and the host, agree).
+__host__ __device__ __forceinline__ int batch_width(float acc, float trials, float c, int K) {
+  const float p = (acc + 0.5f) / (trials + 1.0f);
+  const float w = ceilf(c / p);
+  return w >= (float)K ? K : (w < 1.0f ? 1 : (int)w);
+}
+
 // ------------------------------------------------------------------------------------------------
 // Transfer functions (Section 2) and losses (Eq. 2 with R = 0). ACT < 0 selects at run time.
 //

@@ -20,7 +20,11 @@ constexpr int kMaxClasses = kSR - 2;
 constexpr int kLoopThreads = 512; // threads per CTA of the trial-loop kernel
 constexpr int kLoopWarps = kLoopThreads / 32;
 constexpr int kMaxSubs = 8;       // sub-chunks of one candidate inside one sample range
-constexpr int kRangeTarget = 64;  // samples per range below which fewer CTAs are used
+constexpr int kRangeTarget = 64;
+// Batch width: ceil(c / p) candidates, p = (A + 0.5) / (T + 1) from counts decayed per batch.
+constexpr float kRateDecay = 0.95f;
+constexpr float kWidthMlp2 = 3.0f;
+constexpr float kWidthDeep = 1.5f;  // samples per range below which fewer CTAs are used
 constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
 
 // Device-resident run state (one per handle).
@@ -29,6 +33,8 @@ struct DevState {
   unsigned long long trials, accepts, candidates, batches, wasted, forced, trace_written;
   unsigned long long alg_bytes;  // compulsory DRAM bytes of the evaluated candidates and commits
   unsigned long long phase_ns[4];  // CTA 0: propose+evaluate, barrier, reduce+decide, commit
+  unsigned long long alg_flops;    // deep path: FLOPs of the evaluated candidates' chains
+  float rate_acc, rate_trials;     // decayed counts of accepts and trials (batch-width choice)
   int err;                   // first device-side error (mca_status), 0 = none
   int pad;
 };
@@ -63,6 +69,7 @@ struct Mlp2Args {
   int strict;
   unsigned long long seed, tau0, n_trials;
   int K;
+  int fixed_K;
   float* partial;            // [2 x kKmax x NR] per-candidate, per-range loss changes
   GridBarrier* bar;
   DevState* st;
@@ -225,4 +232,5 @@ struct mca_handle {
   unsigned long long tau = 0;
   unsigned long long launches = 0, resyncs = 0;
   bool broken = false;                   // a sticky CUDA error or device timeout was seen
+  float rate_acc = 0.0f, rate_trials = 0.0f;   // deep path: acceptance counts (batch width)
 };

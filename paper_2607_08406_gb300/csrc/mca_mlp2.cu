@@ -289,14 +289,17 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   unsigned int gen = 0;
   unsigned long long tau = a.tau0;
   if (tid == 0) s_tau_hi = a.tau0;
+  // acceptance-rate estimate behind the batch width: the same in every CTA
+  float rate_a = st->rate_acc, rate_t = st->rate_trials;
   const unsigned long long end = a.tau0 + a.n_trials;
   int buf = 0;
   __syncthreads();
 
   while (explicit_mode || tau < end) {
     const unsigned long long t_a = stats_thread ? globaltimer_ns() : 0ull;
+    const int Kw = a.fixed_K ? a.K : batch_width(rate_a, rate_t, kWidthMlp2, a.K);
     const int Kb = explicit_mode ? a.n_explicit
-                                 : (int)((end - tau) < (unsigned long long)a.K ? (end - tau) : a.K);
+                                 : (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
     // ---- propose: every CTA draws every candidate
     for (int k = tid; k < Kb; k += kLoopThreads) {
       Cand c;
@@ -563,9 +566,13 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
       __syncthreads();
       if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
       tau += (unsigned long long)(kstar + 1);
+      rate_a = rate_a * kRateDecay + 1.0f;
+      rate_t = rate_t * kRateDecay + (float)(kstar + 1);
     } else {
       if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
       tau += (unsigned long long)Kb;
+      rate_a = rate_a * kRateDecay;
+      rate_t = rate_t * kRateDecay + (float)Kb;
     }
     if (stats_thread) {
       const unsigned long long t_e = globaltimer_ns();
@@ -600,6 +607,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
     st->phase_ns[1] += ph1;
     st->phase_ns[2] += ph2;
     st->phase_ns[3] += ph3;
+    st->rate_acc = rate_a;
+    st->rate_trials = rate_t;
   }
 }
 

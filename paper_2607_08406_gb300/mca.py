@@ -42,14 +42,14 @@ class mca_dataset(Structure):
 class mca_options(Structure):
     _fields_ = [("K", c_int32), ("resync_period", c_int32), ("stream", c_void_p),
                 ("trace_cap", c_int32), ("grid", c_int32), ("workspace", c_void_p),
-                ("workspace_bytes", c_size_t)]
+                ("workspace_bytes", c_size_t), ("fixed_K", c_int32)]
 
 
 class mca_run_stats(Structure):
     _fields_ = [("trials", c_uint64), ("accepts", c_uint64), ("candidates", c_uint64),
                 ("batches", c_uint64), ("wasted", c_uint64), ("forced", c_uint64),
                 ("resyncs", c_uint64), ("launches", c_uint64), ("tau", c_uint64), ("S", c_double),
-                ("alg_bytes", c_uint64), ("phase_ns", c_uint64 * 4)]
+                ("alg_bytes", c_uint64), ("phase_ns", c_uint64 * 4), ("alg_flops", c_uint64)]
 
     def asdict(self):
         d = {f: getattr(self, f) for f, _ in self._fields_ if f != "phase_ns"}
@@ -167,7 +167,7 @@ def mca_workspace_size(layers, loss: str, X, y, K: int = 32, trace_cap: int = 0,
     lib = load_library()
     L = _layers(layers)
     ds = mca_dataset(_ptr(X), _ptr(y), int(X.shape[0]), int(X.shape[1]))
-    opt = mca_options(K, 0, stream, trace_cap, 0, None, 0)
+    opt = mca_options(K, 0, stream, trace_cap, 0, None, 0, 0)
     out = c_size_t(0)
     _check(lib.mca_workspace_size(L, len(layers), LOSS[loss], ctypes.byref(ds), ctypes.byref(opt),
                                   ctypes.byref(out)))
@@ -175,7 +175,8 @@ def mca_workspace_size(layers, loss: str, X, y, K: int = 32, trace_cap: int = 0,
 
 
 def mca_create(layers, loss: str, domain, X, y, init, K: int = 32, resync_period: int = 0,
-               trace_cap: int = 0, grid: int = 0, stream=None, torch_workspace: bool = True):
+               trace_cap: int = 0, grid: int = 0, stream=None, torch_workspace: bool = True,
+               fixed_K: bool = False):
     """X: [N, D] float32, y: [N] int32, init: [P] float32 -- torch tensors (CUDA or CPU) or numpy
     arrays. The workspace is a torch CUDA tensor the handle keeps alive."""
     import torch
@@ -194,7 +195,7 @@ def mca_create(layers, loss: str, domain, X, y, init, K: int = 32, resync_period
         ws_ptr = (base + 255) // 256 * 256
         ws_bytes = nbytes
         keep.append(ws)
-    opt = mca_options(K, resync_period, stream, trace_cap, grid, ws_ptr, ws_bytes)
+    opt = mca_options(K, resync_period, stream, trace_cap, grid, ws_ptr, ws_bytes, int(fixed_K))
     h = c_void_p(None)
     _check(lib.mca_create(L, len(layers), LOSS[loss], ctypes.byref(dom), ctypes.byref(ds),
                           _ptr(init), ctypes.byref(opt), ctypes.byref(h)))
