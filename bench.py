@@ -217,7 +217,8 @@ def run_ours(args):
     yd = torch.from_numpy(wl.y).cuda()
     initd = torch.from_numpy(wl.init).cuda()
     h = mca.mca_create(wl.layers, wl.loss, wl.domain, Xd, yd, initd, K=wl.K,
-                       resync_period=args.resync, stream=stream.cuda_stream)
+                       resync_period=args.resync, stream=stream.cuda_stream, grid=args.grid,
+                       fixed_K=args.fixed_K)
     # one full forward pass (the resync step), timed on its own
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -294,7 +295,8 @@ def run_ours(args):
 
         def job():
             hh = mca.mca_create(wl.layers, wl.loss, wl.domain, Xh, yh, ih, K=wl.K,
-                                resync_period=args.resync, stream=stream.cuda_stream)
+                                resync_period=args.resync, stream=stream.cuda_stream,
+                                grid=args.grid, fixed_K=args.fixed_K)
             mca.mca_run(hh, e2e_trials, wl.seed)
             mca.mca_get_params(hh, wl.n_params, out)
             lv = mca.mca_loss(hh)
@@ -373,6 +375,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--trials-per-step", dest="trials_per_step", type=int, default=0)
     ap.add_argument("--resync", type=int, default=0)
+    ap.add_argument("--grid", type=int, default=0)
+    ap.add_argument("--fixed-K", dest="fixed_K", action="store_true")
     ap.add_argument("--cpu-trials", dest="cpu_trials", type=int, default=2000)
     ap.add_argument("--ref-trials", dest="ref_trials", type=int, default=200)
     ap.add_argument("--e2e-steps", dest="e2e_steps", type=int, default=1)

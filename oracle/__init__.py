@@ -6,3 +6,4 @@ check the CUDA path. Only the tests, ``__graft_entry__.smoke()`` and the ``cpu_b
 its Python binding) never imports, links or calls anything in here, and it shares no code with it.
 """
 from .mca_oracle import *  # noqa: F401,F403
+from .mca_tfm import *  # noqa: F401,F403

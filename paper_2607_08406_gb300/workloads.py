@@ -203,3 +203,103 @@ MLP_WORKLOADS = {
 def make(name: str, **kw) -> MLPWorkload:
     return MLP_WORKLOADS[name](**kw)
 
+
+
+# ------------------------------------------------------------------------------------------------
+# Character-level Transformer workload (stand-in for Tiny Shakespeare, Section 2.5)
+# ------------------------------------------------------------------------------------------------
+
+@dataclass
+class TfmSpec:
+    vocab: int = 65
+    ctx: int = 64
+    d_model: int = 128
+    n_layer: int = 2
+    n_head: int = 4
+    d_ff: int = 512
+    act: str = "gelu"           # FFN transfer function: "gelu" (exact erf) or "gaussian"
+    act_param: float = 1.0      # gamma of the Gaussian
+    ln_eps: float = 1e-5
+
+    def blocks(self):
+        """Flat parameter layout: (name, shape) in order. Matrices are [out x in] row-major."""
+        d, f, v, t = self.d_model, self.d_ff, self.vocab, self.ctx
+        out = [("tok_emb", (v, d)), ("pos_emb", (t, d))]
+        for b in range(self.n_layer):
+            out += [(f"b{b}.ln1.g", (d,)), (f"b{b}.ln1.b", (d,)),
+                    (f"b{b}.wq", (d, d)), (f"b{b}.bq", (d,)),
+                    (f"b{b}.wk", (d, d)), (f"b{b}.bk", (d,)),
+                    (f"b{b}.wv", (d, d)), (f"b{b}.bv", (d,)),
+                    (f"b{b}.wo", (d, d)), (f"b{b}.bo", (d,)),
+                    (f"b{b}.ln2.g", (d,)), (f"b{b}.ln2.b", (d,)),
+                    (f"b{b}.w1", (f, d)), (f"b{b}.b1", (f,)),
+                    (f"b{b}.w2", (d, f)), (f"b{b}.b2", (d,))]
+        out += [("lnf.g", (d,)), ("lnf.b", (d,)), ("w_head", (v, d)), ("b_head", (v,))]
+        return out
+
+    @property
+    def n_params(self) -> int:
+        return int(sum(np.prod(s) for _, s in self.blocks()))
+
+
+@dataclass
+class TfmWorkload:
+    name: str
+    spec: TfmSpec
+    tokens: np.ndarray          # [B, ctx + 1] int32: inputs tokens[:, :ctx], targets tokens[:, 1:]
+    init: np.ndarray            # [P] float32, flat layout of spec.blocks()
+    n_trials: int
+    K: int
+    seed: int = 0
+    domain: Domain = field(default_factory=Domain)
+
+    @property
+    def n_params(self) -> int:
+        return self.spec.n_params
+
+
+def markov_text(rng: np.random.Generator, vocab: int, length: int, alpha: float = 0.1):
+    """A stream of `length` symbols from an order-2 Markov chain over `vocab` symbols whose
+    transition rows are Dirichlet(alpha) draws; the first two symbols are uniform."""
+    rows = rng.dirichlet(np.full(vocab, alpha), size=vocab * vocab)
+    cdf = np.cumsum(rows, axis=1)
+    cdf[:, -1] = 1.0
+    u = rng.random(length)
+    out = np.empty(length, dtype=np.int32)
+    out[:2] = rng.integers(0, vocab, 2)
+    for t in range(2, length):
+        r = out[t - 2] * vocab + out[t - 1]
+        out[t] = min(int(np.searchsorted(cdf[r], u[t], side="right")), vocab - 1)
+    return out
+
+
+def tfm_init(rng: np.random.Generator, spec: TfmSpec, std: float = 0.02) -> np.ndarray:
+    """GPT-style initialisation: N(0, std) matrices and embeddings, zero biases, LN gains 1."""
+    parts = []
+    for name, shape in spec.blocks():
+        n = int(np.prod(shape))
+        if name.endswith(".g"):
+            parts.append(np.ones(n, np.float32))
+        elif len(shape) == 1:
+            parts.append(np.zeros(n, np.float32))
+        else:
+            parts.append(rng.normal(0.0, std, n).astype(np.float32))
+    return np.ascontiguousarray(np.concatenate(parts).astype(np.float32))
+
+
+def char_transformer(seed: int = 0, batch: int = 256, text_len: int = 1_000_000,
+                     spec: Optional[TfmSpec] = None, n_trials: int = 500_000,
+                     K: int = 64) -> TfmWorkload:
+    """Tiny char-level Transformer: vocab 65, context 64, d_model 128, 2 pre-LN blocks of 4 heads,
+    FFN 512 (exact GELU), learned positions, untied head; next-char CE over a fixed batch of 256
+    windows of an order-2 Markov stream (Dirichlet(0.1) rows, 1M symbols)."""
+    wid = 6
+    spec = spec or TfmSpec()
+    rng = _rng(wid, seed, _S_X)
+    text = markov_text(rng, spec.vocab, text_len)
+    starts = _rng(wid, seed, _S_TEACHER).integers(0, text_len - spec.ctx - 1, batch)
+    tokens = np.stack([text[s:s + spec.ctx + 1] for s in starts]).astype(np.int32)
+    init = tfm_init(_rng(wid, seed, _S_INIT), spec)
+    name = (f"gpt_v{spec.vocab}_t{spec.ctx}_d{spec.d_model}_l{spec.n_layer}_h{spec.n_head}"
+            f"_f{spec.d_ff}_b{batch}")
+    return TfmWorkload(name, spec, np.ascontiguousarray(tokens), init, n_trials, K, seed)
