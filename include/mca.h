@@ -152,6 +152,21 @@ typedef struct {
   double S;                /* loss sum before the trial */
 } mca_trace_rec;
 
+/* Character-level Transformer (Section 2.5): token + learned position embeddings, n_layer pre-LN
+ * blocks (causal multi-head self-attention; feed-forward d_model -> d_ff -> d_model with act =
+ * MCA_ACT_GELU or MCA_ACT_GAUSSIAN), a final LN and an untied head; loss = sum over positions of the
+ * next-token softmax cross-entropy. Limits of this build: ctx <= 64, d_model <= 128,
+ * d_model / n_head <= 64, vocab <= 128, n_layer <= 8.
+ * Flat parameter order (matrices [out x in] row-major): tok_emb [vocab x d], pos_emb [ctx x d];
+ * per block: ln1.g [d], ln1.b [d], wq [d x d], bq [d], wk, bk, wv, bv, wo, bo, ln2.g, ln2.b,
+ * w1 [d_ff x d], b1 [d_ff], w2 [d x d_ff], b2 [d]; then lnf.g, lnf.b, w_head [vocab x d], b_head. */
+typedef struct {
+  int32_t vocab, ctx, d_model, n_layer, n_head, d_ff;
+  int32_t act;
+  float act_param;
+  float ln_eps;
+} mca_tfm_spec;
+
 typedef struct mca_handle mca_handle;
 
 /* Bytes of device workspace mca_create needs for this spec and dataset (counts the non-zeros of
@@ -170,6 +185,18 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
 mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
                       const mca_domain* dom, const mca_dataset* data, const float* init_params,
                       const mca_options* opt, mca_handle** out);
+
+/* Bytes of device workspace mca_create_transformer needs. */
+mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const mca_options* opt,
+                                  size_t* bytes);
+
+/* Build a trial loop for the Transformer `spec` on n_seq fixed sequences. tokens: [n_seq x (ctx+1)]
+ * int32, host or device (inputs tokens[:, :ctx], targets tokens[:, 1:]); init_params: [P] fp32,
+ * host or device, in the flat order above. Every parameter is an fp32 weight (Eq. 1 replacement or
+ * perturbation). mca_loss reports S / (n_seq * ctx). Errors as for mca_create. */
+mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
+                                  const int32_t* tokens, int64_t n_seq, const float* init_params,
+                                  const mca_options* opt, mca_handle** out);
 
 /* Run n_trials sequential trials tau, tau+1, ... (Eq. 1 proposals drawn from Philox4x32-10 with
  * key = seed and counter = tau; Eq. 6 selection). Returns when they are done. stats: nullable.

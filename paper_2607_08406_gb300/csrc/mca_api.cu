@@ -361,7 +361,16 @@ mca::DeepArgs deep_args(mca_handle* h) {
 }
 
 // Full forward pass: every cached field, every sample's loss, and S (Section 2.4's cache).
+mca::TfmArgs tfm_args(mca_handle* h);
+
 mca_status resync(mca_handle* h) {
+  if (h->tfm) {
+    const mca::TfmArgs a = tfm_args(h);
+    CUDA_TRY(h, mca::launch_tfm_forward(a, h->stream));
+    CUDA_TRY(h, mca::launch_sum_loss(h->ell, a.B, h->st, h->stream));
+    h->launches += 2;
+    return MCA_OK;
+  }
   if (h->deep) {
     const mca::DeepArgs a = deep_args(h);
     for (int l = 0; l < a.L; ++l) CUDA_TRY(h, mca::launch_deep_forward_layer(a, l, h->stream));
@@ -441,6 +450,135 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
   s->alg_bytes = d.alg_bytes;
   for (int q = 0; q < 4; ++q) s->phase_ns[q] = d.phase_ns[q];
   s->alg_flops = d.alg_flops;
+}
+
+// ---------------------------------------------------------------- Transformer handles
+
+struct TfmLayout {
+  unsigned long long o_tok, o_pos, o_blk0, blk, o_lnf_g, o_lnf_b, o_wh, o_bh, P;
+  unsigned int r[16];        // ln1g ln1b wq bq wk bk wv bv wo bo ln2g ln2b w1 b1 w2 b2
+};
+
+TfmLayout tfm_offsets(const mca_tfm_spec& t) {
+  TfmLayout L;
+  const unsigned long long d = t.d_model, f = t.d_ff, v = t.vocab, c = t.ctx;
+  L.o_tok = 0;
+  L.o_pos = v * d;
+  L.o_blk0 = L.o_pos + c * d;
+  const unsigned long long sizes[16] = {d, d, d * d, d, d * d, d, d * d, d, d * d, d, d, d,
+                                        f * d, f, d * f, d};
+  unsigned long long o = 0;
+  for (int q = 0; q < 16; ++q) {
+    L.r[q] = (unsigned int)o;
+    o += sizes[q];
+  }
+  L.blk = o;
+  L.o_lnf_g = L.o_blk0 + (unsigned long long)t.n_layer * L.blk;
+  L.o_lnf_b = L.o_lnf_g + d;
+  L.o_wh = L.o_lnf_b + d;
+  L.o_bh = L.o_wh + v * d;
+  L.P = L.o_bh + v;
+  return L;
+}
+
+mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
+  if (!t) return fail(nullptr, MCA_ERR_INVALID, "spec is NULL");
+  if (n_seq <= 0 || n_seq > 65535) return fail(nullptr, MCA_ERR_INVALID, "n_seq outside 1..65535");
+  if (t->vocab < 2 || t->ctx < 1 || t->d_model < 1 || t->n_layer < 1 || t->n_head < 1 ||
+      t->d_ff < 1)
+    return fail(nullptr, MCA_ERR_INVALID, "bad transformer sizes");
+  if (t->d_model % t->n_head != 0) return fail(nullptr, MCA_ERR_INVALID, "d_model % n_head != 0");
+  if (t->act != MCA_ACT_GELU && t->act != MCA_ACT_GAUSSIAN)
+    return fail(nullptr, MCA_ERR_INVALID, "feed-forward act must be GELU or Gaussian");
+  if (!std::isfinite(t->act_param) || !(t->ln_eps > 0.0f))
+    return fail(nullptr, MCA_ERR_INVALID, "bad act_param or ln_eps");
+  if (t->ctx > mca::kTfmMaxT || t->d_model > mca::kTfmMaxD || t->vocab > mca::kTfmMaxV ||
+      t->d_model / t->n_head > 64 || t->n_layer > mca::kTfmMaxBlocks)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "transformer larger than this build supports");
+  if (mca::tfm_smem_bytes(t->ctx, t->d_model, t->d_model / t->n_head, t->vocab) > 227 * 1024)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "transformer tile exceeds shared memory");
+  if (tfm_offsets(*t).P >= (1ull << 32)) return fail(nullptr, MCA_ERR_INVALID, "P >= 2^32");
+  return MCA_OK;
+}
+
+struct TfmMem {
+  size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, scratch, total;
+};
+
+TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap) {
+  TfmMem M;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align256(o + bytes);
+    return at;
+  };
+  const TfmLayout L = tfm_offsets(t);
+  M.params = take(sizeof(float) * L.P);
+  M.tokens = take(sizeof(int) * (size_t)B * (t.ctx + 1));
+  M.X = take(sizeof(float) * (size_t)(t.n_layer + 1) * B * t.ctx * t.d_model);
+  M.ell = take(sizeof(float) * (size_t)B);
+  M.partial = take(sizeof(float) * (size_t)mca::kKmax * B);
+  M.st = take(sizeof(DevState));
+  M.ctl = take(sizeof(mca::DeepCtl));
+  M.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
+  M.ex_idx = take(sizeof(unsigned int) * mca::kKmax);
+  M.ex_new = take(sizeof(float) * mca::kKmax);
+  M.ex_out = take(sizeof(double) * mca::kKmax);
+  M.scratch = take(sizeof(int) * 8);
+  M.total = o;
+  return M;
+}
+
+mca::TfmArgs tfm_args(mca_handle* h) {
+  mca::TfmArgs a;
+  std::memset(&a, 0, sizeof(a));
+  const mca_tfm_spec& t = h->tspec;
+  const TfmLayout L = tfm_offsets(t);
+  a.V = t.vocab;
+  a.T = t.ctx;
+  a.d = t.d_model;
+  a.H = t.n_head;
+  a.dh = t.d_model / t.n_head;
+  a.F = t.d_ff;
+  a.nL = t.n_layer;
+  a.B = (int)(h->N / t.ctx);
+  a.eps = t.ln_eps;
+  a.act = t.act;
+  a.g = t.act_param;
+  a.o_tok = L.o_tok;
+  a.o_pos = L.o_pos;
+  a.o_blk0 = L.o_blk0;
+  a.blk_size = L.blk;
+  a.o_lnf_g = L.o_lnf_g;
+  a.o_lnf_b = L.o_lnf_b;
+  a.o_wh = L.o_wh;
+  a.o_bh = L.o_bh;
+  a.P = L.P;
+  unsigned int* r[16] = {&a.r_ln1g, &a.r_ln1b, &a.r_wq, &a.r_bq, &a.r_wk, &a.r_bk, &a.r_wv,
+                         &a.r_bv, &a.r_wo, &a.r_bo, &a.r_ln2g, &a.r_ln2b, &a.r_w1, &a.r_b1,
+                         &a.r_w2, &a.r_b2};
+  for (int q = 0; q < 16; ++q) *r[q] = L.r[q];
+  a.params = h->params;
+  a.tokens = h->tokens;
+  a.X = h->X;
+  a.ell = h->ell;
+  a.op = h->dom.op;
+  a.lo = h->dom.lo;
+  a.hi = h->dom.hi;
+  a.delta = h->dom.delta;
+  a.bound = h->dom.bound;
+  a.strict = h->dom.strict;
+  a.smem = mca::tfm_smem_bytes(a.T, a.d, a.dh, a.V);
+  a.partial = h->partial;
+  a.st = h->st;
+  a.ctl = h->ctl;
+  a.trace = h->trace;
+  a.trace_cap = h->trace_cap;
+  a.ftau = h->ftau;
+  a.facc = h->facc;
+  a.nforce = h->nforce;
+  return a;
 }
 
 }  // namespace
@@ -674,10 +812,12 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
   if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
   if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
   uint64_t remaining = n_trials;
-  if (h->deep) {
+  if (h->deep || h->tfm) {
     // one batch per round trip: evaluate, decide, commit, then read how many trials it consumed
-    mca::DeepArgs a = deep_args(h);
+    mca::DeepArgs a = h->deep ? deep_args(h) : mca::DeepArgs{};
+    mca::TfmArgs ta = h->tfm ? tfm_args(h) : mca::TfmArgs{};
     a.seed = seed;
+    ta.seed = seed;
     const uint64_t R = (uint64_t)h->opt.resync_period;
     while (remaining > 0) {
       const int Kw = h->opt.fixed_K ? h->opt.K
@@ -685,11 +825,19 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
                                                        mca::kWidthDeep, h->opt.K);
       uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)Kw);
       if (R > 0) kb = std::min<uint64_t>(kb, R - h->tau % R);
-      a.tau = h->tau;
-      a.Kb = (int)kb;
-      CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
-      CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
-      CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+      if (h->tfm) {
+        ta.tau = h->tau;
+        ta.Kb = (int)kb;
+        CUDA_TRY(h, mca::launch_tfm_eval(ta, h->stream));
+        CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
+        CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
+      } else {
+        a.tau = h->tau;
+        a.Kb = (int)kb;
+        CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
+        CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
+        CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+      }
       h->launches += 3;
       mca::DeepCtl ctl;
       CUDA_TRY(h, cudaMemcpyAsync(&ctl, h->ctl, sizeof(ctl), cudaMemcpyDeviceToHost, h->stream));
@@ -867,7 +1015,16 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
                               h->stream));
   CUDA_TRY(h, cudaMemcpyAsync(h->ex_new, new_w, sizeof(float) * n, cudaMemcpyHostToDevice,
                               h->stream));
-  if (h->deep) {
+  if (h->tfm) {
+    mca::TfmArgs a = tfm_args(h);
+    a.n_explicit = (int)n;
+    a.ex_idx = h->ex_idx;
+    a.ex_new = h->ex_new;
+    a.ex_out = h->ex_out;
+    CUDA_TRY(h, mca::launch_tfm_eval(a, h->stream));
+    CUDA_TRY(h, mca::launch_tfm_decide(a, h->stream));
+    h->launches += 2;
+  } else if (h->deep) {
     mca::DeepArgs a = deep_args(h);
     a.n_explicit = (int)n;
     a.ex_idx = h->ex_idx;
@@ -896,6 +1053,119 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
     h->broken = true;
     return fail(h, MCA_ERR_TIMEOUT, "device-side wait timed out");
   }
+  return MCA_OK;
+}
+
+mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const mca_options* opt,
+                                  size_t* bytes) {
+  mca_status rc = tfm_check(spec, n_seq);
+  if (rc != MCA_OK) return rc;
+  if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
+  const mca_options o = opt ? *opt : default_options();
+  *bytes = tfm_plan(*spec, n_seq, o.trace_cap).total;
+  return MCA_OK;
+}
+
+mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
+                                  const int32_t* tokens, int64_t n_seq, const float* init_params,
+                                  const mca_options* opt, mca_handle** out) {
+  if (!out) return fail(nullptr, MCA_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  mca_status rc = tfm_check(spec, n_seq);
+  if (rc != MCA_OK) return rc;
+  if (!tokens || !init_params) return fail(nullptr, MCA_ERR_INVALID, "NULL tokens or params");
+  const mca_options o = opt ? *opt : default_options();
+  if (o.K < 1 || o.K > mca::kKmax)
+    return fail(nullptr, MCA_ERR_INVALID, "K = %d outside 1..%d", o.K, mca::kKmax);
+  if (o.resync_period < 0 || o.trace_cap < 0) return fail(nullptr, MCA_ERR_INVALID, "negative option");
+  const mca_domain d = dom ? *dom : default_domain();
+  if (d.op != MCA_OP_REPLACE && d.op != MCA_OP_PERTURB)
+    return fail(nullptr, MCA_ERR_INVALID, "unknown op %d", d.op);
+  if (!std::isfinite(d.lo) || !std::isfinite(d.hi) || !std::isfinite(d.delta) || !(d.hi > d.lo))
+    return fail(nullptr, MCA_ERR_INVALID, "bad domain");
+  mca_handle* h = new (std::nothrow) mca_handle();
+  if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
+  auto bail = [&](mca_status st) {
+    g_create_err = h->err;
+    mca_destroy(h);
+    return st;
+  };
+  h->tfm = true;
+  h->tspec = *spec;
+  h->dom = d;
+  h->opt = o;
+  h->stream = (cudaStream_t)o.stream;
+  h->N = n_seq * spec->ctx;
+  h->C = spec->vocab;
+  h->trace_cap = o.trace_cap;
+  const TfmLayout TL = tfm_offsets(*spec);
+  h->P = TL.P;
+  mca_layer pseudo;
+  std::memset(&pseudo, 0, sizeof(pseudo));
+  pseudo.n_in = (int32_t)TL.P;
+  pseudo.n_out = 1;
+  pseudo.wkind = MCA_W_FP32;
+  h->layers.push_back(pseudo);
+  h->off.push_back(0);
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e == cudaSuccess)
+    e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+  if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
+  const TfmMem M = tfm_plan(*spec, n_seq, o.trace_cap);
+  if (o.workspace) {
+    if (o.workspace_bytes < M.total)
+      return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
+                       M.total));
+    if (reinterpret_cast<uintptr_t>(o.workspace) % 256 != 0)
+      return bail(fail(h, MCA_ERR_INVALID, "workspace not 256-byte aligned"));
+    h->ws = o.workspace;
+    h->ws_bytes = o.workspace_bytes;
+  } else {
+    e = cudaMalloc(&h->ws, M.total);
+    if (e != cudaSuccess) return bail(fail(h, MCA_ERR_OOM, "%s", cudaGetErrorString(e)));
+    h->ws_owned = true;
+    h->ws_bytes = M.total;
+  }
+  char* base = static_cast<char*>(h->ws);
+  h->params = reinterpret_cast<float*>(base + M.params);
+  h->w_eff.push_back(h->params);
+  h->code.push_back(nullptr);
+  h->wfix.push_back(nullptr);
+  h->tokens = reinterpret_cast<int*>(base + M.tokens);
+  h->X = reinterpret_cast<float*>(base + M.X);
+  h->ell = reinterpret_cast<float*>(base + M.ell);
+  h->partial = reinterpret_cast<float*>(base + M.partial);
+  h->st = reinterpret_cast<DevState*>(base + M.st);
+  h->ctl = reinterpret_cast<mca::DeepCtl*>(base + M.ctl);
+  h->trace = o.trace_cap > 0 ? reinterpret_cast<mca_trace_rec*>(base + M.trace) : nullptr;
+  h->ex_idx = reinterpret_cast<unsigned int*>(base + M.ex_idx);
+  h->ex_new = reinterpret_cast<float*>(base + M.ex_new);
+  h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
+  e = cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream);
+  if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
+  {
+    const size_t nt = (size_t)n_seq * (spec->ctx + 1);
+    std::vector<int> th(nt);
+    e = cudaMemcpyAsync(th.data(), tokens, sizeof(int) * nt, cudaMemcpyDefault, h->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+    if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
+    for (size_t q = 0; q < nt; ++q)
+      if (th[q] < 0 || th[q] >= spec->vocab)
+        return bail(fail(h, MCA_ERR_INVALID, "token %d outside [0, %d)", th[q], spec->vocab));
+    e = cudaMemcpyAsync(h->tokens, th.data(), sizeof(int) * nt, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+    if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
+  }
+  rc = load_params(h, init_params, nullptr);
+  if (rc != MCA_OK) return bail(rc);
+  rc = resync(h);
+  if (rc != MCA_OK) return bail(rc);
+  DevState ds;
+  rc = read_state(h, &ds);
+  if (rc != MCA_OK) return bail(rc);
+  if (!std::isfinite(ds.S)) return bail(fail(h, MCA_ERR_NUMERIC, "initial loss is not finite"));
+  *out = h;
   return MCA_OK;
 }
 

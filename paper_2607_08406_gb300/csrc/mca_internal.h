@@ -147,6 +147,63 @@ cudaError_t launch_deep_commit(const DeepArgs& a, cudaStream_t s);  // grid ntil
 cudaError_t launch_deep_forward_layer(const DeepArgs& a, int l, cudaStream_t s);
 cudaError_t launch_deep_losses(const DeepArgs& a, cudaStream_t s);
 
+// ------------------------------------------------------------------------------------------------
+// Character-level Transformer path: pre-LN GPT blocks over B sequences of T tokens. All parameters
+// live in one flat fp32 array; a candidate recomputes each sequence from the first stage its
+// parameter feeds (embeddings, block b, or the final LN and head), reading the parameters through
+// a one-element patch (index midx reads mval), on the cached residual stream at that stage.
+// ------------------------------------------------------------------------------------------------
+constexpr int kTfmMaxBlocks = 8;
+constexpr int kTfmThreads = 512;
+constexpr int kTfmMaxT = 64;
+constexpr int kTfmMaxD = 128;
+constexpr int kTfmMaxV = 128;
+constexpr int kTfmFC = 128;        // FFN hidden columns per chunk
+
+enum TfmMode { kTfmEval = 0, kTfmCommit = 1, kTfmForward = 2 };
+
+struct TfmArgs {
+  int V, T, d, H, dh, F, nL, B;
+  float eps;
+  int act;
+  float g;
+  // flat offsets: embeddings, the first block, the block stride, the final LN and the head; and the
+  // offsets inside a block
+  unsigned long long o_tok, o_pos, o_blk0, blk_size, o_lnf_g, o_lnf_b, o_wh, o_bh, P;
+  unsigned int r_ln1g, r_ln1b, r_wq, r_bq, r_wk, r_bk, r_wv, r_bv, r_wo, r_bo, r_ln2g, r_ln2b,
+      r_w1, r_b1, r_w2, r_b2;
+  float* params;             // [P]
+  const int* tokens;         // [B x (T + 1)]
+  float* X;                  // [(nL + 1) x B x T x d] residual stream entering block b (b = nL: final)
+  float* ell;                // [B] per-sequence loss sums
+  int loss_unused;
+  int op;
+  float lo, hi, delta, bound;
+  int strict;
+  unsigned long long seed, tau;
+  int Kb;
+  int mode;
+  size_t smem;               // dynamic shared memory of the sequence kernel
+  float* partial;            // [kKmax x B]
+  DevState* st;
+  DeepCtl* ctl;
+  mca_trace_rec* trace;
+  int trace_cap;
+  const unsigned long long* ftau;
+  const unsigned char* facc;
+  int nforce;
+  int n_explicit;
+  const unsigned int* ex_idx;
+  const float* ex_new;
+  double* ex_out;
+};
+
+size_t tfm_smem_bytes(int T, int d, int dh, int V);
+cudaError_t launch_tfm_eval(const TfmArgs& a, cudaStream_t s);      // grid (Kb, B)
+cudaError_t launch_tfm_decide(const TfmArgs& a, cudaStream_t s);    // one CTA
+cudaError_t launch_tfm_commit(const TfmArgs& a, cudaStream_t s);    // grid B
+cudaError_t launch_tfm_forward(const TfmArgs& a, cudaStream_t s);   // grid B, writes every stage
+
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
 cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
 cudaError_t launch_csr_count(const float* XT, int Np, int N, int D, int* cnt, cudaStream_t s);
@@ -233,4 +290,10 @@ struct mca_handle {
   unsigned long long launches = 0, resyncs = 0;
   bool broken = false;                   // a sticky CUDA error or device timeout was seen
   float rate_acc = 0.0f, rate_trials = 0.0f;   // deep path: acceptance counts (batch width)
+  // transformer path
+  bool tfm = false;
+  mca_tfm_spec tspec{};
+  float* params = nullptr;               // [P] flat parameters
+  int* tokens = nullptr;                 // [B x (ctx + 1)]
+  float* X = nullptr;                    // cached residual stream at every stage
 };

@@ -45,6 +45,12 @@ class mca_options(Structure):
                 ("workspace_bytes", c_size_t), ("fixed_K", c_int32)]
 
 
+class mca_tfm_spec(Structure):
+    _fields_ = [("vocab", c_int32), ("ctx", c_int32), ("d_model", c_int32), ("n_layer", c_int32),
+                ("n_head", c_int32), ("d_ff", c_int32), ("act", c_int32), ("act_param", c_float),
+                ("ln_eps", c_float)]
+
+
 class mca_run_stats(Structure):
     _fields_ = [("trials", c_uint64), ("accepts", c_uint64), ("candidates", c_uint64),
                 ("batches", c_uint64), ("wasted", c_uint64), ("forced", c_uint64),
@@ -75,6 +81,11 @@ SIGNATURES = {
     "mca_create": (c_int32, [POINTER(mca_layer), c_int32, c_int32, POINTER(mca_domain),
                              POINTER(mca_dataset), c_void_p, POINTER(mca_options),
                              POINTER(c_void_p)]),
+    "mca_tfm_workspace_size": (c_int32, [POINTER(mca_tfm_spec), c_int64, POINTER(mca_options),
+                                         POINTER(c_size_t)]),
+    "mca_create_transformer": (c_int32, [POINTER(mca_tfm_spec), POINTER(mca_domain), c_void_p,
+                                         c_int64, c_void_p, POINTER(mca_options),
+                                         POINTER(c_void_p)]),
     "mca_run": (c_int32, [c_void_p, c_uint64, c_uint64, POINTER(mca_run_stats)]),
     "mca_loss": (c_int32, [c_void_p, POINTER(c_double)]),
     "mca_get_params": (c_int32, [c_void_p, c_void_p, c_size_t]),
@@ -200,6 +211,51 @@ def mca_create(layers, loss: str, domain, X, y, init, K: int = 32, resync_period
     _check(lib.mca_create(L, len(layers), LOSS[loss], ctypes.byref(dom), ctypes.byref(ds),
                           _ptr(init), ctypes.byref(opt), ctypes.byref(h)))
     return Handle(h, keep)
+
+
+def _tfm_spec(sp) -> mca_tfm_spec:
+    return mca_tfm_spec(sp.vocab, sp.ctx, sp.d_model, sp.n_layer, sp.n_head, sp.d_ff, ACT[sp.act],
+                        float(sp.act_param), float(sp.ln_eps))
+
+
+def mca_tfm_workspace_size(spec, n_seq: int, K: int = 32, trace_cap: int = 0) -> int:
+    opt = mca_options(K, 0, None, trace_cap, 0, None, 0, 0)
+    out = c_size_t(0)
+    sp = _tfm_spec(spec)
+    _check(load_library().mca_tfm_workspace_size(ctypes.byref(sp), n_seq, ctypes.byref(opt),
+                                                 ctypes.byref(out)))
+    return out.value
+
+
+def mca_create_transformer(spec, domain, tokens, init, K: int = 32, resync_period: int = 0,
+                           trace_cap: int = 0, stream=None, fixed_K: bool = False):
+    """tokens: [B, ctx + 1] int32, init: [P] float32 (torch tensors or numpy arrays, host or
+    device). The workspace is a torch CUDA tensor the handle keeps alive."""
+    import torch
+    lib = load_library()
+    if stream is None:
+        stream = torch.cuda.current_stream().cuda_stream
+    n_seq = int(tokens.shape[0])
+    nbytes = mca_tfm_workspace_size(spec, n_seq, K, trace_cap)
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
+    ws_ptr = (ws.data_ptr() + 255) // 256 * 256
+    opt = mca_options(K, resync_period, stream, trace_cap, 0, ws_ptr, nbytes, int(fixed_K))
+    sp = _tfm_spec(spec)
+    dom = _domain(domain)
+    h = c_void_p(None)
+    _check(lib.mca_create_transformer(ctypes.byref(sp), ctypes.byref(dom), _ptr(tokens), n_seq,
+                                      _ptr(init), ctypes.byref(opt), ctypes.byref(h)))
+    return Handle(h, [tokens, init, ws])
+
+
+def create_from_tfm_workload(wl, device: bool = True, **kw) -> Handle:
+    import torch
+    tokens, init = wl.tokens, wl.init
+    if device:
+        tokens = torch.from_numpy(tokens).cuda()
+        init = torch.from_numpy(init).cuda()
+    kw.setdefault("K", wl.K)
+    return mca_create_transformer(wl.spec, wl.domain, tokens, init, **kw)
 
 
 def mca_run(h: Handle, n_trials: int, seed: int) -> dict:
