@@ -122,19 +122,59 @@ def load_peaks():
 def make_workload(args, rank):
     from paper_2607_08406_gb300 import workloads as W
     kw = {}
-    if args.N:
-        kw["N"] = args.N
-    if args.H:
-        kw["H"] = args.H
-    wl = W.make(args.workload, **kw)
+    if args.workload == "char_transformer":
+        if args.N:
+            kw["batch"] = args.N
+        wl = W.char_transformer(**kw)
+    else:
+        if args.N:
+            kw["N"] = args.N
+        if args.H:
+            kw["H"] = args.H
+        wl = W.make(args.workload, **kw)
     wl.seed = args.seed + rank
     if args.K:
         wl.K = args.K
     return wl
 
 
+def is_tfm(wl) -> bool:
+    return hasattr(wl, "spec")
+
+
+def host_arrays(wl):
+    """The arrays a job uploads: (X, y, init) for an MLP, (tokens, init) for the Transformer."""
+    return (wl.tokens, wl.init) if is_tfm(wl) else (wl.X, wl.y, wl.init)
+
+
+def create_handle(mca, wl, arrays, **kw):
+    if is_tfm(wl):
+        tokens, init = arrays
+        return mca.mca_create_transformer(wl.spec, wl.domain, tokens, init, K=wl.K, **kw)
+    X, y, init = arrays
+    return mca.mca_create(wl.layers, wl.loss, wl.domain, X, y, init, K=wl.K, **kw)
+
+
 def cpu_oracle_rate(wl, n_trials, warm=0):
-    """Trials/s of the oracle's incremental mode after its untimed cache build (forward pass)."""
+    """A function running oracle trials t0 .. t0+n: the incremental mode (after an untimed cache
+    build) for the MLPs, the full-recompute loop for the Transformer."""
+    if is_tfm(wl):
+        from oracle import mca_tfm as T
+        flat = np.array(wl.init, dtype=np.float32)
+        state = {"S": float(T.tfm_seq_losses(wl.spec, flat.astype(np.float64), wl.tokens).sum())}
+
+        def tfm_trials(t0, n):
+            for t in range(t0, t0 + n):
+                idx, old, new, valid = T.tfm_propose(wl.seed, t, flat, wl.domain)
+                if not valid:
+                    continue
+                flat[idx] = np.float32(new)
+                S_new = float(T.tfm_seq_losses(wl.spec, flat.astype(np.float64), wl.tokens).sum())
+                if S_new <= state["S"]:
+                    state["S"] = S_new
+                else:
+                    flat[idx] = np.float32(old)
+        return tfm_trials
     from oracle import mca_oracle as O
     XT = np.ascontiguousarray(wl.X.astype(np.float64).T)
     params = O.Params(wl.layers, wl.init)
@@ -178,7 +218,8 @@ def run_reference(args):
     dt = time.perf_counter() - t0
     rate = per_step * args.steps / dt
     cores = len(os.sched_getaffinity(0))
-    sample = (f"oracle incremental mode (fp64 numpy), trials {per_step * args.warmup}.."
+    mode = "full-recompute" if is_tfm(wl) else "incremental"
+    sample = (f"oracle {mode} mode (fp64 numpy), trials {per_step * args.warmup}.."
               f"{tau} of {wl.name}, after an untimed forward pass")
     line = {"impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
@@ -213,12 +254,10 @@ def run_ours(args):
     T = args.trials_per_step or math.ceil(JOB_TRIALS / (K + W_))
     stream = torch.cuda.current_stream()
 
-    Xd = torch.from_numpy(wl.X).cuda()
-    yd = torch.from_numpy(wl.y).cuda()
-    initd = torch.from_numpy(wl.init).cuda()
-    h = mca.mca_create(wl.layers, wl.loss, wl.domain, Xd, yd, initd, K=wl.K,
-                       resync_period=args.resync, stream=stream.cuda_stream, grid=args.grid,
-                       fixed_K=args.fixed_K)
+    dev_arrays = [torch.from_numpy(a).cuda() for a in host_arrays(wl)]
+    extra = {} if is_tfm(wl) else {"grid": args.grid}
+    h = create_handle(mca, wl, dev_arrays, resync_period=args.resync, stream=stream.cuda_stream,
+                      fixed_K=args.fixed_K, **extra)
     # one full forward pass (the resync step), timed on its own
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -254,7 +293,7 @@ def run_ours(args):
     # falls in the step), HBM-bound; deep nets -- the candidate chains (SIMT fp32 FMA), whose
     # FLOPs are divided by the whole step time (a lower bound: the step also holds the decide and
     # commit kernels and one host round trip per batch)
-    deep = len(wl.layers) > 2
+    deep = is_tfm(wl) or len(wl.layers) > 2
     peak, peak_kind = load_peaks()
     traffic = None
     if deep:
@@ -266,7 +305,8 @@ def run_ours(args):
         flops_timed = st1["alg_flops"] - st0["alg_flops"]
         achieved = flops_timed / (total_ms / 1e3) / 1e12
         roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak, "traffic": None, "kernel": "deep_chain_kernel",
+                    "frac": achieved / peak, "traffic": None,
+                    "kernel": "tfm_seq_kernel" if is_tfm(wl) else "deep_chain_kernel",
                     "peak_kind": peak_kind,
                     "flops": "FLOPs of the evaluated candidates' recomputation, counted by the "
                              "library, over the whole step time"}
@@ -287,16 +327,13 @@ def run_ours(args):
     # (create from host arrays -> JOB_TRIALS trials -> parameters back to host)
     e2e = None
     if not args.no_e2e:
-        Xh = torch.from_numpy(wl.X).pin_memory()
-        yh = torch.from_numpy(wl.y).pin_memory()
-        ih = torch.from_numpy(wl.init).pin_memory()
+        pinned = [torch.from_numpy(a).pin_memory() for a in host_arrays(wl)]
         out = torch.empty(wl.n_params, dtype=torch.float32).pin_memory()
         e2e_trials = args.e2e_trials or JOB_TRIALS
 
         def job():
-            hh = mca.mca_create(wl.layers, wl.loss, wl.domain, Xh, yh, ih, K=wl.K,
-                                resync_period=args.resync, stream=stream.cuda_stream,
-                                grid=args.grid, fixed_K=args.fixed_K)
+            hh = create_handle(mca, wl, pinned, resync_period=args.resync,
+                               stream=stream.cuda_stream, fixed_K=args.fixed_K, **extra)
             mca.mca_run(hh, e2e_trials, wl.seed)
             mca.mca_get_params(hh, wl.n_params, out)
             lv = mca.mca_loss(hh)
@@ -315,7 +352,7 @@ def run_ours(args):
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             dt = float(t.item())
         e2e = {"value": e2e_trials * args.e2e_steps * world / dt, "unit": UNIT,
-               "h2d_bytes_per_step": int(wl.X.nbytes + wl.y.nbytes + wl.init.nbytes),
+               "h2d_bytes_per_step": int(sum(a.nbytes for a in host_arrays(wl))),
                "d2h_bytes_per_step": int(out.numel() * 4 + 8),
                "step": f"create from pinned host arrays + {e2e_trials} trials + params to host"}
 
@@ -325,9 +362,10 @@ def run_ours(args):
         t0 = time.perf_counter()
         trials(0, args.cpu_trials)
         dt = time.perf_counter() - t0
+        mode = "full-recompute" if is_tfm(wl) else "incremental"
         cpu = {"value": args.cpu_trials / dt, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
                "kind": "oracle",
-               "sample": f"first {args.cpu_trials} trials of {wl.name}, oracle incremental mode "
+               "sample": f"first {args.cpu_trials} trials of {wl.name}, oracle {mode} mode "
                          f"(fp64 numpy), after an untimed forward pass"}
 
     if rank == 0:
@@ -335,13 +373,16 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": W_, "ms_per_step": total_ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": wl.name, "N": wl.N, "hidden": wl.layers[0].n_out,
-                       "layers": len(wl.layers),
+            "config": {"workload": wl.name,
+                       "N": int(wl.tokens.shape[0] * wl.spec.ctx) if is_tfm(wl) else wl.N,
+                       "hidden": wl.spec.d_model if is_tfm(wl) else wl.layers[0].n_out,
+                       "layers": wl.spec.n_layer if is_tfm(wl) else len(wl.layers),
                        "K": wl.K, "trials_per_step": T,
                        "trial_range": [W_ * T, (W_ + K) * T], "seed": args.seed,
                        "resync_period": args.resync, "resync_ms": resync_ms,
-                       "l2": "no flush: the cached fields exceed L2" if not deep else
-                             "no flush: the cached fields of all layers (256 MB) exceed L2",
+                       "l2": ("no flush: the cached hidden fields (3.9 GB) exceed L2"
+                              if not deep else "no flush: a step's candidates recompute from "
+                              "cached fields / residual streams that exceed L2 or are rewritten"),
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
