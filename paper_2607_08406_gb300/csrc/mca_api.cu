@@ -219,7 +219,7 @@ mca_status count_nnz(const mca_dataset* d, cudaStream_t s, long long* nnz) {
 // Sample ranges of the trial loop: one CTA per range, all CTAs co-resident. Ranges hold a multiple
 // of 8 samples (whole 32-byte sectors of a hidden-field row) and at least about kRangeTarget.
 struct Ranges {
-  int NR, RS, SUB, smem_records;
+  int NR, RS, SUB, smem_records, window;
 };
 
 mca_status choose_ranges(const std::vector<mca_layer>& layers, int loss, long long N, int grid_opt,
@@ -243,12 +243,18 @@ mca_status choose_ranges(const std::vector<mca_layer>& layers, int loss, long lo
     const int NR = (int)((N + RS - 1) / RS);
     int SUB = (RS + mca::kMaxSubs - 1) / mca::kMaxSubs;
     SUB = std::max(128, (SUB + 31) / 32 * 32);
-    Ranges R{NR, RS, SUB, 0};
+    Ranges R{NR, RS, SUB, 0, 0};
     if (smem_records && (size_t)RS * mca::kSR * sizeof(float) <= (size_t)mca::kSmemRecordBytes) {
       probe.smem_records = 1;
       probe.RS = RS;
       if (mca::mlp2_loop_max_grid(probe, sms) < NR) continue;
       R.smem_records = 1;
+      // the windowed loop when its records and candidate window fit next to the static state
+      if (mca::mlp2_window_smem_bytes(RS) + 24 * 1024 <= 227 * 1024) {
+        probe.window = 1;
+        if (mca::mlp2_loop_max_grid(probe, sms) >= NR) R.window = 1;
+        probe.window = 0;
+      }
     } else if (smem_records) {
       continue;
     }
@@ -272,6 +278,7 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.RS = h->RS;
   a.SUB = h->SUB;
   a.smem_records = h->smem_records;
+  a.window = h->window;
   a.P = h->P;
   a.P1 = (unsigned long long)L1.n_in * L1.n_out;
   a.xs_off = h->xs_off;
@@ -695,6 +702,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     h->RS = R.RS;
     h->SUB = R.SUB;
     h->smem_records = R.smem_records;
+    h->window = R.window;
   }
   const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap, h->NR);
   if (o.workspace) {

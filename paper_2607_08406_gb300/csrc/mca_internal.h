@@ -26,6 +26,12 @@ constexpr float kRateDecay = 0.95f;
 constexpr float kWidthMlp2 = 3.0f;
 constexpr float kWidthDeep = 1.5f;  // samples per range below which fewer CTAs are used
 constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
+// Window of the trial loop: kWS candidate slots per CTA, each caching up to kCap entries of the
+// candidate's segment (range-local sample, activation change, new hidden field); kPF of them are
+// prepared while the CTA waits at the grid barrier. Batches are at most kWS - kPF wide.
+constexpr int kWS = 96;
+constexpr int kCap = 160;
+constexpr int kPF = 32;
 
 // Device-resident run state (one per handle).
 struct DevState {
@@ -45,6 +51,7 @@ struct Mlp2Args {
   int N, D, H, C, Np;
   int NR, RS, SUB;           // ranges, samples per range, entries per sub-chunk (multiple of 32)
   int smem_records;          // 1: each CTA keeps its range's sample records in shared memory
+  int window;                // 1: run the windowed trial loop (records and window in shared memory)
   unsigned long long P, P1;
   const int* xs_off;         // [D + 1] CSR of X by feature: entries of feature i in [off[i], off[i+1])
   const int* xs_n;           // [nnz] sample index of each entry (ascending inside a feature)
@@ -223,6 +230,7 @@ cudaError_t launch_mlp2_outputs(const Mlp2Args& a, const int* y, cudaStream_t s)
 cudaError_t launch_sum_loss(const float* ell, int N, DevState* st, cudaStream_t s);
 // Cooperative persistent trial loop, one CTA per sample range (grid = NR).
 cudaError_t launch_mlp2_loop(const Mlp2Args& a, cudaStream_t s);
+size_t mlp2_window_smem_bytes(int RS);
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);
 size_t mlp2_loop_smem_bytes(const Mlp2Args& a);
 
@@ -273,7 +281,7 @@ struct mca_handle {
   mca::DeepCtl* ctl = nullptr;
   int ntiles = 0;
   float* partial = nullptr;
-  int NR = 0, RS = 0, SUB = 0, smem_records = 0;
+  int NR = 0, RS = 0, SUB = 0, smem_records = 0, window = 0;
   mca::GridBarrier* bar = nullptr;
   mca::DevState* st = nullptr;
   mca_trace_rec* trace = nullptr;

@@ -612,23 +612,553 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
   }
 }
 
+// ------------------------------------------------------------------------------------------------
+// Windowed trial loop. Same work split, order of sums and decisions as mlp2_trial_loop, but each CTA
+// keeps a ring of kWS candidate slots: slot (t mod kWS) holds trial t's candidate for this CTA's range
+// and, for first-layer candidates with at most kCap entries in the range, the gathered entries
+// (range-local sample, activation change f(z + delta x) - f(z), new field z + delta x). A batch then
+// evaluates and commits from shared memory only. While thread 0 waits at the grid barrier, the other
+// warps prepare the next kPF slots (Philox, weight, CSR and z1 gathers). After a commit every prepared
+// slot that depends on what changed is dropped or patched: the same weight (old value), a first-layer
+// candidate of the same hidden row (z1 changed), or the W2 column of a first-layer candidate.
+// ------------------------------------------------------------------------------------------------
+struct WSlot {
+  Cand c;
+  unsigned long long tau;
+  int state;                 // 0 empty, 1 entries cached (or nothing to evaluate), 2 read from global
+  int pad;
+};
+
+size_t mlp2_window_smem_bytes(int RS) {
+  return sizeof(float) * (size_t)kRecFields * RS +
+         (size_t)kWS * kCap * (sizeof(unsigned short) + 2 * sizeof(float));
+}
+
+// One cached entry: l' - l from the activation change da (COMMIT: also the new record).
+template <int ACT2, int LOSS, int NC, bool COMMIT>
+__device__ __forceinline__ float entry_cached(const Mlp2Args& a, Recs R,
+                                              const float (&w)[NC > 0 ? NC : kMaxC], int nl,
+                                              float da) {
+  if (da == 0.0f) return 0.0f;
+  constexpr int M = NC > 0 ? NC : kMaxC;
+  const int C = NC > 0 ? NC : a.C;
+  float zz[M];
+  float ell;
+  int y;
+  load_srec(R.rec, R.pitch, nl, zz, ell, y);
+#pragma unroll
+  for (int k = 0; k < M; ++k)
+    if (k < C) zz[k] = fmaf(w[k], da, zz[k]);
+  const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
+  if (COMMIT) store_srec(R.rec, R.pitch, nl, zz, ln, y);
+  return ln - ell;
+}
+
+// Warp prepares slot sl for trial t: proposal, W2 column, and (cacheable first-layer candidates)
+// the gathered entries.
+template <int ACT1>
+__device__ __forceinline__ void prepare_slot(const Mlp2Args& a, WSlot* slots, float (*w2c)[kMaxC],
+                                             unsigned short* e_nl, float* e_da, float* e_zn,
+                                             int sl, unsigned long long t, int r, int s0, int s1) {
+  const int lane = threadIdx.x & 31;
+  if (lane == 0) {
+    const uint4 w = trial_words(a.seed, t);
+    const unsigned int idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
+    Cand c;
+    fill_candidate(a, idx, w.y, false, 0.0f, r, s0, s1, c);
+    slots[sl].c = c;
+    slots[sl].tau = t;
+    slots[sl].state = 0;
+  }
+  __syncwarp();
+  const Cand c = slots[sl].c;
+  if (c.layer == 0 && c.gcnt > 0) {
+    for (int q = lane; q < kMaxC; q += 32)
+      w2c[sl][q] = q < a.C ? a.w2[(size_t)q * a.H + c.row] : 0.0f;
+  }
+  int state = 2;
+  if (c.gcnt == 0) {
+    state = 1;
+  } else if (c.layer == 0 && c.ecnt <= kCap) {
+    const float* zrow = a.z1 + (size_t)c.row * a.Np;
+    unsigned short* nl = e_nl + (size_t)sl * kCap;
+    float* da = e_da + (size_t)sl * kCap;
+    float* zn = e_zn + (size_t)sl * kCap;
+    for (int e0 = 0; e0 < c.ecnt; e0 += 128) {
+      int nn[4];
+      float xv[4], zv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int e = e0 + u * 32 + lane;
+        nn[u] = -1;
+        xv[u] = 0.0f;
+        if (e < c.ecnt) {
+          nn[u] = __ldg(a.xs_n + c.ebeg + e);
+          xv[u] = __ldg(a.xs_v + c.ebeg + e);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) zv[u] = nn[u] >= 0 ? zrow[nn[u]] : 0.0f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int e = e0 + u * 32 + lane;
+        if (nn[u] < 0) continue;
+        const float z2 = fmaf(c.delta, xv[u], zv[u]);
+        nl[e] = (unsigned short)(nn[u] - s0);
+        zn[e] = z2;
+        da[e] = act<ACT1>(z2, a.g1, a.act1) - act<ACT1>(zv[u], a.g1, a.act1);
+      }
+    }
+    state = 1;
+  }
+  __syncwarp();
+  if (lane == 0) slots[sl].state = state;
+}
+
+__device__ __forceinline__ bool slot_ready(const WSlot* slots, unsigned long long t) {
+  const WSlot& s = slots[t % kWS];
+  return s.tau == t && s.state != 0;
+}
+
+template <int ACT1, int ACT2, int LOSS, int NC>
+__global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) {
+  extern __shared__ __align__(16) float s_dyn[];
+  __shared__ WSlot s_slot[kWS];
+  __shared__ float s_w2c[kWS][kMaxC];
+  __shared__ float s_sub[kKmax * kMaxSubs];
+  __shared__ int s_bslot[kKmax];       // batch position -> slot
+  __shared__ int s_sub0[kKmax], s_nsub[kKmax];
+  __shared__ float s_dS[kKmax];
+  __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
+  __shared__ int s_flag, s_kstar, s_total, s_bvalid;
+  __shared__ unsigned long long s_bbytes, s_tau_hi;
+  float* s_records = s_dyn;
+  unsigned short* e_nl = reinterpret_cast<unsigned short*>(s_dyn + kRecFields * a.RS);
+  float* e_da = reinterpret_cast<float*>(e_nl + kWS * kCap);
+  float* e_zn = e_da + kWS * kCap;
+  constexpr int M = NC > 0 ? NC : kMaxC;
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int r = blockIdx.x;
+  const int s0 = min(r * a.RS, a.N), s1 = min(s0 + a.RS, a.N);
+  const Recs R{s_records, a.RS};
+  {
+    const int ns = s1 - s0;
+    for (int t = tid; t < kRecFields * ns; t += kLoopThreads) {
+      const int f = t / ns, nl = t - f * ns;
+      s_records[f * a.RS + nl] = a.srec[(size_t)f * a.Np + s0 + nl];
+    }
+  }
+  for (int q = tid; q < kWS; q += kLoopThreads) {
+    s_slot[q].state = 0;
+    s_slot[q].tau = ~0ull;
+  }
+  DevState* st = a.st;
+  const bool stats_thread = r == 0 && tid == 0;
+  double S = 0.0;
+  unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
+                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0;
+  if (stats_thread) {
+    S = st->S;
+    n_trace = st->trace_written;
+  }
+  unsigned int gen = 0;
+  unsigned long long tau = a.tau0;
+  const unsigned long long end = a.tau0 + a.n_trials;
+  if (tid == 0) s_tau_hi = a.tau0;
+  float rate_a = st->rate_acc, rate_t = st->rate_trials;
+  int buf = 0;
+  const int kmaxw = min(a.K, kWS - kPF);
+  __syncthreads();
+
+  while (tau < end) {
+    const unsigned long long t_a = stats_thread ? globaltimer_ns() : 0ull;
+    const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
+    const int Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
+    // ---- slots of this batch (prepared ahead in the common case)
+    for (int k = warp; k < Kb; k += kLoopWarps) {
+      const unsigned long long t = tau + (unsigned long long)k;
+      if (!slot_ready(s_slot, t))
+        prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, r, s0, s1);
+    }
+    __syncthreads();
+    if (warp == 0) {                 // sub-chunk scan and batch statistics
+      int v[4], loc = 0;
+      unsigned long long bytes = 0ull;
+      int valid = 0;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = lane * 4 + u;
+        v[u] = 0;
+        if (k < Kb) {
+          const int sl = (int)((tau + (unsigned long long)k) % kWS);
+          s_bslot[k] = sl;
+          const Cand& c = s_slot[sl].c;
+          v[u] = c.nsub;
+          if (tau + (unsigned long long)k >= s_tau_hi) bytes += c.bytes;
+          valid += c.valid;
+        }
+        loc += v[u];
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
+        valid += __shfl_xor_sync(0xffffffffu, valid, o);
+      }
+      int inc = loc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      int ex = inc - loc;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = lane * 4 + u;
+        if (k < Kb) {
+          s_sub0[k] = ex;
+          s_nsub[k] = v[u];
+        }
+        ex += v[u];
+      }
+      if (lane == 31) s_total = inc;
+      if (lane == 0) {
+        s_bbytes = bytes;
+        s_bvalid = valid;
+      }
+    }
+    __syncthreads();
+    // ---- evaluate: warp per sub-chunk; cached slots from shared memory, the rest from global
+    {
+      const int total = s_total;
+      int k = 0;
+      for (int it = warp; it < total; it += kLoopWarps) {
+        while (s_sub0[k] + s_nsub[k] <= it) ++k;
+        const int sl = s_bslot[k];
+        const Cand& c = s_slot[sl].c;
+        const int q = it - s_sub0[k];
+        float v;
+        if (s_slot[sl].state == 1) {
+          float w[M];
+          load_w2c<NC>(s_w2c[sl], a.C, w);
+          const unsigned short* nl = e_nl + (size_t)sl * kCap;
+          const float* da = e_da + (size_t)sl * kCap;
+          const int e_lo = q * a.SUB, e_hi = min(e_lo + a.SUB, c.ecnt);
+          float acc = 0.0f;
+          for (int g = e_lo; g < e_hi; g += 128) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int e = g + u * 32 + lane;
+              if (e < e_hi) acc += entry_cached<ACT2, LOSS, NC, false>(a, R, w, nl[e], da[e]);
+            }
+          }
+          v = warp_sum(acc);
+        } else {
+          v = eval_sub<ACT1, ACT2, LOSS, NC>(a, R, s0, c, s_w2c[sl], q);
+        }
+        if (lane == 0) s_sub[it] = v;
+      }
+    }
+    __syncthreads();
+    float* part = a.partial + (size_t)buf * kKmax * a.NR;
+    for (int k = tid; k < Kb; k += kLoopThreads) {
+      float sum = 0.0f;
+      for (int q = 0; q < s_nsub[k]; ++q) sum += s_sub[s_sub0[k] + q];
+      part[(size_t)k * a.NR + r] = sum;
+    }
+    const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
+    // ---- grid barrier, split: arrive, prepare the next slots, wait
+    __syncthreads();
+    unsigned int g_arr = gen;
+    if (tid == 0) {
+      __threadfence();
+      const unsigned int prev = atomicAdd(&a.bar->count, 1u);
+      if (prev == gridDim.x - 1) {
+        a.bar->count = 0u;
+        __threadfence();
+        st_release_gpu(&a.bar->gen, gen + 1u);
+      }
+    }
+    if (warp > 0) {
+      const unsigned long long t_lo = tau + (unsigned long long)Kb;
+      for (int k = warp - 1; k < kPF; k += kLoopWarps - 1) {
+        const unsigned long long t = t_lo + (unsigned long long)k;
+        if (t < end && !slot_ready(s_slot, t))
+          prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, r, s0, s1);
+      }
+    }
+    if (tid == 0) {
+      int ok = 1;
+      const unsigned long long w0 = globaltimer_ns();
+      unsigned int spins = 0;
+      while (ld_acquire_gpu(&a.bar->gen) == g_arr) {
+        if (ld_volatile_int(&st->err) != 0) {
+          ok = 0;
+          break;
+        }
+        if ((++spins & 63u) == 0u && globaltimer_ns() - w0 > kBarrierTimeoutNs) {
+          atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
+          ok = 0;
+          break;
+        }
+      }
+      __threadfence();
+      s_flag = ok && ld_volatile_int(&st->err) == 0;
+    }
+    gen = g_arr + 1u;
+    __syncthreads();
+    if (!s_flag) break;
+    const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
+
+    // ---- dS of every candidate: the NR partials in the fixed order of mlp2_trial_loop
+    for (int k0 = warp; k0 < Kb; k0 += 4 * kLoopWarps) {
+      float hi[4] = {0.0f, 0.0f, 0.0f, 0.0f}, lo[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      for (int q0 = 0; q0 < a.NR; q0 += 32 * 8) {
+        float v[4][8];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int k = k0 + u * kLoopWarps;
+          const bool live = k < Kb && s_slot[s_bslot[k]].c.gcnt > 0;
+#pragma unroll
+          for (int m = 0; m < 8; ++m) {
+            const int q = q0 + m * 32 + lane;
+            v[u][m] = (live && q < a.NR) ? part[(size_t)k * a.NR + q] : 0.0f;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int m = 0; m < 8; ++m) two_sum_add(hi[u], lo[u], v[u][m]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int k = k0 + u * kLoopWarps;
+        const float t = warp_sum_comp(hi[u], lo[u]);
+        if (lane == 0 && k < Kb)
+          s_dS[k] = s_slot[s_bslot[k]].c.valid ? t : __int_as_float(0x7fc00000);
+      }
+    }
+    __syncthreads();
+
+    // ---- decide (the same in every CTA)
+    if (warp < kKmax / 32) {
+      bool acc = false, bad = false, forced = false;
+      const int k = tid;
+      if (k < Kb && s_slot[s_bslot[k]].c.valid) {
+        const unsigned long long tk = tau + (unsigned long long)k;
+        bool facc = false;
+        if (a.nforce > 0) {
+          int lo = 0, hi = a.nforce;
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (a.ftau[mid] < tk)
+              lo = mid + 1;
+            else
+              hi = mid;
+          }
+          if (lo < a.nforce && a.ftau[lo] == tk) {
+            forced = true;
+            facc = a.facc[lo] != 0;
+          }
+        }
+        const float d = s_dS[k];
+        if (forced) {
+          acc = facc;
+        } else {
+          bad = !isfinite(d);
+          acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
+        }
+      }
+      const unsigned int ma = __ballot_sync(0xffffffffu, acc);
+      const unsigned int mb = __ballot_sync(0xffffffffu, bad);
+      const unsigned int mf = __ballot_sync(0xffffffffu, forced);
+      if (lane == 0) {
+        s_macc[warp] = ma;
+        s_mbad[warp] = mb;
+        s_mforced[warp] = mf;
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int kstar = -1, kbad = -1;
+      for (int w = 0; w < kKmax / 32 && kstar < 0; ++w)
+        if (s_macc[w]) kstar = w * 32 + __ffs(s_macc[w]) - 1;
+      for (int w = 0; w < kKmax / 32 && kbad < 0; ++w)
+        if (s_mbad[w]) kbad = w * 32 + __ffs(s_mbad[w]) - 1;
+      if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
+      s_kstar = kstar;
+      if (stats_thread) {
+        const int last = kstar >= 0 ? kstar : Kb - 1;
+        if (a.trace_cap > 0) {
+          for (int k = 0; k <= last; ++k) {
+            const Cand& c = s_slot[s_bslot[k]].c;
+            mca_trace_rec rec;
+            rec.tau = tau + (unsigned long long)k;
+            rec.idx = c.idx;
+            rec.accept = k == kstar ? 1 : 0;
+            rec.old_w = c.oldw;
+            rec.new_w = c.neww;
+            rec.valid = c.valid;
+            rec.forced = (int)((s_mforced[k >> 5] >> (k & 31)) & 1u);
+            rec.dS = (double)s_dS[k];
+            rec.S = S;
+            a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
+            ++n_trace;
+          }
+        }
+        for (int w = 0; w < kKmax / 32; ++w) {
+          unsigned int m = s_mforced[w];
+          const int hi = last - w * 32;
+          if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
+          n_forced += (unsigned long long)__popc(m);
+        }
+        n_cand += (unsigned long long)s_bvalid;
+        n_bytes += s_bbytes;
+        ++n_batch;
+        if (kstar >= 0) {
+          const Cand& c = s_slot[s_bslot[kstar]].c;
+          n_trials += (unsigned long long)(kstar + 1);
+          ++n_acc;
+          n_waste += (unsigned long long)(Kb - kstar - 1);
+          S += (double)s_dS[kstar];
+          if (c.layer == 0 && c.gcnt > 0)
+            n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
+        } else if (kstar == -1) {
+          n_trials += (unsigned long long)Kb;
+        }
+      }
+    }
+    __syncthreads();
+    const int kstar = s_kstar;
+    const unsigned long long t_d = stats_thread ? globaltimer_ns() : 0ull;
+    if (kstar == -2) {
+      if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
+      break;
+    }
+    if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
+
+    // ---- commit to this CTA's samples, then drop or patch the prepared slots it invalidates
+    if (kstar >= 0) {
+      const int sl = s_bslot[kstar];
+      const Cand c = s_slot[sl].c;
+      if (c.gcnt > 0) {
+        if (s_slot[sl].state == 1) {
+          float w[M];
+          load_w2c<NC>(s_w2c[sl], a.C, w);
+          float* zrow = a.z1 + (size_t)c.row * a.Np + s0;
+          const unsigned short* nl = e_nl + (size_t)sl * kCap;
+          const float* da = e_da + (size_t)sl * kCap;
+          const float* zn = e_zn + (size_t)sl * kCap;
+          for (int e = tid; e < c.ecnt; e += kLoopThreads) {
+            zrow[nl[e]] = zn[e];
+            (void)entry_cached<ACT2, LOSS, NC, true>(a, R, w, nl[e], da[e]);
+          }
+        } else if (c.layer == 0) {
+          float* zrow = a.z1 + (size_t)c.row * a.Np;
+          float w[M];
+          load_w2c<NC>(s_w2c[sl], a.C, w);
+          for (int e = tid; e < c.ecnt; e += kLoopThreads) {
+            const int n = __ldg(a.xs_n + c.ebeg + e);
+            const float x = __ldg(a.xs_v + c.ebeg + e);
+            (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
+                                                      zrow + n);
+          }
+        } else {
+          const float* zrow = a.z1 + (size_t)c.col * a.Np;
+          for (int e = tid; e < c.ecnt; e += kLoopThreads)
+            (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
+        }
+      }
+      if (tid == 0) {
+        const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
+        (c.layer ? a.w2 : a.w1)[off] = c.neww;
+        const int wk = c.layer ? a.wk2 : a.wk1;
+        if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
+      }
+      __syncthreads();
+      const unsigned long long t_acc = tau + (unsigned long long)kstar;
+      for (int q = tid; q < kWS; q += kLoopThreads) {
+        WSlot& o = s_slot[q];
+        if (o.state == 0 || o.tau <= t_acc || o.tau == ~0ull) continue;
+        const Cand& oc = o.c;
+        if (oc.idx == c.idx) {
+          o.state = 0;                                   // its old value changed
+        } else if (c.layer == 0 && c.gcnt > 0 && oc.layer == 0 && oc.row == c.row) {
+          o.state = 0;                                   // its hidden-field row changed
+        } else if (c.layer == 1 && oc.layer == 0 && oc.row == c.col) {
+          s_w2c[q][c.row] = c.neww;                      // its W2 column changed
+        }
+      }
+      __syncthreads();
+      tau += (unsigned long long)(kstar + 1);
+      rate_a = rate_a * kRateDecay + 1.0f;
+      rate_t = rate_t * kRateDecay + (float)(kstar + 1);
+    } else {
+      tau += (unsigned long long)Kb;
+      rate_a = rate_a * kRateDecay;
+      rate_t = rate_t * kRateDecay + (float)Kb;
+    }
+    if (stats_thread) {
+      const unsigned long long t_e = globaltimer_ns();
+      ph0 += t_b - t_a;
+      ph1 += t_c - t_b;
+      ph2 += t_d - t_c;
+      ph3 += t_e - t_d;
+    }
+    buf ^= 1;
+  }
+
+  __syncthreads();
+  {
+    const int ns = s1 - s0;
+    for (int t = tid; t < kRecFields * ns; t += kLoopThreads) {
+      const int f = t / ns, nl = t - f * ns;
+      a.srec[(size_t)f * a.Np + s0 + nl] = s_records[f * a.RS + nl];
+    }
+  }
+  if (stats_thread) {
+    st->S = S;
+    st->trials += n_trials;
+    st->accepts += n_acc;
+    st->candidates += n_cand;
+    st->batches += n_batch;
+    st->wasted += n_waste;
+    st->forced += n_forced;
+    st->alg_bytes += n_bytes;
+    st->trace_written = n_trace;
+    st->phase_ns[0] += ph0;
+    st->phase_ns[1] += ph1;
+    st->phase_ns[2] += ph2;
+    st->phase_ns[3] += ph3;
+    st->rate_acc = rate_a;
+    st->rate_trials = rate_t;
+  }
+}
+
 // Kernel variants with 10 classes: (tanh, sigmoid, MSE), (tanh, identity, CE), (Gaussian, sigmoid,
 // MSE); and a generic one that switches on transfer functions, loss and class count at run time.
 using LoopFn = void (*)(Mlp2Args);
 
+template <int A1, int A2, int LS, int NC>
+static LoopFn loop_variant(bool window) {
+  return window ? mlp2_window_loop<A1, A2, LS, NC> : mlp2_trial_loop<A1, A2, LS, NC>;
+}
+
 static LoopFn pick_loop(const Mlp2Args& a) {
+  const bool w = a.window && a.n_explicit == 0;
   if (a.C == 10) {
     if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_SIGMOID && a.loss == MCA_LOSS_MSE_ONEHOT)
-      return mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>;
+      return loop_variant<MCA_ACT_TANH, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>(w);
     if (a.act1 == MCA_ACT_TANH && a.act2 == MCA_ACT_IDENTITY && a.loss == MCA_LOSS_SOFTMAX_CE)
-      return mlp2_trial_loop<MCA_ACT_TANH, MCA_ACT_IDENTITY, MCA_LOSS_SOFTMAX_CE, 10>;
+      return loop_variant<MCA_ACT_TANH, MCA_ACT_IDENTITY, MCA_LOSS_SOFTMAX_CE, 10>(w);
     if (a.act1 == MCA_ACT_GAUSSIAN && a.act2 == MCA_ACT_SIGMOID && a.loss == MCA_LOSS_MSE_ONEHOT)
-      return mlp2_trial_loop<MCA_ACT_GAUSSIAN, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>;
+      return loop_variant<MCA_ACT_GAUSSIAN, MCA_ACT_SIGMOID, MCA_LOSS_MSE_ONEHOT, 10>(w);
   }
-  return mlp2_trial_loop<-1, -1, -1, -1>;
+  return loop_variant<-1, -1, -1, -1>(w);
 }
 
 size_t mlp2_loop_smem_bytes(const Mlp2Args& a) {
+  if (a.window && a.n_explicit == 0) return mlp2_window_smem_bytes(a.RS);
   return a.smem_records ? (size_t)a.RS * kRecFields * sizeof(float) : 0;
 }
 
