@@ -60,8 +60,8 @@ bool is_device_ptr(const void* p) {
 }
 
 struct Layout {
-  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, bar, st, trace, ex_idx,
-      ex_new, ex_out, scratch, ell, ctl, total;
+  size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, accum, bar, st, trace,
+      ex_idx, ex_new, ex_out, scratch, ell, ctl, total;
   std::vector<size_t> w_eff, code, wfix, Z;
 };
 
@@ -110,6 +110,7 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
     L.srec = take(sizeof(float) * (size_t)mca::kSR * Np);
     L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
   }
+  L.accum = take(sizeof(unsigned long long) * 3 * 2 * mca::kKmax);
   L.bar = take(sizeof(GridBarrier));
   L.st = take(sizeof(DevState));
   L.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
@@ -312,6 +313,7 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.K = h->opt.K;
   a.fixed_K = h->opt.fixed_K;
   a.partial = h->partial;
+  a.accum = h->accum;
   a.bar = h->bar;
   a.st = h->st;
   a.trace = h->trace;
@@ -742,6 +744,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     h->srec = reinterpret_cast<float*>(base + L.srec);
   }
   h->partial = reinterpret_cast<float*>(base + L.partial);
+  h->accum = reinterpret_cast<unsigned long long*>(base + L.accum);
   h->bar = reinterpret_cast<GridBarrier*>(base + L.bar);
   h->st = reinterpret_cast<DevState*>(base + L.st);
   h->trace = o.trace_cap > 0 ? reinterpret_cast<mca_trace_rec*>(base + L.trace) : nullptr;
@@ -874,6 +877,8 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     a.tau0 = h->tau;
     a.n_trials = seg;
     CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
+    CUDA_TRY(h, cudaMemsetAsync(h->accum, 0, sizeof(unsigned long long) * 3 * 2 * mca::kKmax,
+                                h->stream));
     CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
     h->launches++;
     h->tau += seg;

@@ -78,6 +78,7 @@ struct Mlp2Args {
   int K;
   int fixed_K;
   float* partial;            // [2 x kKmax x NR] per-candidate, per-range loss changes
+  unsigned long long* accum; // [3 x 2 x kKmax] windowed loop: fixed-point dS sums, bad counts
   GridBarrier* bar;
   DevState* st;
   mca_trace_rec* trace;
@@ -281,6 +282,7 @@ struct mca_handle {
   mca::DeepCtl* ctl = nullptr;
   int ntiles = 0;
   float* partial = nullptr;
+  unsigned long long* accum = nullptr;
   int NR = 0, RS = 0, SUB = 0, smem_records = 0, window = 0;
   mca::GridBarrier* bar = nullptr;
   mca::DevState* st = nullptr;

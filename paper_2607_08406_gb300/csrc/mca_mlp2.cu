@@ -767,7 +767,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   const unsigned long long end = a.tau0 + a.n_trials;
   if (tid == 0) s_tau_hi = a.tau0;
   float rate_a = st->rate_acc, rate_t = st->rate_trials;
-  int buf = 0;
+  unsigned int bidx = 0;
   const int kmaxw = min(a.K, kWS - kPF);
   __syncthreads();
 
@@ -860,11 +860,19 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       }
     }
     __syncthreads();
-    float* part = a.partial + (size_t)buf * kKmax * a.NR;
+    // this range's loss change of every candidate, added in fixed point (2^-32 units) to the
+    // candidate's 64-bit accumulator: integer sums are exact and independent of the order of
+    // arrival, so dS is the same in every CTA and for every batch width
+    unsigned long long* acc_sum = a.accum + (size_t)(bidx % 3) * 2 * kKmax;
+    unsigned long long* acc_bad = acc_sum + kKmax;
     for (int k = tid; k < Kb; k += kLoopThreads) {
+      if (s_nsub[k] == 0) continue;
       float sum = 0.0f;
       for (int q = 0; q < s_nsub[k]; ++q) sum += s_sub[s_sub0[k] + q];
-      part[(size_t)k * a.NR + r] = sum;
+      if (isfinite(sum) && fabsf(sum) < 0x1p30f)
+        atomicAdd(acc_sum + k, (unsigned long long)__float2ll_rn(sum * 0x1p32f));
+      else
+        atomicAdd(acc_bad + k, 1ull);
     }
     const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
     // ---- grid barrier, split: arrive, prepare the next slots, wait
@@ -910,33 +918,17 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     if (!s_flag) break;
     const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
 
-    // ---- dS of every candidate: the NR partials in the fixed order of mlp2_trial_loop
-    for (int k0 = warp; k0 < Kb; k0 += 4 * kLoopWarps) {
-      float hi[4] = {0.0f, 0.0f, 0.0f, 0.0f}, lo[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-      for (int q0 = 0; q0 < a.NR; q0 += 32 * 8) {
-        float v[4][8];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int k = k0 + u * kLoopWarps;
-          const bool live = k < Kb && s_slot[s_bslot[k]].c.gcnt > 0;
-#pragma unroll
-          for (int m = 0; m < 8; ++m) {
-            const int q = q0 + m * 32 + lane;
-            v[u][m] = (live && q < a.NR) ? part[(size_t)k * a.NR + q] : 0.0f;
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int m = 0; m < 8; ++m) two_sum_add(hi[u], lo[u], v[u][m]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int k = k0 + u * kLoopWarps;
-        const float t = warp_sum_comp(hi[u], lo[u]);
-        if (lane == 0 && k < Kb)
-          s_dS[k] = s_slot[s_bslot[k]].c.valid ? t : __int_as_float(0x7fc00000);
-      }
+    // ---- dS of every candidate from its accumulator
+    for (int k = tid; k < Kb; k += kLoopThreads) {
+      const Cand& c = s_slot[s_bslot[k]].c;
+      const long long q = (long long)__ldcg(acc_sum + k);
+      const unsigned long long nbad = __ldcg(acc_bad + k);
+      s_dS[k] = (!c.valid || nbad) ? __int_as_float(0x7fc00000) : __ll2float_rn(q) * 0x1p-32f;
+    }
+    // CTA 0 clears the buffer of batch bidx + 2 (last read before this batch's barrier)
+    if (r == 0) {
+      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * 2 * kKmax;
+      for (int q = tid; q < 2 * kKmax; q += kLoopThreads) z[q] = 0ull;
     }
     __syncthreads();
 
@@ -1105,7 +1097,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       ph2 += t_d - t_c;
       ph3 += t_e - t_d;
     }
-    buf ^= 1;
+    ++bidx;
   }
 
   __syncthreads();
