@@ -110,7 +110,7 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
     L.srec = take(sizeof(float) * (size_t)mca::kSR * Np);
     L.partial = take(sizeof(float) * 2 * (size_t)mca::kKmax * NR);
   }
-  L.accum = take(sizeof(unsigned long long) * 3 * 2 * mca::kKmax);
+  L.accum = take(sizeof(unsigned long long) * 3 * mca::kAccStride);
   L.bar = take(sizeof(GridBarrier));
   L.st = take(sizeof(DevState));
   L.trace = take(sizeof(mca_trace_rec) * (size_t)std::max(trace_cap, 0));
@@ -877,7 +877,7 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     a.tau0 = h->tau;
     a.n_trials = seg;
     CUDA_TRY(h, cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
-    CUDA_TRY(h, cudaMemsetAsync(h->accum, 0, sizeof(unsigned long long) * 3 * 2 * mca::kKmax,
+    CUDA_TRY(h, cudaMemsetAsync(h->accum, 0, sizeof(unsigned long long) * 3 * mca::kAccStride,
                                 h->stream));
     CUDA_TRY(h, mca::launch_mlp2_loop(a, h->stream));
     h->launches++;

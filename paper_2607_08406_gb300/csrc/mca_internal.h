@@ -32,6 +32,9 @@ constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their record
 constexpr int kWS = 96;
 constexpr int kCap = 160;
 constexpr int kPF = 32;
+// Per-batch accumulator buffer of the windowed loop: fixed-point sums [kKmax], non-finite counts
+// [kKmax], the arrival counter, padding. Three buffers rotate.
+constexpr int kAccStride = 2 * kKmax + 32;
 
 // Device-resident run state (one per handle).
 struct DevState {
@@ -78,7 +81,7 @@ struct Mlp2Args {
   int K;
   int fixed_K;
   float* partial;            // [2 x kKmax x NR] per-candidate, per-range loss changes
-  unsigned long long* accum; // [3 x 2 x kKmax] windowed loop: fixed-point dS sums, bad counts
+  unsigned long long* accum; // [3 x kAccStride] windowed loop: fixed-point sums, counts, arrivals
   GridBarrier* bar;
   DevState* st;
   mca_trace_rec* trace;

@@ -762,7 +762,6 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     S = st->S;
     n_trace = st->trace_written;
   }
-  unsigned int gen = 0;
   unsigned long long tau = a.tau0;
   const unsigned long long end = a.tau0 + a.n_trials;
   if (tid == 0) s_tau_hi = a.tau0;
@@ -863,8 +862,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     // this range's loss change of every candidate, added in fixed point (2^-32 units) to the
     // candidate's 64-bit accumulator: integer sums are exact and independent of the order of
     // arrival, so dS is the same in every CTA and for every batch width
-    unsigned long long* acc_sum = a.accum + (size_t)(bidx % 3) * 2 * kKmax;
+    unsigned long long* acc_sum = a.accum + (size_t)(bidx % 3) * kAccStride;
     unsigned long long* acc_bad = acc_sum + kKmax;
+    unsigned long long* acc_cnt = acc_sum + 2 * kKmax;     // CTAs that have added their share
     for (int k = tid; k < Kb; k += kLoopThreads) {
       if (s_nsub[k] == 0) continue;
       float sum = 0.0f;
@@ -875,17 +875,12 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         atomicAdd(acc_bad + k, 1ull);
     }
     const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
-    // ---- grid barrier, split: arrive, prepare the next slots, wait
+    // ---- grid-wide arrival on the buffer's counter (release), prepare the next slots, then wait
+    // (acquire) until every CTA has added its share; no separate barrier state
     __syncthreads();
-    unsigned int g_arr = gen;
     if (tid == 0) {
       __threadfence();
-      const unsigned int prev = atomicAdd(&a.bar->count, 1u);
-      if (prev == gridDim.x - 1) {
-        a.bar->count = 0u;
-        __threadfence();
-        st_release_gpu(&a.bar->gen, gen + 1u);
-      }
+      atomicAdd(acc_cnt, 1ull);
     }
     if (warp > 0) {
       const unsigned long long t_lo = tau + (unsigned long long)Kb;
@@ -899,7 +894,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       int ok = 1;
       const unsigned long long w0 = globaltimer_ns();
       unsigned int spins = 0;
-      while (ld_acquire_gpu(&a.bar->gen) == g_arr) {
+      while (ld_acquire_gpu_u64(acc_cnt) < (unsigned long long)gridDim.x) {
         if (ld_volatile_int(&st->err) != 0) {
           ok = 0;
           break;
@@ -913,7 +908,6 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       __threadfence();
       s_flag = ok && ld_volatile_int(&st->err) == 0;
     }
-    gen = g_arr + 1u;
     __syncthreads();
     if (!s_flag) break;
     const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
@@ -927,8 +921,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     }
     // CTA 0 clears the buffer of batch bidx + 2 (last read before this batch's barrier)
     if (r == 0) {
-      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * 2 * kKmax;
-      for (int q = tid; q < 2 * kKmax; q += kLoopThreads) z[q] = 0ull;
+      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
+      for (int q = tid; q < kAccStride; q += kLoopThreads) z[q] = 0ull;
     }
     __syncthreads();
 
