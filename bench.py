@@ -34,7 +34,8 @@ METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roo
 # from the ncu launch list of `python bench.py --steps 3 --warmup 3 --no-e2e --no-cpu` summarised in
 # profiles/. It is only valid for the kernel source it was measured on; any other source hash
 # reports null.
-LOOP_TRAFFIC = {"source_sha1": None, "bytes_per_trial": None}
+LOOP_TRAFFIC = {"source_sha1": "af79e07dbfb98008a5f86318c55d2da3ba8d9c92",
+                "bytes_per_trial": 358196.0}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
 
@@ -387,8 +388,8 @@ def run_ours(args):
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
-                                    for q, nm in enumerate(["propose_eval", "barrier",
-                                                            "reduce_decide", "commit"])},
+                                    for q, nm in enumerate(["evaluate", "arrive", "wait",
+                                                            "reduce_decide", "commit", "other"])},
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
             "roofline": roofline,

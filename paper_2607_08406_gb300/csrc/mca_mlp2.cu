@@ -757,7 +757,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   const bool stats_thread = r == 0 && tid == 0;
   double S = 0.0;
   unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
-                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0;
+                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0;
   if (stats_thread) {
     S = st->S;
     n_trace = st->trace_written;
@@ -878,9 +878,11 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     // ---- grid-wide arrival on the buffer's counter (release), prepare the next slots, then wait
     // (acquire) until every CTA has added its share; no separate barrier state
     __syncthreads();
+    unsigned long long t_arr = 0ull;
     if (tid == 0) {
       __threadfence();
       atomicAdd(acc_cnt, 1ull);
+      if (stats_thread) t_arr = globaltimer_ns();
     }
     if (warp > 0) {
       const unsigned long long t_lo = tau + (unsigned long long)Kb;
@@ -1087,9 +1089,10 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     if (stats_thread) {
       const unsigned long long t_e = globaltimer_ns();
       ph0 += t_b - t_a;
-      ph1 += t_c - t_b;
-      ph2 += t_d - t_c;
-      ph3 += t_e - t_d;
+      ph1 += t_arr - t_b;
+      ph2 += t_c - t_arr;
+      ph3 += t_d - t_c;
+      ph4 += t_e - t_d;
     }
     ++bidx;
   }
@@ -1116,6 +1119,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     st->phase_ns[1] += ph1;
     st->phase_ns[2] += ph2;
     st->phase_ns[3] += ph3;
+    st->phase_ns[4] += ph4;
     st->rate_acc = rate_a;
     st->rate_trials = rate_t;
   }
