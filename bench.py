@@ -388,8 +388,9 @@ def run_ours(args):
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
-                                    for q, nm in enumerate(["evaluate", "arrive", "wait",
-                                                            "reduce_decide", "commit", "other"])},
+                                    for q, nm in enumerate(["setup", "evaluate", "arrive", "wait",
+                                                            "reduce_decide", "commit",
+                                                            "wait_mean_all_ctas"])},
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
             "roofline": roofline,

@@ -135,9 +135,9 @@ typedef struct {
                               feature's non-zeros touch + 8 B per non-zero; per output-layer
                               candidate 4 B per sample (one hidden-field row); per accepted
                               first-layer candidate the sectors written back */
-  uint64_t phase_ns[6];    /* device time of the trial loop's first CTA in: prepare + evaluate,
-                              arrival (fence + atomic), wait for the other CTAs, reduce + decide,
-                              commit, other */
+  uint64_t phase_ns[8];    /* device time of the trial loop's first CTA in: batch set-up,
+                              evaluation, arrival (fence + atomic), wait for the other CTAs,
+                              reduce + decide, commit; [6] the wait averaged over all CTAs; [7] 0 */
   uint64_t alg_flops;      /* deep nets: FLOPs of the evaluated candidates' recomputation (2 per
                               multiply-add: the row update, the rank-1 layer, the dense layers) */
 } mca_run_stats;

@@ -457,7 +457,7 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
   s->tau = h->tau;
   s->S = d.S;
   s->alg_bytes = d.alg_bytes;
-  for (int q = 0; q < 6; ++q) s->phase_ns[q] = d.phase_ns[q];
+  for (int q = 0; q < 8; ++q) s->phase_ns[q] = d.phase_ns[q];
   s->alg_flops = d.alg_flops;
 }
 

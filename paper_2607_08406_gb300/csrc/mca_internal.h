@@ -41,7 +41,8 @@ struct DevState {
   double S;                  // loss sum of the cached state
   unsigned long long trials, accepts, candidates, batches, wasted, forced, trace_written;
   unsigned long long alg_bytes;  // compulsory DRAM bytes of the evaluated candidates and commits
-  unsigned long long phase_ns[6];  // CTA 0: evaluate, arrive, wait, reduce+decide, commit, other
+  unsigned long long phase_ns[8];  // CTA 0: set-up, evaluate, arrive, wait, reduce+decide, commit;
+                                   // [6] wait averaged over all CTAs
   unsigned long long alg_flops;    // deep path: FLOPs of the evaluated candidates' chains
   float rate_acc, rate_trials;     // decayed counts of accepts and trials (batch-width choice)
   int err;                   // first device-side error (mca_status), 0 = none

@@ -757,7 +757,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   const bool stats_thread = r == 0 && tid == 0;
   double S = 0.0;
   unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
-                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0;
+                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0,
+                     ph5 = 0, my_wait = 0;
   if (stats_thread) {
     S = st->S;
     n_trace = st->trace_written;
@@ -827,6 +828,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       }
     }
     __syncthreads();
+    const unsigned long long t_s = stats_thread ? globaltimer_ns() : 0ull;
     // ---- evaluate: warp per sub-chunk; cached slots from shared memory, the rest from global
     {
       const int total = s_total;
@@ -882,7 +884,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     if (tid == 0) {
       __threadfence();
       atomicAdd(acc_cnt, 1ull);
-      if (stats_thread) t_arr = globaltimer_ns();
+      t_arr = globaltimer_ns();
     }
     if (warp > 0) {
       const unsigned long long t_lo = tau + (unsigned long long)Kb;
@@ -909,6 +911,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       }
       __threadfence();
       s_flag = ok && ld_volatile_int(&st->err) == 0;
+      my_wait += globaltimer_ns() - t_arr;
     }
     __syncthreads();
     if (!s_flag) break;
@@ -1088,11 +1091,12 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     }
     if (stats_thread) {
       const unsigned long long t_e = globaltimer_ns();
-      ph0 += t_b - t_a;
-      ph1 += t_arr - t_b;
-      ph2 += t_c - t_arr;
-      ph3 += t_d - t_c;
-      ph4 += t_e - t_d;
+      ph0 += t_s - t_a;
+      ph1 += t_b - t_s;
+      ph2 += t_arr - t_b;
+      ph3 += t_c - t_arr;
+      ph4 += t_d - t_c;
+      ph5 += t_e - t_d;
     }
     ++bidx;
   }
@@ -1105,6 +1109,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       a.srec[(size_t)f * a.Np + s0 + nl] = s_records[f * a.RS + nl];
     }
   }
+  if (tid == 0) atomicAdd(&st->phase_ns[6], my_wait / (unsigned long long)gridDim.x);
   if (stats_thread) {
     st->S = S;
     st->trials += n_trials;
@@ -1120,6 +1125,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     st->phase_ns[2] += ph2;
     st->phase_ns[3] += ph3;
     st->phase_ns[4] += ph4;
+    st->phase_ns[5] += ph5;
     st->rate_acc = rate_a;
     st->rate_trials = rate_t;
   }
