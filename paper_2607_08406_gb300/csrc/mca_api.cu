@@ -251,7 +251,8 @@ mca_status choose_ranges(const std::vector<mca_layer>& layers, int loss, long lo
       if (mca::mlp2_loop_max_grid(probe, sms) < NR) continue;
       R.smem_records = 1;
       // the windowed loop when its records and candidate window fit next to the static state
-      if (mca::mlp2_window_smem_bytes(RS) + 24 * 1024 <= 227 * 1024) {
+      if (NR <= mca::kWindowMaxRanges &&
+          mca::mlp2_window_smem_bytes(RS) + 24 * 1024 <= 227 * 1024) {
         probe.window = 1;
         if (mca::mlp2_loop_max_grid(probe, sms) >= NR) R.window = 1;
         probe.window = 0;

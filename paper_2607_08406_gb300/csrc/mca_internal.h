@@ -32,9 +32,12 @@ constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their record
 constexpr int kWS = 96;
 constexpr int kCap = 160;
 constexpr int kPF = 32;
-// Per-batch accumulator buffer of the windowed loop: fixed-point sums [kKmax], non-finite counts
-// [kKmax], the arrival counter, padding. Three buffers rotate.
+// Per-batch accumulator buffer of the windowed loop: packed words (arrival count in bits 56..63,
+// fixed-point sum below) [kKmax], flags of out-of-range shares [kKmax], padding. Three buffers
+// rotate. One warp reads a batch's words, two per lane; the count field caps the ranges at 255.
 constexpr int kAccStride = 2 * kKmax + 32;
+constexpr int kWindowMaxRanges = 255;
+static_assert(kWS - kPF <= 64, "a windowed batch is read by one warp, two candidates per lane");
 
 // Device-resident run state (one per handle).
 struct DevState {

@@ -729,7 +729,6 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   __shared__ int s_bslot[kKmax];       // batch position -> slot
   __shared__ int s_sub0[kKmax], s_nsub[kKmax];
   __shared__ float s_dS[kKmax];
-  __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
   __shared__ int s_flag, s_kstar, s_total, s_bvalid;
   __shared__ unsigned long long s_bbytes, s_tau_hi;
   float* s_records = s_dyn;
@@ -860,32 +859,32 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         if (lane == 0) s_sub[it] = v;
       }
     }
+    if (r == 0 && warp == 1) __threadfence();    // the clearing of the previous batch (below)
     __syncthreads();
-    // this range's loss change of every candidate, added in fixed point (2^-32 units) to the
-    // candidate's 64-bit accumulator: integer sums are exact and independent of the order of
-    // arrival, so dS is the same in every CTA and for every batch width
-    unsigned long long* acc_sum = a.accum + (size_t)(bidx % 3) * kAccStride;
-    unsigned long long* acc_bad = acc_sum + kKmax;
-    unsigned long long* acc_cnt = acc_sum + 2 * kKmax;     // CTAs that have added their share
+    // this range's loss change of every candidate, added into the candidate's packed 64-bit word:
+    // bits 56..63 count the CTAs that have added, bits 0..55 hold the sum over CTAs of
+    // (share in units of 2^-26) + 2^47. Integer sums are exact and independent of the order of
+    // arrival, so dS is the same in every CTA and for every batch width; the count is the batch's
+    // only grid-wide wait. A share that is not finite or not below 2^21 in magnitude is flagged in
+    // the candidate's second word first (made visible before the count).
+    unsigned long long* acc = a.accum + (size_t)(bidx % 3) * kAccStride;
     for (int k = tid; k < Kb; k += kLoopThreads) {
-      if (s_nsub[k] == 0) continue;
+      const Cand& c = s_slot[s_bslot[k]].c;
+      if (!c.valid || c.gcnt == 0) continue;
       float sum = 0.0f;
       for (int q = 0; q < s_nsub[k]; ++q) sum += s_sub[s_sub0[k] + q];
-      if (isfinite(sum) && fabsf(sum) < 0x1p30f)
-        atomicAdd(acc_sum + k, (unsigned long long)__float2ll_rn(sum * 0x1p32f));
-      else
-        atomicAdd(acc_bad + k, 1ull);
+      unsigned long long w = (1ull << 56) + (1ull << 47);
+      if (isfinite(sum) && fabsf(sum) < 0x1p21f) {
+        w += (unsigned long long)__float2ll_rn(sum * 0x1p26f);
+      } else {
+        atomicAdd(acc + kKmax + k, 1ull);
+        __threadfence();
+      }
+      atomicAdd(acc + k, w);
     }
     const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
-    // ---- grid-wide arrival on the buffer's counter (release), prepare the next slots, then wait
-    // (acquire) until every CTA has added its share; no separate barrier state
-    __syncthreads();
-    unsigned long long t_arr = 0ull;
-    if (tid == 0) {
-      __threadfence();
-      atomicAdd(acc_cnt, 1ull);
-      t_arr = globaltimer_ns();
-    }
+    // ---- warp 0 waits until every CTA has added to every live candidate (bounded); the other
+    // warps prepare the next slots meanwhile
     if (warp > 0) {
       const unsigned long long t_lo = tau + (unsigned long long)Kb;
       for (int k = warp - 1; k < kPF; k += kLoopWarps - 1) {
@@ -893,135 +892,162 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         if (t < end && !slot_ready(s_slot, t))
           prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, r, s0, s1);
       }
-    }
-    if (tid == 0) {
+    } else {
+      const unsigned long long need = (unsigned long long)gridDim.x;
       int ok = 1;
+      unsigned long long v[2] = {0ull, 0ull};
+      bool live[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int k = lane + 32 * h;
+        live[h] = false;
+        if (k < Kb) {
+          const Cand& c = s_slot[s_bslot[k]].c;
+          live[h] = c.valid && c.gcnt > 0;
+        }
+      }
       const unsigned long long w0 = globaltimer_ns();
       unsigned int spins = 0;
-      while (ld_acquire_gpu_u64(acc_cnt) < (unsigned long long)gridDim.x) {
-        if (ld_volatile_int(&st->err) != 0) {
-          ok = 0;
-          break;
+      for (;;) {
+        bool mine = true;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (live[h] && (v[h] >> 56) < need) {
+            v[h] = ld_acquire_gpu_u64(acc + lane + 32 * h);
+            mine = mine && (v[h] >> 56) >= need;
+          }
         }
-        if ((++spins & 63u) == 0u && globaltimer_ns() - w0 > kBarrierTimeoutNs) {
-          atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
+        if (__all_sync(0xffffffffu, mine)) break;
+        int stop = 0;
+        if (lane == 0 && (++spins & 63u) == 0u) {
+          if (ld_volatile_int(&st->err) != 0) {
+            stop = 1;
+          } else if (globaltimer_ns() - w0 > kBarrierTimeoutNs) {
+            atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
+            stop = 1;
+          }
+        }
+        if (__shfl_sync(0xffffffffu, stop, 0)) {
           ok = 0;
           break;
         }
       }
-      __threadfence();
-      s_flag = ok && ld_volatile_int(&st->err) == 0;
-      my_wait += globaltimer_ns() - t_arr;
+      // ---- decide in the same warp (the same in every CTA): lowest-index candidate with
+      // dS <= 0 (Eq. 6); decisions forced by the caller take precedence; a non-finite dS at or
+      // before the first acceptance stops the run
+      unsigned int mask_a[2], mask_b[2], mask_f[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int k = lane + 32 * h;
+        bool accept = false, bad = false, forced = false;
+        if (k < Kb) {
+          const Cand& c = s_slot[s_bslot[k]].c;
+          float d = 0.0f;
+          if (!c.valid || (live[h] && ld_acquire_gpu_u64(acc + kKmax + k) != 0ull)) {
+            d = __int_as_float(0x7fc00000);
+          } else if (live[h]) {
+            const long long q = (long long)(v[h] & ((1ull << 56) - 1ull)) - (long long)(need << 47);
+            d = __ll2float_rn(q) * 0x1p-26f;
+          }
+          s_dS[k] = d;
+          if (c.valid) {
+            const unsigned long long tk = tau + (unsigned long long)k;
+            bool facc = false;
+            if (a.nforce > 0) {
+              int lo = 0, hi = a.nforce;
+              while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (a.ftau[mid] < tk)
+                  lo = mid + 1;
+                else
+                  hi = mid;
+              }
+              if (lo < a.nforce && a.ftau[lo] == tk) {
+                forced = true;
+                facc = a.facc[lo] != 0;
+              }
+            }
+            if (forced) {
+              accept = facc;
+            } else {
+              bad = !isfinite(d);
+              accept = a.strict ? (d < 0.0f) : (d <= 0.0f);
+            }
+          }
+        }
+        mask_a[h] = __ballot_sync(0xffffffffu, accept);
+        mask_b[h] = __ballot_sync(0xffffffffu, bad);
+        mask_f[h] = __ballot_sync(0xffffffffu, forced);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        my_wait += globaltimer_ns() - w0;
+        ok = ok && ld_volatile_int(&st->err) == 0;
+        s_flag = ok;
+        int kstar = mask_a[0] ? __ffs(mask_a[0]) - 1 : (mask_a[1] ? 31 + __ffs(mask_a[1]) : -1);
+        const int kbad = mask_b[0] ? __ffs(mask_b[0]) - 1 : (mask_b[1] ? 31 + __ffs(mask_b[1]) : -1);
+        if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
+        s_kstar = kstar;
+        if (stats_thread && ok) {
+          const int last = kstar >= 0 ? kstar : Kb - 1;
+          if (a.trace_cap > 0) {
+            for (int k = 0; k <= last; ++k) {
+              const Cand& c = s_slot[s_bslot[k]].c;
+              mca_trace_rec rec;
+              rec.tau = tau + (unsigned long long)k;
+              rec.idx = c.idx;
+              rec.accept = k == kstar ? 1 : 0;
+              rec.old_w = c.oldw;
+              rec.new_w = c.neww;
+              rec.valid = c.valid;
+              rec.forced = (int)((mask_f[k >> 5] >> (k & 31)) & 1u);
+              rec.dS = (double)s_dS[k];
+              rec.S = S;
+              a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
+              ++n_trace;
+            }
+          }
+#pragma unroll
+          for (int w = 0; w < 2; ++w) {
+            unsigned int m = mask_f[w];
+            const int hi = last - w * 32;
+            if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
+            n_forced += (unsigned long long)__popc(m);
+          }
+          n_cand += (unsigned long long)s_bvalid;
+          n_bytes += s_bbytes;
+          ++n_batch;
+          if (kstar >= 0) {
+            const Cand& c = s_slot[s_bslot[kstar]].c;
+            n_trials += (unsigned long long)(kstar + 1);
+            ++n_acc;
+            n_waste += (unsigned long long)(Kb - kstar - 1);
+            S += (double)s_dS[kstar];
+            if (c.layer == 0 && c.gcnt > 0)
+              n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
+          } else if (kstar == -1) {
+            n_trials += (unsigned long long)Kb;
+          }
+        }
+      }
     }
     __syncthreads();
     if (!s_flag) break;
-    const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
-
-    // ---- dS of every candidate from its accumulator
-    for (int k = tid; k < Kb; k += kLoopThreads) {
-      const Cand& c = s_slot[s_bslot[k]].c;
-      const long long q = (long long)__ldcg(acc_sum + k);
-      const unsigned long long nbad = __ldcg(acc_bad + k);
-      s_dS[k] = (!c.valid || nbad) ? __int_as_float(0x7fc00000) : __ll2float_rn(q) * 0x1p-32f;
-    }
-    // CTA 0 clears the buffer of batch bidx + 2 (last read before this batch's barrier)
-    if (r == 0) {
-      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
-      for (int q = tid; q < kAccStride; q += kLoopThreads) z[q] = 0ull;
-    }
-    __syncthreads();
-
-    // ---- decide (the same in every CTA)
-    if (warp < kKmax / 32) {
-      bool acc = false, bad = false, forced = false;
-      const int k = tid;
-      if (k < Kb && s_slot[s_bslot[k]].c.valid) {
-        const unsigned long long tk = tau + (unsigned long long)k;
-        bool facc = false;
-        if (a.nforce > 0) {
-          int lo = 0, hi = a.nforce;
-          while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (a.ftau[mid] < tk)
-              lo = mid + 1;
-            else
-              hi = mid;
-          }
-          if (lo < a.nforce && a.ftau[lo] == tk) {
-            forced = true;
-            facc = a.facc[lo] != 0;
-          }
-        }
-        const float d = s_dS[k];
-        if (forced) {
-          acc = facc;
-        } else {
-          bad = !isfinite(d);
-          acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
-        }
-      }
-      const unsigned int ma = __ballot_sync(0xffffffffu, acc);
-      const unsigned int mb = __ballot_sync(0xffffffffu, bad);
-      const unsigned int mf = __ballot_sync(0xffffffffu, forced);
-      if (lane == 0) {
-        s_macc[warp] = ma;
-        s_mbad[warp] = mb;
-        s_mforced[warp] = mf;
-      }
-    }
-    __syncthreads();
-    if (tid == 0) {
-      int kstar = -1, kbad = -1;
-      for (int w = 0; w < kKmax / 32 && kstar < 0; ++w)
-        if (s_macc[w]) kstar = w * 32 + __ffs(s_macc[w]) - 1;
-      for (int w = 0; w < kKmax / 32 && kbad < 0; ++w)
-        if (s_mbad[w]) kbad = w * 32 + __ffs(s_mbad[w]) - 1;
-      if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
-      s_kstar = kstar;
-      if (stats_thread) {
-        const int last = kstar >= 0 ? kstar : Kb - 1;
-        if (a.trace_cap > 0) {
-          for (int k = 0; k <= last; ++k) {
-            const Cand& c = s_slot[s_bslot[k]].c;
-            mca_trace_rec rec;
-            rec.tau = tau + (unsigned long long)k;
-            rec.idx = c.idx;
-            rec.accept = k == kstar ? 1 : 0;
-            rec.old_w = c.oldw;
-            rec.new_w = c.neww;
-            rec.valid = c.valid;
-            rec.forced = (int)((s_mforced[k >> 5] >> (k & 31)) & 1u);
-            rec.dS = (double)s_dS[k];
-            rec.S = S;
-            a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
-            ++n_trace;
-          }
-        }
-        for (int w = 0; w < kKmax / 32; ++w) {
-          unsigned int m = s_mforced[w];
-          const int hi = last - w * 32;
-          if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
-          n_forced += (unsigned long long)__popc(m);
-        }
-        n_cand += (unsigned long long)s_bvalid;
-        n_bytes += s_bbytes;
-        ++n_batch;
-        if (kstar >= 0) {
-          const Cand& c = s_slot[s_bslot[kstar]].c;
-          n_trials += (unsigned long long)(kstar + 1);
-          ++n_acc;
-          n_waste += (unsigned long long)(Kb - kstar - 1);
-          S += (double)s_dS[kstar];
-          if (c.layer == 0 && c.gcnt > 0)
-            n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
-        } else if (kstar == -1) {
-          n_trials += (unsigned long long)Kb;
-        }
-      }
-    }
-    __syncthreads();
     const int kstar = s_kstar;
-    const unsigned long long t_d = stats_thread ? globaltimer_ns() : 0ull;
+    const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
+    // CTA 0 clears the buffer of batch bidx + 2, which is also that of batch bidx - 1: every CTA
+    // has added its share of batch bidx, so every CTA has finished waiting on batch bidx - 1. Only
+    // the words of the first 64 candidates are used. Warp 1 fences the clearing before the
+    // __syncthreads that precedes CTA 0's additions to batch bidx + 1, for which every CTA waits
+    // before it adds to batch bidx + 2.
+    if (r == 0 && warp == 1) {
+      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
+      z[lane] = 0ull;
+      z[lane + 32] = 0ull;
+      z[kKmax + lane] = 0ull;
+      z[kKmax + lane + 32] = 0ull;
+    }
+    const unsigned long long t_d = t_c;
     if (kstar == -2) {
       if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
       break;
@@ -1093,8 +1119,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       const unsigned long long t_e = globaltimer_ns();
       ph0 += t_s - t_a;
       ph1 += t_b - t_s;
-      ph2 += t_arr - t_b;
-      ph3 += t_c - t_arr;
+      ph3 += t_c - t_b;
       ph4 += t_d - t_c;
       ph5 += t_e - t_d;
     }
