@@ -388,9 +388,10 @@ def run_ours(args):
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
-                                    for q, nm in enumerate(["setup", "evaluate", "arrive", "wait",
-                                                            "reduce_decide", "commit",
-                                                            "wait_mean_all_ctas"])},
+                                    for q, nm in enumerate(["setup", "evaluate", "wait_decide",
+                                                            "wait_cta", "add_shares", "commit",
+                                                            "slot_wait"])},
+                       "slots_reprepared": st1["phase_ns"][7] - st0["phase_ns"][7],
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},
             "roofline": roofline,

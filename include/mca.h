@@ -135,9 +135,16 @@ typedef struct {
                               feature's non-zeros touch + 8 B per non-zero; per output-layer
                               candidate 4 B per sample (one hidden-field row); per accepted
                               first-layer candidate the sectors written back */
-  uint64_t phase_ns[8];    /* device time of the trial loop's first CTA in: batch set-up,
-                              evaluation, arrival (fence + atomic), wait for the other CTAs,
-                              reduce + decide, commit; [6] the wait averaged over all CTAs; [7] 0 */
+  uint64_t phase_ns[8];    /* two-layer nets, device time per phase of the trial loop. Windowed
+                              loop (used when its shared-memory window fits), mean over CTAs:
+                              [0] batch set-up, [1] evaluation, [2] the waiting warp's wait for
+                              every CTA's shares + decision, [3] the whole CTA's wait (including
+                              the preparation of later candidates), [4] adding the CTA's shares,
+                              [5] commit, [6] the consumer warps' wait for slots still being
+                              prepared (summed over warps), [7] (a count) slots prepared again
+                              after a commit invalidated them. Other loop, first CTA:
+                              [0] proposal + evaluation, [1] grid barrier, [2] reduction +
+                              decision, [3] commit. Rest 0 */
   uint64_t alg_flops;      /* deep nets: FLOPs of the evaluated candidates' recomputation (2 per
                               multiply-add: the row update, the rank-1 layer, the dense layers) */
 } mca_run_stats;

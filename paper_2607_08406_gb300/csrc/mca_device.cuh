@@ -238,6 +238,33 @@ __device__ __forceinline__ void st_release_gpu(unsigned int* p, unsigned int v) 
   asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
+// CTA-scope acquire / release on shared memory (flags between the warps of one CTA).
+__device__ __forceinline__ unsigned long long ld_acquire_cta_shared_u64(
+    const unsigned long long* p) {
+  unsigned long long v;
+  const unsigned int a = (unsigned int)__cvta_generic_to_shared(p);
+  asm volatile("ld.acquire.cta.shared.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared_u64(unsigned long long* p,
+                                                          unsigned long long v) {
+  const unsigned int a = (unsigned int)__cvta_generic_to_shared(p);
+  asm volatile("st.release.cta.shared.u64 [%0], %1;" ::"r"(a), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire_cta_shared_s32(const int* p) {
+  int v;
+  const unsigned int a = (unsigned int)__cvta_generic_to_shared(p);
+  asm volatile("ld.acquire.cta.shared.s32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared_s32(int* p, int v) {
+  const unsigned int a = (unsigned int)__cvta_generic_to_shared(p);
+  asm volatile("st.release.cta.shared.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+
 __device__ __forceinline__ int ld_volatile_int(const int* p) {
   return *reinterpret_cast<const volatile int*>(p);
 }

@@ -27,17 +27,18 @@ constexpr float kWidthMlp2 = 3.0f;
 constexpr float kWidthDeep = 1.5f;  // samples per range below which fewer CTAs are used
 constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
 // Window of the trial loop: kWS candidate slots per CTA, each caching up to kCap entries of the
-// candidate's segment (range-local sample, activation change, new hidden field); kPF of them are
-// prepared while the CTA waits at the grid barrier. Batches are at most kWS - kPF wide.
+// candidate's segment (range-local sample, activation change, new hidden field), prepared ahead of
+// the batches. Batches are at most kWinBatch wide.
 constexpr int kWS = 96;
 constexpr int kCap = 160;
-constexpr int kPF = 32;
-// Per-batch accumulator buffer of the windowed loop: packed words (arrival count in bits 56..63,
-// fixed-point sum below) [kKmax], flags of out-of-range shares [kKmax], padding. Three buffers
-// rotate. One warp reads a batch's words, two per lane; the count field caps the ranges at 255.
+constexpr int kWinBatch = 64;
+// Per-batch accumulator buffer of the windowed loop: one packed word per candidate (arrival count
+// in bits 56..63, count of out-of-range shares in 48..55, fixed-point sum below), padding. Three
+// buffers rotate. One warp reads a batch's words, two per lane; the count fields cap the ranges at
+// 255.
 constexpr int kAccStride = 2 * kKmax + 32;
 constexpr int kWindowMaxRanges = 255;
-static_assert(kWS - kPF <= 64, "a windowed batch is read by one warp, two candidates per lane");
+static_assert(kWinBatch <= 64 && kWinBatch < kWS, "a windowed batch is read by one warp, two per lane");
 
 // Device-resident run state (one per handle).
 struct DevState {

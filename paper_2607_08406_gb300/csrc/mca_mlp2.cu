@@ -617,17 +617,49 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
 // keeps a ring of kWS candidate slots: slot (t mod kWS) holds trial t's candidate for this CTA's range
 // and, for first-layer candidates with at most kCap entries in the range, the gathered entries
 // (range-local sample, activation change f(z + delta x) - f(z), new field z + delta x). A batch then
-// evaluates and commits from shared memory only. While thread 0 waits at the grid barrier, the other
-// warps prepare the next kPF slots (Philox, weight, CSR and z1 gathers). After a commit every prepared
-// slot that depends on what changed is dropped or patched: the same weight (old value), a first-layer
-// candidate of the same hidden row (z1 changed), or the W2 column of a first-layer candidate.
+// evaluates and commits from shared memory only.
+//
+// The CTA's warps have two roles. kProdWarps producer warps prepare slots ahead of the batches
+// (Philox, weight, CSR and z1 gathers), in trial order, never more than kWS trials ahead; they take
+// no part in the batch's barriers, so their memory latency overlaps everything else. The other
+// (consumer) warps run the batches: set-up, evaluation, the grid-wide exchange, decision, commit.
+// A slot records how many commits this CTA had made when its preparation began (its epoch); every
+// commit is appended to a log. Before a batch uses a slot, the log entries since its epoch are
+// replayed: a commit of the same weight (its old value changed) or of a first-layer weight on the
+// same hidden row (z1 changed) sends the slot back for preparation; a commit of its W2 column is
+// patched in.
 // ------------------------------------------------------------------------------------------------
 struct WSlot {
   Cand c;
-  unsigned long long tau;
-  int state;                 // 0 empty, 1 entries cached (or nothing to evaluate), 2 read from global
-  int pad;
+  unsigned long long ticket;  // trial + 1 once the slot is ready for it (written last)
+  int state;                  // 1 entries cached (or nothing to evaluate), 2 read from global
+  int epoch;                  // commits of this CTA before the slot's data were read
 };
+
+// One logged commit of the windowed loop.
+struct CommitLog {
+  unsigned int idx;
+  int layer, row, col;
+  float neww;
+  int changes_z1;             // a first-layer commit with entries: its z1 row changed
+};
+
+// Per-phase device timers of the windowed loop (statistics only; each read of the global timer
+// sits on the batch's critical path). Built in with -DMCA_PHASE_TIMERS=1.
+#ifndef MCA_PHASE_TIMERS
+#define MCA_PHASE_TIMERS 0
+#endif
+constexpr bool kPhaseTimers = MCA_PHASE_TIMERS != 0;
+constexpr int kLogLen = 128;
+static_assert(kLogLen > kWS, "a slot is used at most kWS commits after its preparation began");
+constexpr int kProdWarps = 4;
+constexpr int kConsWarps = kLoopWarps - kProdWarps;
+constexpr int kConsThreads = kConsWarps * 32;
+
+// Barrier of the consumer warps only (named barrier 1).
+__device__ __forceinline__ void cons_sync() {
+  asm volatile("bar.sync 1, %0;" ::"r"(kConsThreads) : "memory");
+}
 
 size_t mlp2_window_smem_bytes(int RS) {
   return sizeof(float) * (size_t)kRecFields * RS +
@@ -655,11 +687,12 @@ __device__ __forceinline__ float entry_cached(const Mlp2Args& a, Recs R,
 }
 
 // Warp prepares slot sl for trial t: proposal, W2 column, and (cacheable first-layer candidates)
-// the gathered entries.
+// the gathered entries; then publishes it. `epoch` was read before any of the data.
 template <int ACT1>
 __device__ __forceinline__ void prepare_slot(const Mlp2Args& a, WSlot* slots, float (*w2c)[kMaxC],
                                              unsigned short* e_nl, float* e_da, float* e_zn,
-                                             int sl, unsigned long long t, int r, int s0, int s1) {
+                                             int sl, unsigned long long t, int epoch, int r, int s0,
+                                             int s1) {
   const int lane = threadIdx.x & 31;
   if (lane == 0) {
     const uint4 w = trial_words(a.seed, t);
@@ -667,8 +700,7 @@ __device__ __forceinline__ void prepare_slot(const Mlp2Args& a, WSlot* slots, fl
     Cand c;
     fill_candidate(a, idx, w.y, false, 0.0f, r, s0, s1, c);
     slots[sl].c = c;
-    slots[sl].tau = t;
-    slots[sl].state = 0;
+    slots[sl].epoch = epoch;
   }
   __syncwarp();
   const Cand c = slots[sl].c;
@@ -712,12 +744,51 @@ __device__ __forceinline__ void prepare_slot(const Mlp2Args& a, WSlot* slots, fl
     state = 1;
   }
   __syncwarp();
-  if (lane == 0) slots[sl].state = state;
+  if (lane == 0) {
+    slots[sl].state = state;
+    st_release_cta_shared_u64(&slots[sl].ticket, t + 1ull);
+  }
+  __syncwarp();
 }
 
+// Acquires the slot's data when it is ready for trial t.
 __device__ __forceinline__ bool slot_ready(const WSlot* slots, unsigned long long t) {
-  const WSlot& s = slots[t % kWS];
-  return s.tau == t && s.state != 0;
+  return ld_acquire_cta_shared_u64(&slots[t % kWS].ticket) == t + 1ull;
+}
+
+// The warp replays the commits [slot epoch, epoch) on a ready slot, 32 log entries at a time.
+// Returns false (in every lane) when the slot must be prepared again.
+__device__ __forceinline__ bool revalidate(WSlot& s, float* w2c, const CommitLog* log, int epoch) {
+  const int lane = threadIdx.x & 31;
+  const int e0 = s.epoch;
+  if (epoch - e0 >= kLogLen) return false;
+  const unsigned int idx = s.c.idx;
+  const int layer = s.c.layer, row = s.c.row;
+  for (int base = e0; base < epoch; base += 32) {
+    const int e = base + lane;
+    bool stale = false, patch = false;
+    int prow = 0;
+    float pval = 0.0f;
+    if (e < epoch) {
+      const CommitLog& L = log[e % kLogLen];
+      stale = L.idx == idx || (layer == 0 && L.layer == 0 && L.changes_z1 && L.row == row);
+      patch = layer == 0 && L.layer == 1 && L.col == row;
+      prow = L.row;
+      pval = L.neww;
+    }
+    if (__any_sync(0xffffffffu, stale)) return false;
+    unsigned int pm = __ballot_sync(0xffffffffu, patch);
+    while (pm) {                       // in commit order: the latest value of a row wins
+      const int j = __ffs(pm) - 1;
+      pm &= pm - 1u;
+      if (lane == j) w2c[prow] = pval;
+      __syncwarp();
+    }
+  }
+  __syncwarp();
+  if (lane == 0) s.epoch = epoch;
+  __syncwarp();
+  return true;
 }
 
 template <int ACT1, int ACT2, int LOSS, int NC>
@@ -726,11 +797,12 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   __shared__ WSlot s_slot[kWS];
   __shared__ float s_w2c[kWS][kMaxC];
   __shared__ float s_sub[kKmax * kMaxSubs];
+  __shared__ CommitLog s_log[kLogLen];
   __shared__ int s_bslot[kKmax];       // batch position -> slot
   __shared__ int s_sub0[kKmax], s_nsub[kKmax];
   __shared__ float s_dS[kKmax];
-  __shared__ int s_flag, s_kstar, s_total, s_bvalid;
-  __shared__ unsigned long long s_bbytes, s_tau_hi;
+  __shared__ int s_flag, s_kstar, s_total, s_bvalid, s_fail, s_done, s_epoch;
+  __shared__ unsigned long long s_bbytes, s_tau_hi, s_next, s_cons_tau;
   float* s_records = s_dyn;
   unsigned short* e_nl = reinterpret_cast<unsigned short*>(s_dyn + kRecFields * a.RS);
   float* e_da = reinterpret_cast<float*>(e_nl + kWS * kCap);
@@ -748,382 +820,465 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       s_records[f * a.RS + nl] = a.srec[(size_t)f * a.Np + s0 + nl];
     }
   }
-  for (int q = tid; q < kWS; q += kLoopThreads) {
-    s_slot[q].state = 0;
-    s_slot[q].tau = ~0ull;
-  }
+  for (int q = tid; q < kWS; q += kLoopThreads) s_slot[q].ticket = 0ull;
   DevState* st = a.st;
-  const bool stats_thread = r == 0 && tid == 0;
-  double S = 0.0;
-  unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
-                     n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0,
-                     ph5 = 0, my_wait = 0;
-  if (stats_thread) {
-    S = st->S;
-    n_trace = st->trace_written;
-  }
   unsigned long long tau = a.tau0;
   const unsigned long long end = a.tau0 + a.n_trials;
-  if (tid == 0) s_tau_hi = a.tau0;
-  float rate_a = st->rate_acc, rate_t = st->rate_trials;
-  unsigned int bidx = 0;
-  const int kmaxw = min(a.K, kWS - kPF);
+  if (tid == 0) {
+    s_tau_hi = a.tau0;
+    s_next = a.tau0;
+    s_cons_tau = a.tau0;
+    s_fail = 0;
+    s_done = 0;
+    s_epoch = 0;
+  }
   __syncthreads();
 
-  while (tau < end) {
-    const unsigned long long t_a = stats_thread ? globaltimer_ns() : 0ull;
-    const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
-    const int Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
-    // ---- slots of this batch (prepared ahead in the common case)
-    for (int k = warp; k < Kb; k += kLoopWarps) {
-      const unsigned long long t = tau + (unsigned long long)k;
-      if (!slot_ready(s_slot, t))
-        prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, r, s0, s1);
-    }
-    __syncthreads();
-    if (warp == 0) {                 // sub-chunk scan and batch statistics
-      int v[4], loc = 0;
-      unsigned long long bytes = 0ull;
-      int valid = 0;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int k = lane * 4 + u;
-        v[u] = 0;
-        if (k < Kb) {
-          const int sl = (int)((tau + (unsigned long long)k) % kWS);
-          s_bslot[k] = sl;
-          const Cand& c = s_slot[sl].c;
-          v[u] = c.nsub;
-          if (tau + (unsigned long long)k >= s_tau_hi) bytes += c.bytes;
-          valid += c.valid;
-        }
-        loc += v[u];
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
-        valid += __shfl_xor_sync(0xffffffffu, valid, o);
-      }
-      int inc = loc;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, inc, o);
-        if (lane >= o) inc += y;
-      }
-      int ex = inc - loc;
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int k = lane * 4 + u;
-        if (k < Kb) {
-          s_sub0[k] = ex;
-          s_nsub[k] = v[u];
-        }
-        ex += v[u];
-      }
-      if (lane == 31) s_total = inc;
+  if (warp >= kConsWarps) {
+    // ---- producers: prepare slots in trial order, at most kWS trials ahead of the batch
+    for (;;) {
+      unsigned long long t = 0ull;
+      if (lane == 0) t = atomicAdd(&s_next, 1ull);
+      t = __shfl_sync(0xffffffffu, t, 0);
+      if (t >= end) break;
+      int go = 1;
       if (lane == 0) {
-        s_bbytes = bytes;
-        s_bvalid = valid;
-      }
-    }
-    __syncthreads();
-    const unsigned long long t_s = stats_thread ? globaltimer_ns() : 0ull;
-    // ---- evaluate: warp per sub-chunk; cached slots from shared memory, the rest from global
-    {
-      const int total = s_total;
-      int k = 0;
-      for (int it = warp; it < total; it += kLoopWarps) {
-        while (s_sub0[k] + s_nsub[k] <= it) ++k;
-        const int sl = s_bslot[k];
-        const Cand& c = s_slot[sl].c;
-        const int q = it - s_sub0[k];
-        float v;
-        if (s_slot[sl].state == 1) {
-          float w[M];
-          load_w2c<NC>(s_w2c[sl], a.C, w);
-          const unsigned short* nl = e_nl + (size_t)sl * kCap;
-          const float* da = e_da + (size_t)sl * kCap;
-          const int e_lo = q * a.SUB, e_hi = min(e_lo + a.SUB, c.ecnt);
-          float acc = 0.0f;
-          for (int g = e_lo; g < e_hi; g += 128) {
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const int e = g + u * 32 + lane;
-              if (e < e_hi) acc += entry_cached<ACT2, LOSS, NC, false>(a, R, w, nl[e], da[e]);
-            }
+        const unsigned long long w0 = globaltimer_ns();
+        while (t >= *(volatile unsigned long long*)&s_cons_tau + (unsigned long long)kWS) {
+          if (*(volatile int*)&s_done) {
+            go = 0;
+            break;
           }
-          v = warp_sum(acc);
-        } else {
-          v = eval_sub<ACT1, ACT2, LOSS, NC>(a, R, s0, c, s_w2c[sl], q);
+          if (globaltimer_ns() - w0 > kBarrierTimeoutNs) {
+            atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);   // the consumers stop at their decision
+            go = 0;
+            break;
+          }
+          __nanosleep(64);
         }
-        if (lane == 0) s_sub[it] = v;
       }
+      if (!__shfl_sync(0xffffffffu, go, 0)) break;
+      int epoch = 0;
+      if (lane == 0) epoch = ld_acquire_cta_shared_s32(&s_epoch);
+      __syncwarp();
+      epoch = __shfl_sync(0xffffffffu, epoch, 0);
+      prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, epoch, r, s0, s1);
     }
-    if (r == 0 && warp == 1) __threadfence();    // the clearing of the previous batch (below)
-    __syncthreads();
-    // this range's loss change of every candidate, added into the candidate's packed 64-bit word:
-    // bits 56..63 count the CTAs that have added, bits 0..55 hold the sum over CTAs of
-    // (share in units of 2^-26) + 2^47. Integer sums are exact and independent of the order of
-    // arrival, so dS is the same in every CTA and for every batch width; the count is the batch's
-    // only grid-wide wait. A share that is not finite or not below 2^21 in magnitude is flagged in
-    // the candidate's second word first (made visible before the count).
-    unsigned long long* acc = a.accum + (size_t)(bidx % 3) * kAccStride;
-    for (int k = tid; k < Kb; k += kLoopThreads) {
-      const Cand& c = s_slot[s_bslot[k]].c;
-      if (!c.valid || c.gcnt == 0) continue;
-      float sum = 0.0f;
-      for (int q = 0; q < s_nsub[k]; ++q) sum += s_sub[s_sub0[k] + q];
-      unsigned long long w = (1ull << 56) + (1ull << 47);
-      if (isfinite(sum) && fabsf(sum) < 0x1p21f) {
-        w += (unsigned long long)__float2ll_rn(sum * 0x1p26f);
-      } else {
-        atomicAdd(acc + kKmax + k, 1ull);
-        __threadfence();
-      }
-      atomicAdd(acc + k, w);
+  } else {
+    // ---- consumers: the batches
+    const bool stats_thread = r == 0 && tid == 0;
+    const bool timer = kPhaseTimers && tid == 0;   // phase times of every CTA, mean over CTAs
+    double S = 0.0;
+    unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
+                       n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0,
+                       ph5 = 0, n_starve = 0, n_reprep = 0;
+    if (stats_thread) {
+      S = st->S;
+      n_trace = st->trace_written;
     }
-    const unsigned long long t_b = stats_thread ? globaltimer_ns() : 0ull;
-    // ---- warp 0 waits until every CTA has added to every live candidate (bounded); the other
-    // warps prepare the next slots meanwhile
-    if (warp > 0) {
-      const unsigned long long t_lo = tau + (unsigned long long)Kb;
-      for (int k = warp - 1; k < kPF; k += kLoopWarps - 1) {
-        const unsigned long long t = t_lo + (unsigned long long)k;
-        if (t < end && !slot_ready(s_slot, t))
-          prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, r, s0, s1);
+    float rate_a = st->rate_acc, rate_t = st->rate_trials;
+    unsigned int bidx = 0;
+    int epoch = 0;                     // commits of this CTA so far (consumer copy of s_epoch)
+    const int kmaxw = min(a.K, kWinBatch);
+
+    while (tau < end) {
+      const unsigned long long t_a = timer ? globaltimer_ns() : 0ull;
+      if (tid == 0) *(volatile unsigned long long*)&s_cons_tau = tau;
+      const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
+      const int Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
+      // ---- slots of this batch: wait for the producers (bounded), replay the commits since
+      // their preparation, prepare again what they invalidate
+      for (int k = warp; k < Kb; k += kConsWarps) {
+        const unsigned long long t = tau + (unsigned long long)k;
+        const int sl = (int)(t % kWS);
+        int ok = 1;
+        if (lane == 0) {
+          if (!slot_ready(s_slot, t)) {
+            const unsigned long long w0 = globaltimer_ns();
+            unsigned int spins = 0;
+            while (!slot_ready(s_slot, t)) {
+              if ((++spins & 63u) == 0u && globaltimer_ns() - w0 > kBarrierTimeoutNs) {
+                atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
+                *(volatile int*)&s_fail = 1;
+                ok = 0;
+                break;
+              }
+            }
+            if (kPhaseTimers) n_starve += globaltimer_ns() - w0;
+          }
+        }
+        __syncwarp();
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (ok == 1 && !revalidate(s_slot[sl], s_w2c[sl], s_log, epoch)) {
+          ok = 2;
+          if (lane == 0) ++n_reprep;
+        }
+        if (ok == 2)
+          prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, sl, t, epoch, r, s0, s1);
       }
-    } else {
-      const unsigned long long need = (unsigned long long)gridDim.x;
-      int ok = 1;
-      unsigned long long v[2] = {0ull, 0ull};
-      bool live[2];
+      cons_sync();
+      if (*(volatile int*)&s_fail) break;
+      if (warp == 0) {                 // sub-chunk scan and batch statistics
+        int v[4], loc = 0;
+        unsigned long long bytes = 0ull;
+        int valid = 0;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int k = lane + 32 * h;
-        live[h] = false;
-        if (k < Kb) {
-          const Cand& c = s_slot[s_bslot[k]].c;
-          live[h] = c.valid && c.gcnt > 0;
+        for (int u = 0; u < 4; ++u) {
+          const int k = lane * 4 + u;
+          v[u] = 0;
+          if (k < Kb) {
+            const int sl = (int)((tau + (unsigned long long)k) % kWS);
+            s_bslot[k] = sl;
+            const Cand& c = s_slot[sl].c;
+            v[u] = c.nsub;
+            if (tau + (unsigned long long)k >= s_tau_hi) bytes += c.bytes;
+            valid += c.valid;
+          }
+          loc += v[u];
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
+          valid += __shfl_xor_sync(0xffffffffu, valid, o);
+        }
+        int inc = loc;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, inc, o);
+          if (lane >= o) inc += y;
+        }
+        int ex = inc - loc;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int k = lane * 4 + u;
+          if (k < Kb) {
+            s_sub0[k] = ex;
+            s_nsub[k] = v[u];
+          }
+          ex += v[u];
+        }
+        if (lane == 31) s_total = inc;
+        if (lane == 0) {
+          s_bbytes = bytes;
+          s_bvalid = valid;
         }
       }
-      const unsigned long long w0 = globaltimer_ns();
-      unsigned int spins = 0;
-      for (;;) {
-        bool mine = true;
+      cons_sync();
+      const unsigned long long t_s = timer ? globaltimer_ns() : 0ull;
+      // ---- evaluate: warp per sub-chunk; cached slots from shared memory, the rest from global
+      {
+        const int total = s_total;
+        int k = 0;
+        for (int it = warp; it < total; it += kConsWarps) {
+          while (s_sub0[k] + s_nsub[k] <= it) ++k;
+          const int sl = s_bslot[k];
+          const Cand& c = s_slot[sl].c;
+          const int q = it - s_sub0[k];
+          float v;
+          if (s_slot[sl].state == 1) {
+            float w[M];
+            load_w2c<NC>(s_w2c[sl], a.C, w);
+            const unsigned short* nl = e_nl + (size_t)sl * kCap;
+            const float* da = e_da + (size_t)sl * kCap;
+            const int e_lo = q * a.SUB, e_hi = min(e_lo + a.SUB, c.ecnt);
+            float acc = 0.0f;
+            for (int g = e_lo; g < e_hi; g += 128) {
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const int e = g + u * 32 + lane;
+                if (e < e_hi) acc += entry_cached<ACT2, LOSS, NC, false>(a, R, w, nl[e], da[e]);
+              }
+            }
+            v = warp_sum(acc);
+          } else {
+            v = eval_sub<ACT1, ACT2, LOSS, NC>(a, R, s0, c, s_w2c[sl], q);
+          }
+          if (lane == 0) s_sub[it] = v;
+        }
+      }
+      const unsigned long long t_v = timer ? globaltimer_ns() : 0ull;
+      if (r == 0 && warp == 1) __threadfence();    // the clearing of the previous batch (below)
+      cons_sync();
+      // this range's loss change of every candidate, added into the candidate's packed 64-bit
+      // word: bits 56..63 count the CTAs that have added, bits 48..55 those whose share was not
+      // finite or not below 2^19 in magnitude, bits 0..47 the sum over the other CTAs of
+      // (share in units of 2^-20) + 2^39. Integer sums are exact and independent of the order of
+      // arrival, so dS is the same in every CTA and for every batch width; the count is the
+      // batch's only grid-wide wait, and one load of the word gives everything.
+      unsigned long long* acc = a.accum + (size_t)(bidx % 3) * kAccStride;
+      for (int k = tid; k < Kb; k += kConsThreads) {
+        const Cand& c = s_slot[s_bslot[k]].c;
+        if (!c.valid || c.gcnt == 0) continue;
+        float sum = 0.0f;
+        for (int q = 0; q < s_nsub[k]; ++q) sum += s_sub[s_sub0[k] + q];
+        unsigned long long w = 1ull << 56;
+        if (isfinite(sum) && fabsf(sum) < 0x1p19f)
+          w += (1ull << 39) + (unsigned long long)__float2ll_rn(sum * 0x1p20f);
+        else
+          w += 1ull << 48;
+        atomicAdd(acc + k, w);
+      }
+      const unsigned long long t_b = timer ? globaltimer_ns() : 0ull;
+      // ---- warp 0 waits until every CTA has added to every live candidate (bounded), then
+      // decides
+      if (warp == 0) {
+        const unsigned long long need = (unsigned long long)gridDim.x;
+        int ok = 1;
+        unsigned long long v[2] = {0ull, 0ull};
+        bool live[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          if (live[h] && (v[h] >> 56) < need) {
-            v[h] = ld_acquire_gpu_u64(acc + lane + 32 * h);
-            mine = mine && (v[h] >> 56) >= need;
+          const int k = lane + 32 * h;
+          live[h] = false;
+          if (k < Kb) {
+            const Cand& c = s_slot[s_bslot[k]].c;
+            live[h] = c.valid && c.gcnt > 0;
           }
         }
-        if (__all_sync(0xffffffffu, mine)) break;
-        int stop = 0;
-        if (lane == 0 && (++spins & 63u) == 0u) {
-          if (ld_volatile_int(&st->err) != 0) {
-            stop = 1;
-          } else if (globaltimer_ns() - w0 > kBarrierTimeoutNs) {
-            atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
-            stop = 1;
-          }
-        }
-        if (__shfl_sync(0xffffffffu, stop, 0)) {
-          ok = 0;
-          break;
-        }
-      }
-      // ---- decide in the same warp (the same in every CTA): lowest-index candidate with
-      // dS <= 0 (Eq. 6); decisions forced by the caller take precedence; a non-finite dS at or
-      // before the first acceptance stops the run
-      unsigned int mask_a[2], mask_b[2], mask_f[2];
+        // the clock is read only once the wait has lasted 64 polls (and for the phase timers)
+        unsigned long long w0 = kPhaseTimers ? globaltimer_ns() : 0ull;
+        unsigned int spins = 0;
+        for (;;) {
+          bool mine = true;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int k = lane + 32 * h;
-        bool accept = false, bad = false, forced = false;
-        if (k < Kb) {
-          const Cand& c = s_slot[s_bslot[k]].c;
-          float d = 0.0f;
-          if (!c.valid || (live[h] && ld_acquire_gpu_u64(acc + kKmax + k) != 0ull)) {
-            d = __int_as_float(0x7fc00000);
-          } else if (live[h]) {
-            const long long q = (long long)(v[h] & ((1ull << 56) - 1ull)) - (long long)(need << 47);
-            d = __ll2float_rn(q) * 0x1p-26f;
+          for (int h = 0; h < 2; ++h) {
+            if (live[h] && (v[h] >> 56) < need) {
+              v[h] = ld_acquire_gpu_u64(acc + lane + 32 * h);
+              mine = mine && (v[h] >> 56) >= need;
+            }
           }
-          s_dS[k] = d;
-          if (c.valid) {
-            const unsigned long long tk = tau + (unsigned long long)k;
-            bool facc = false;
-            if (a.nforce > 0) {
-              int lo = 0, hi = a.nforce;
-              while (lo < hi) {
-                const int mid = (lo + hi) >> 1;
-                if (a.ftau[mid] < tk)
-                  lo = mid + 1;
-                else
-                  hi = mid;
-              }
-              if (lo < a.nforce && a.ftau[lo] == tk) {
-                forced = true;
-                facc = a.facc[lo] != 0;
-              }
+          if (__all_sync(0xffffffffu, mine)) break;
+          int stop = 0;
+          if (lane == 0 && (++spins & 63u) == 0u) {
+            const unsigned long long now = globaltimer_ns();
+            if (spins == 64u && !kPhaseTimers) w0 = now;
+            if (ld_volatile_int(&st->err) != 0) {
+              stop = 1;
+            } else if (now - w0 > kBarrierTimeoutNs) {
+              atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
+              stop = 1;
             }
-            if (forced) {
-              accept = facc;
-            } else {
-              bad = !isfinite(d);
-              accept = a.strict ? (d < 0.0f) : (d <= 0.0f);
-            }
+          }
+          if (__shfl_sync(0xffffffffu, stop, 0)) {
+            ok = 0;
+            break;
           }
         }
-        mask_a[h] = __ballot_sync(0xffffffffu, accept);
-        mask_b[h] = __ballot_sync(0xffffffffu, bad);
-        mask_f[h] = __ballot_sync(0xffffffffu, forced);
-      }
-      __syncwarp();
-      if (lane == 0) {
-        my_wait += globaltimer_ns() - w0;
-        ok = ok && ld_volatile_int(&st->err) == 0;
-        s_flag = ok;
-        int kstar = mask_a[0] ? __ffs(mask_a[0]) - 1 : (mask_a[1] ? 31 + __ffs(mask_a[1]) : -1);
-        const int kbad = mask_b[0] ? __ffs(mask_b[0]) - 1 : (mask_b[1] ? 31 + __ffs(mask_b[1]) : -1);
-        if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
-        s_kstar = kstar;
-        if (stats_thread && ok) {
-          const int last = kstar >= 0 ? kstar : Kb - 1;
-          if (a.trace_cap > 0) {
-            for (int k = 0; k <= last; ++k) {
-              const Cand& c = s_slot[s_bslot[k]].c;
-              mca_trace_rec rec;
-              rec.tau = tau + (unsigned long long)k;
-              rec.idx = c.idx;
-              rec.accept = k == kstar ? 1 : 0;
-              rec.old_w = c.oldw;
-              rec.new_w = c.neww;
-              rec.valid = c.valid;
-              rec.forced = (int)((mask_f[k >> 5] >> (k & 31)) & 1u);
-              rec.dS = (double)s_dS[k];
-              rec.S = S;
-              a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
-              ++n_trace;
-            }
-          }
+        // decide in the same warp (the same in every CTA): lowest-index candidate with dS <= 0
+        // (Eq. 6); decisions forced by the caller take precedence; a non-finite dS at or before
+        // the first acceptance stops the run
+        unsigned int mask_a[2], mask_b[2], mask_f[2];
 #pragma unroll
-          for (int w = 0; w < 2; ++w) {
-            unsigned int m = mask_f[w];
-            const int hi = last - w * 32;
-            if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
-            n_forced += (unsigned long long)__popc(m);
+        for (int h = 0; h < 2; ++h) {
+          const int k = lane + 32 * h;
+          bool accept = false, bad = false, forced = false;
+          if (k < Kb) {
+            const Cand& c = s_slot[s_bslot[k]].c;
+            float d = 0.0f;
+            const unsigned long long nbad = (v[h] >> 48) & 255ull;
+            if (!c.valid || (live[h] && nbad != 0ull)) {
+              d = __int_as_float(0x7fc00000);
+            } else if (live[h]) {
+              const long long q =
+                  (long long)(v[h] & ((1ull << 48) - 1ull)) - (long long)(need << 39);
+              d = __ll2float_rn(q) * 0x1p-20f;
+            }
+            s_dS[k] = d;
+            if (c.valid) {
+              const unsigned long long tk = tau + (unsigned long long)k;
+              bool facc = false;
+              if (a.nforce > 0) {
+                int lo = 0, hi = a.nforce;
+                while (lo < hi) {
+                  const int mid = (lo + hi) >> 1;
+                  if (a.ftau[mid] < tk)
+                    lo = mid + 1;
+                  else
+                    hi = mid;
+                }
+                if (lo < a.nforce && a.ftau[lo] == tk) {
+                  forced = true;
+                  facc = a.facc[lo] != 0;
+                }
+              }
+              if (forced) {
+                accept = facc;
+              } else {
+                bad = !isfinite(d);
+                accept = a.strict ? (d < 0.0f) : (d <= 0.0f);
+              }
+            }
           }
-          n_cand += (unsigned long long)s_bvalid;
-          n_bytes += s_bbytes;
-          ++n_batch;
-          if (kstar >= 0) {
-            const Cand& c = s_slot[s_bslot[kstar]].c;
-            n_trials += (unsigned long long)(kstar + 1);
-            ++n_acc;
-            n_waste += (unsigned long long)(Kb - kstar - 1);
-            S += (double)s_dS[kstar];
-            if (c.layer == 0 && c.gcnt > 0)
-              n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
-          } else if (kstar == -1) {
-            n_trials += (unsigned long long)Kb;
+          mask_a[h] = __ballot_sync(0xffffffffu, accept);
+          mask_b[h] = __ballot_sync(0xffffffffu, bad);
+          mask_f[h] = __ballot_sync(0xffffffffu, forced);
+        }
+        __syncwarp();
+        if (lane == 0) {
+          if (kPhaseTimers) ph2 += globaltimer_ns() - w0;
+          s_flag = ok;                 // an error elsewhere ends this CTA's next wait
+          int kstar = mask_a[0] ? __ffs(mask_a[0]) - 1 : (mask_a[1] ? 31 + __ffs(mask_a[1]) : -1);
+          const int kbad =
+              mask_b[0] ? __ffs(mask_b[0]) - 1 : (mask_b[1] ? 31 + __ffs(mask_b[1]) : -1);
+          if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
+          s_kstar = kstar;
+          if (stats_thread && ok) {
+            const int last = kstar >= 0 ? kstar : Kb - 1;
+            if (a.trace_cap > 0) {
+              for (int k = 0; k <= last; ++k) {
+                const Cand& c = s_slot[s_bslot[k]].c;
+                mca_trace_rec rec;
+                rec.tau = tau + (unsigned long long)k;
+                rec.idx = c.idx;
+                rec.accept = k == kstar ? 1 : 0;
+                rec.old_w = c.oldw;
+                rec.new_w = c.neww;
+                rec.valid = c.valid;
+                rec.forced = (int)((mask_f[k >> 5] >> (k & 31)) & 1u);
+                rec.dS = (double)s_dS[k];
+                rec.S = S;
+                a.trace[n_trace % (unsigned long long)a.trace_cap] = rec;
+                ++n_trace;
+              }
+            }
+#pragma unroll
+            for (int w = 0; w < 2; ++w) {
+              unsigned int m = mask_f[w];
+              const int hi = last - w * 32;
+              if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
+              n_forced += (unsigned long long)__popc(m);
+            }
+            n_cand += (unsigned long long)s_bvalid;
+            n_bytes += s_bbytes;
+            ++n_batch;
+            if (kstar >= 0) {
+              const Cand& c = s_slot[s_bslot[kstar]].c;
+              n_trials += (unsigned long long)(kstar + 1);
+              ++n_acc;
+              n_waste += (unsigned long long)(Kb - kstar - 1);
+              S += (double)s_dS[kstar];
+              if (c.layer == 0 && c.gcnt > 0)
+                n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
+            } else if (kstar == -1) {
+              n_trials += (unsigned long long)Kb;
+            }
           }
         }
       }
-    }
-    __syncthreads();
-    if (!s_flag) break;
-    const int kstar = s_kstar;
-    const unsigned long long t_c = stats_thread ? globaltimer_ns() : 0ull;
-    // CTA 0 clears the buffer of batch bidx + 2, which is also that of batch bidx - 1: every CTA
-    // has added its share of batch bidx, so every CTA has finished waiting on batch bidx - 1. Only
-    // the words of the first 64 candidates are used. Warp 1 fences the clearing before the
-    // __syncthreads that precedes CTA 0's additions to batch bidx + 1, for which every CTA waits
-    // before it adds to batch bidx + 2.
-    if (r == 0 && warp == 1) {
-      unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
-      z[lane] = 0ull;
-      z[lane + 32] = 0ull;
-      z[kKmax + lane] = 0ull;
-      z[kKmax + lane + 32] = 0ull;
-    }
-    const unsigned long long t_d = t_c;
-    if (kstar == -2) {
-      if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
-      break;
-    }
-    if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
+      cons_sync();
+      if (!s_flag) break;
+      const int kstar = s_kstar;
+      const unsigned long long t_c = timer ? globaltimer_ns() : 0ull;
+      // CTA 0 clears the buffer of batch bidx + 2, which is also that of batch bidx - 1: every
+      // CTA has added its share of batch bidx, so every CTA has finished waiting on batch
+      // bidx - 1. Only the words of the first 64 candidates are used. Warp 1 fences the clearing
+      // before the barrier that precedes CTA 0's additions to batch bidx + 1, for which every CTA
+      // waits before it adds to batch bidx + 2.
+      if (r == 0 && warp == 1) {
+        unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
+        z[lane] = 0ull;
+        z[lane + 32] = 0ull;
+      }
+      if (kstar == -2) {
+        if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
+        break;
+      }
+      if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
 
-    // ---- commit to this CTA's samples, then drop or patch the prepared slots it invalidates
-    if (kstar >= 0) {
-      const int sl = s_bslot[kstar];
-      const Cand c = s_slot[sl].c;
-      if (c.gcnt > 0) {
-        if (s_slot[sl].state == 1) {
-          float w[M];
-          load_w2c<NC>(s_w2c[sl], a.C, w);
-          float* zrow = a.z1 + (size_t)c.row * a.Np + s0;
-          const unsigned short* nl = e_nl + (size_t)sl * kCap;
-          const float* da = e_da + (size_t)sl * kCap;
-          const float* zn = e_zn + (size_t)sl * kCap;
-          for (int e = tid; e < c.ecnt; e += kLoopThreads) {
-            zrow[nl[e]] = zn[e];
-            (void)entry_cached<ACT2, LOSS, NC, true>(a, R, w, nl[e], da[e]);
+      // ---- commit to this CTA's samples; log it for the slots prepared before it
+      if (kstar >= 0) {
+        const int sl = s_bslot[kstar];
+        const Cand c = s_slot[sl].c;
+        if (c.gcnt > 0) {
+          if (s_slot[sl].state == 1) {
+            float w[M];
+            load_w2c<NC>(s_w2c[sl], a.C, w);
+            float* zrow = a.z1 + (size_t)c.row * a.Np + s0;
+            const unsigned short* nl = e_nl + (size_t)sl * kCap;
+            const float* da = e_da + (size_t)sl * kCap;
+            const float* zn = e_zn + (size_t)sl * kCap;
+            for (int e = tid; e < c.ecnt; e += kConsThreads) {
+              zrow[nl[e]] = zn[e];
+              (void)entry_cached<ACT2, LOSS, NC, true>(a, R, w, nl[e], da[e]);
+            }
+          } else if (c.layer == 0) {
+            float* zrow = a.z1 + (size_t)c.row * a.Np;
+            float w[M];
+            load_w2c<NC>(s_w2c[sl], a.C, w);
+            for (int e = tid; e < c.ecnt; e += kConsThreads) {
+              const int n = __ldg(a.xs_n + c.ebeg + e);
+              const float x = __ldg(a.xs_v + c.ebeg + e);
+              (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
+                                                        zrow + n);
+            }
+          } else {
+            const float* zrow = a.z1 + (size_t)c.col * a.Np;
+            for (int e = tid; e < c.ecnt; e += kConsThreads)
+              (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
           }
-        } else if (c.layer == 0) {
-          float* zrow = a.z1 + (size_t)c.row * a.Np;
-          float w[M];
-          load_w2c<NC>(s_w2c[sl], a.C, w);
-          for (int e = tid; e < c.ecnt; e += kLoopThreads) {
-            const int n = __ldg(a.xs_n + c.ebeg + e);
-            const float x = __ldg(a.xs_v + c.ebeg + e);
-            (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
-                                                      zrow + n);
-          }
-        } else {
-          const float* zrow = a.z1 + (size_t)c.col * a.Np;
-          for (int e = tid; e < c.ecnt; e += kLoopThreads)
-            (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
         }
-      }
-      if (tid == 0) {
-        const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
-        (c.layer ? a.w2 : a.w1)[off] = c.neww;
-        const int wk = c.layer ? a.wk2 : a.wk1;
-        if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
-      }
-      __syncthreads();
-      const unsigned long long t_acc = tau + (unsigned long long)kstar;
-      for (int q = tid; q < kWS; q += kLoopThreads) {
-        WSlot& o = s_slot[q];
-        if (o.state == 0 || o.tau <= t_acc || o.tau == ~0ull) continue;
-        const Cand& oc = o.c;
-        if (oc.idx == c.idx) {
-          o.state = 0;                                   // its old value changed
-        } else if (c.layer == 0 && c.gcnt > 0 && oc.layer == 0 && oc.row == c.row) {
-          o.state = 0;                                   // its hidden-field row changed
-        } else if (c.layer == 1 && oc.layer == 0 && oc.row == c.col) {
-          s_w2c[q][c.row] = c.neww;                      // its W2 column changed
+        if (tid == 0) {
+          const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
+          (c.layer ? a.w2 : a.w1)[off] = c.neww;
+          const int wk = c.layer ? a.wk2 : a.wk1;
+          if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
+          CommitLog& L = s_log[epoch % kLogLen];
+          L.idx = c.idx;
+          L.layer = c.layer;
+          L.row = c.row;
+          L.col = c.col;
+          L.neww = c.neww;
+          L.changes_z1 = c.layer == 0 && c.gcnt > 0;
         }
+        cons_sync();
+        // every consumer's writes of this commit precede the new epoch that producers read
+        ++epoch;
+        if (tid == 0) st_release_cta_shared_s32(&s_epoch, epoch);
+        tau += (unsigned long long)(kstar + 1);
+        rate_a = rate_a * kRateDecay + 1.0f;
+        rate_t = rate_t * kRateDecay + (float)(kstar + 1);
+      } else {
+        tau += (unsigned long long)Kb;
+        rate_a = rate_a * kRateDecay;
+        rate_t = rate_t * kRateDecay + (float)Kb;
       }
-      __syncthreads();
-      tau += (unsigned long long)(kstar + 1);
-      rate_a = rate_a * kRateDecay + 1.0f;
-      rate_t = rate_t * kRateDecay + (float)(kstar + 1);
-    } else {
-      tau += (unsigned long long)Kb;
-      rate_a = rate_a * kRateDecay;
-      rate_t = rate_t * kRateDecay + (float)Kb;
+      if (timer) {
+        const unsigned long long t_e = globaltimer_ns();
+        ph0 += t_s - t_a;
+        ph1 += t_v - t_s;
+        ph4 += t_b - t_v;
+        ph3 += t_c - t_b;
+        ph5 += t_e - t_c;
+      }
+      ++bidx;
+    }
+    if (tid == 0) *(volatile int*)&s_done = 1;
+    if (timer) {
+      const unsigned long long g = (unsigned long long)gridDim.x;
+      atomicAdd(&st->phase_ns[0], ph0 / g);
+      atomicAdd(&st->phase_ns[1], ph1 / g);
+      atomicAdd(&st->phase_ns[2], ph2 / g);
+      atomicAdd(&st->phase_ns[3], ph3 / g);
+      atomicAdd(&st->phase_ns[4], ph4 / g);
+      atomicAdd(&st->phase_ns[5], ph5 / g);
+    }
+    if (lane == 0 && (n_starve | n_reprep)) {
+      atomicAdd(&st->phase_ns[6], n_starve / (unsigned long long)gridDim.x);
+      atomicAdd(&st->phase_ns[7], n_reprep);
     }
     if (stats_thread) {
-      const unsigned long long t_e = globaltimer_ns();
-      ph0 += t_s - t_a;
-      ph1 += t_b - t_s;
-      ph3 += t_c - t_b;
-      ph4 += t_d - t_c;
-      ph5 += t_e - t_d;
+      st->S = S;
+      st->trials += n_trials;
+      st->accepts += n_acc;
+      st->candidates += n_cand;
+      st->batches += n_batch;
+      st->wasted += n_waste;
+      st->forced += n_forced;
+      st->alg_bytes += n_bytes;
+      st->trace_written = n_trace;
+      st->rate_acc = rate_a;
+      st->rate_trials = rate_t;
     }
-    ++bidx;
   }
 
   __syncthreads();
@@ -1133,26 +1288,6 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       const int f = t / ns, nl = t - f * ns;
       a.srec[(size_t)f * a.Np + s0 + nl] = s_records[f * a.RS + nl];
     }
-  }
-  if (tid == 0) atomicAdd(&st->phase_ns[6], my_wait / (unsigned long long)gridDim.x);
-  if (stats_thread) {
-    st->S = S;
-    st->trials += n_trials;
-    st->accepts += n_acc;
-    st->candidates += n_cand;
-    st->batches += n_batch;
-    st->wasted += n_waste;
-    st->forced += n_forced;
-    st->alg_bytes += n_bytes;
-    st->trace_written = n_trace;
-    st->phase_ns[0] += ph0;
-    st->phase_ns[1] += ph1;
-    st->phase_ns[2] += ph2;
-    st->phase_ns[3] += ph3;
-    st->phase_ns[4] += ph4;
-    st->phase_ns[5] += ph5;
-    st->rate_acc = rate_a;
-    st->rate_trials = rate_t;
   }
 }
 
