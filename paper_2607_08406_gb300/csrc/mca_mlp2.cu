@@ -686,6 +686,48 @@ __device__ __forceinline__ float entry_cached(const Mlp2Args& a, Recs R,
   return ln - ell;
 }
 
+// l' - l of one cached entry without branches (0 exactly when da == 0), so that a lane can keep
+// several entries in flight.
+template <int ACT2, int LOSS, int NC>
+__device__ __forceinline__ float cached_delta(const Mlp2Args& a, Recs R,
+                                              const float (&w)[NC > 0 ? NC : kMaxC], int nl,
+                                              float da) {
+  constexpr int M = NC > 0 ? NC : kMaxC;
+  const int C = NC > 0 ? NC : a.C;
+  float zz[M];
+  float ell;
+  int y;
+  load_srec(R.rec, R.pitch, nl, zz, ell, y);
+#pragma unroll
+  for (int k = 0; k < M; ++k)
+    if (k < C) zz[k] = fmaf(w[k], da, zz[k]);
+  const float ln = sample_loss<ACT2, LOSS, M>(zz, C, y, a.g2, a.act2, a.loss);
+  return da == 0.0f ? 0.0f : ln - ell;
+}
+
+// Warp-level sum of l' - l over the cached entries [e_lo, e_hi) of a slot. Lane l takes entries
+// l, l + 32, ... in ascending order, three at a time.
+template <int ACT2, int LOSS, int NC>
+__device__ __forceinline__ float eval_cached(const Mlp2Args& a, Recs R,
+                                             const float (&w)[NC > 0 ? NC : kMaxC],
+                                             const unsigned short* nl, const float* da, int e_lo,
+                                             int e_hi) {
+  const int lane = threadIdx.x & 31;
+  float acc = 0.0f;
+  for (int g = e_lo; g < e_hi; g += 96) {
+    float v[3];
+#pragma unroll
+    for (int u = 0; u < 3; ++u) {
+      const int e = g + u * 32 + lane;
+      const bool in = e < e_hi;
+      v[u] = cached_delta<ACT2, LOSS, NC>(a, R, w, in ? (int)nl[e] : 0, in ? da[e] : 0.0f);
+    }
+#pragma unroll
+    for (int u = 0; u < 3; ++u) acc += v[u];
+  }
+  return warp_sum(acc);
+}
+
 // Warp prepares slot sl for trial t: proposal, W2 column, and (cacheable first-layer candidates)
 // the gathered entries; then publishes it. `epoch` was read before any of the data.
 template <int ACT1>
@@ -978,18 +1020,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
           if (s_slot[sl].state == 1) {
             float w[M];
             load_w2c<NC>(s_w2c[sl], a.C, w);
-            const unsigned short* nl = e_nl + (size_t)sl * kCap;
-            const float* da = e_da + (size_t)sl * kCap;
             const int e_lo = q * a.SUB, e_hi = min(e_lo + a.SUB, c.ecnt);
-            float acc = 0.0f;
-            for (int g = e_lo; g < e_hi; g += 128) {
-#pragma unroll
-              for (int u = 0; u < 4; ++u) {
-                const int e = g + u * 32 + lane;
-                if (e < e_hi) acc += entry_cached<ACT2, LOSS, NC, false>(a, R, w, nl[e], da[e]);
-              }
-            }
-            v = warp_sum(acc);
+            v = eval_cached<ACT2, LOSS, NC>(a, R, w, e_nl + (size_t)sl * kCap,
+                                            e_da + (size_t)sl * kCap, e_lo, e_hi);
           } else {
             v = eval_sub<ACT1, ACT2, LOSS, NC>(a, R, s0, c, s_w2c[sl], q);
           }
