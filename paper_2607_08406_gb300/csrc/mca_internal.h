@@ -37,6 +37,7 @@ constexpr int kWinBatch = 64;
 // buffers rotate. One warp reads a batch's words, two per lane; the count fields cap the ranges at
 // 255.
 constexpr int kAccStride = 2 * kKmax + 32;
+constexpr int kArrivalWord = 64;   // count-only word of a batch without a live candidate
 constexpr int kWindowMaxRanges = 255;
 static_assert(kWinBatch <= 64 && kWinBatch < kWS, "a windowed batch is read by one warp, two per lane");
 

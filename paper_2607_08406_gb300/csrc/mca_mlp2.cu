@@ -833,6 +833,78 @@ __device__ __forceinline__ bool revalidate(WSlot& s, float* w2c, const CommitLog
   return true;
 }
 
+// One lane brings a ready slot from epoch E - 1 to E with log entry L (commit E - 1). Returns false
+// when the slot must be prepared again.
+__device__ __forceinline__ bool replay_one(WSlot& o, float* w2c, const CommitLog& L, int E) {
+  const Cand& c = o.c;
+  if (L.idx == c.idx || (c.layer == 0 && L.layer == 0 && L.changes_z1 && L.row == c.row))
+    return false;
+  if (c.layer == 0 && L.layer == 1 && L.col == c.row) w2c[L.row] = L.neww;
+  o.epoch = E;
+  return true;
+}
+
+// Warp 0: the batch's slots, its sub-chunks (prefix over batch positions, lane k and k + 32) and,
+// in CTA 0, the batch statistics.
+__device__ __forceinline__ void batch_scan(const WSlot* slots, unsigned long long tau, int Kb,
+                                           unsigned int sl_tau, unsigned long long tau_hi, int r,
+                                           int* bslot, int* sub0, int* nsub, unsigned char* map,
+                                           int* total, unsigned long long* bbytes, int* bvalid,
+                                           int* nlive) {
+  const int lane = threadIdx.x & 31;
+  int v[2] = {0, 0}, valid = 0, live = 0;
+  unsigned long long bytes = 0ull;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int k = lane + 32 * h;
+    if (k < Kb) {
+      const int sl = (int)((sl_tau + (unsigned int)k) % (unsigned int)kWS);
+      bslot[k] = sl;
+      const Cand& c = slots[sl].c;
+      v[h] = c.nsub;
+      if (tau + (unsigned long long)k >= tau_hi) bytes += c.bytes;
+      valid += c.valid;
+      live += (c.valid && c.gcnt > 0) ? 1 : 0;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) live += __shfl_xor_sync(0xffffffffu, live, o);
+  if (lane == 0) *nlive = live;
+  int inc[2] = {v[0], v[1]};
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int y = __shfl_up_sync(0xffffffffu, inc[h], o);
+      if (lane >= o) inc[h] += y;
+    }
+  }
+  const int tot0 = __shfl_sync(0xffffffffu, inc[0], 31);
+  const int tot1 = __shfl_sync(0xffffffffu, inc[1], 31);
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int k = lane + 32 * h;
+    if (k < Kb) {
+      const int ex = (h ? tot0 : 0) + inc[h] - v[h];
+      sub0[k] = ex;
+      nsub[k] = v[h];
+      for (int q = 0; q < v[h]; ++q) map[ex + q] = (unsigned char)k;
+    }
+  }
+  if (r == 0) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
+      valid += __shfl_xor_sync(0xffffffffu, valid, o);
+    }
+    if (lane == 0) {
+      *bbytes = bytes;
+      *bvalid = valid;
+    }
+  }
+  if (lane == 0) *total = tot0 + tot1;
+}
+
 template <int ACT1, int ACT2, int LOSS, int NC>
 __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) {
   extern __shared__ __align__(16) float s_dyn[];
@@ -843,7 +915,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   __shared__ int s_bslot[kKmax];       // batch position -> slot
   __shared__ int s_sub0[kKmax], s_nsub[kKmax];
   __shared__ float s_dS[kKmax];
-  __shared__ int s_flag, s_kstar, s_total, s_bvalid, s_fail, s_done, s_epoch;
+  __shared__ unsigned char s_map[kKmax * kMaxSubs];   // sub-chunk -> batch position
+  __shared__ unsigned int s_stale[2];
+  __shared__ int s_flag, s_kstar, s_total, s_bvalid, s_nlive, s_fail, s_done, s_epoch;
   __shared__ unsigned long long s_bbytes, s_tau_hi, s_next, s_cons_tau;
   float* s_records = s_dyn;
   unsigned short* e_nl = reinterpret_cast<unsigned short*>(s_dyn + kRecFields * a.RS);
@@ -907,13 +981,14 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, (int)(t % kWS), t, epoch, r, s0, s1);
     }
   } else {
-    // ---- consumers: the batches
+    // ---- consumers: the batches. The commit of batch b runs at the start of batch b + 1 on warps
+    // 1.., overlapped with that batch's set-up on warp 0, which reads neither records nor z1.
     const bool stats_thread = r == 0 && tid == 0;
     const bool timer = kPhaseTimers && tid == 0;   // phase times of every CTA, mean over CTAs
     double S = 0.0;
     unsigned long long n_trials = 0, n_acc = 0, n_cand = 0, n_batch = 0, n_waste = 0, n_forced = 0,
                        n_bytes = 0, n_trace = 0, ph0 = 0, ph1 = 0, ph2 = 0, ph3 = 0, ph4 = 0,
-                       ph5 = 0, n_starve = 0, n_reprep = 0;
+                       n_starve = 0, n_reprep = 0;
     if (stats_thread) {
       S = st->S;
       n_trace = st->trace_written;
@@ -922,97 +997,171 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
     unsigned int bidx = 0;
     int epoch = 0;                     // commits of this CTA so far (consumer copy of s_epoch)
     const int kmaxw = min(a.K, kWinBatch);
+    unsigned int sl_tau = (unsigned int)(tau % kWS);   // slot of trial tau
+    int pend = -1;                     // slot of the accepted candidate not yet committed
 
-    while (tau < end) {
+    for (;;) {
       const unsigned long long t_a = timer ? globaltimer_ns() : 0ull;
-      if (tid == 0) *(volatile unsigned long long*)&s_cons_tau = tau;
-      const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
-      const int Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
-      // ---- slots of this batch: wait for the producers (bounded), replay the commits since
-      // their preparation, prepare again what they invalidate
-      for (int k = warp; k < Kb; k += kConsWarps) {
-        const unsigned long long t = tau + (unsigned long long)k;
-        const int sl = (int)(t % kWS);
-        int ok = 1;
+      const bool more = tau < end;
+      int Kb = 0;
+      if (more) {
+        const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
+        Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
+      }
+      const int E = epoch + (pend >= 0 ? 1 : 0);    // commits including the pending one
+      if (warp == 0) {
+        // ---- set-up: log the pending commit; the batch's slots ready (bounded wait for the
+        // producers) and replayed up to E, lane k (and k + 32) for batch position k
         if (lane == 0) {
+          if (pend >= 0) {
+            const Cand& pc = s_slot[pend].c;
+            CommitLog& L = s_log[epoch % kLogLen];
+            L.idx = pc.idx;
+            L.layer = pc.layer;
+            L.row = pc.row;
+            L.col = pc.col;
+            L.neww = pc.neww;
+            L.changes_z1 = pc.layer == 0 && pc.gcnt > 0;
+          }
+          // producers may fill slots up to kWS trials past the oldest slot still in use
+          *(volatile unsigned long long*)&s_cons_tau = pend >= 0 ? tau - 1ull : tau;
+        }
+        __syncwarp();
+        bool full[2] = {false, false}, stale[2] = {false, false};
+        int sl[2] = {0, 0};
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int k = lane + 32 * h;
+          if (k >= Kb) continue;
+          const unsigned long long t = tau + (unsigned long long)k;
+          sl[h] = (int)((sl_tau + (unsigned int)k) % (unsigned int)kWS);
           if (!slot_ready(s_slot, t)) {
             const unsigned long long w0 = globaltimer_ns();
             unsigned int spins = 0;
+            bool ok = true;
             while (!slot_ready(s_slot, t)) {
               if ((++spins & 63u) == 0u && globaltimer_ns() - w0 > kBarrierTimeoutNs) {
                 atomicCAS(&st->err, 0, (int)MCA_ERR_TIMEOUT);
                 *(volatile int*)&s_fail = 1;
-                ok = 0;
+                ok = false;
                 break;
               }
             }
             if (kPhaseTimers) n_starve += globaltimer_ns() - w0;
+            if (!ok) continue;
+          }
+          WSlot& o = s_slot[sl[h]];
+          if (o.epoch == E - 1)          // the one commit since its last check
+            stale[h] = !replay_one(o, s_w2c[sl[h]], s_log[(E - 1) % kLogLen], E);
+          else if (o.epoch != E)
+            full[h] = true;
+        }
+        // older commits to replay (slots published after the last look): warp-wide, rare
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          unsigned int m = __ballot_sync(0xffffffffu, full[h]);
+          while (m) {
+            const int j = __ffs(m) - 1;
+            m &= m - 1u;
+            const int slj = __shfl_sync(0xffffffffu, sl[h], j);
+            const bool okj = revalidate(s_slot[slj], s_w2c[slj], s_log, E);
+            if (lane == j) stale[h] = !okj;
           }
         }
-        __syncwarp();
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (ok == 1 && !revalidate(s_slot[sl], s_w2c[sl], s_log, epoch)) {
-          ok = 2;
-          if (lane == 0) ++n_reprep;
-        }
-        if (ok == 2)
-          prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn, sl, t, epoch, r, s0, s1);
-      }
-      cons_sync();
-      if (*(volatile int*)&s_fail) break;
-      if (warp == 0) {                 // sub-chunk scan and batch statistics
-        int v[4], loc = 0;
-        unsigned long long bytes = 0ull;
-        int valid = 0;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int k = lane * 4 + u;
-          v[u] = 0;
-          if (k < Kb) {
-            const int sl = (int)((tau + (unsigned long long)k) % kWS);
-            s_bslot[k] = sl;
-            const Cand& c = s_slot[sl].c;
-            v[u] = c.nsub;
-            if (tau + (unsigned long long)k >= s_tau_hi) bytes += c.bytes;
-            valid += c.valid;
-          }
-          loc += v[u];
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
-          valid += __shfl_xor_sync(0xffffffffu, valid, o);
-        }
-        int inc = loc;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, inc, o);
-          if (lane >= o) inc += y;
-        }
-        int ex = inc - loc;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int k = lane * 4 + u;
-          if (k < Kb) {
-            s_sub0[k] = ex;
-            s_nsub[k] = v[u];
-          }
-          ex += v[u];
-        }
-        if (lane == 31) s_total = inc;
+        const unsigned int ms0 = __ballot_sync(0xffffffffu, stale[0]);
+        const unsigned int ms1 = __ballot_sync(0xffffffffu, stale[1]);
         if (lane == 0) {
-          s_bbytes = bytes;
-          s_bvalid = valid;
+          s_stale[0] = ms0;
+          s_stale[1] = ms1;
+        }
+        if ((ms0 | ms1) == 0u) batch_scan(s_slot, tau, Kb, sl_tau, s_tau_hi, r, s_bslot, s_sub0, s_nsub,
+                                          s_map, &s_total, &s_bbytes, &s_bvalid, &s_nlive);
+      } else if (pend >= 0) {
+        // ---- commit of the pending candidate to this CTA's samples (threads 32..)
+        const int sl = pend;
+        const Cand c = s_slot[sl].c;
+        const int i0 = tid - 32, istride = kConsThreads - 32;
+        if (c.gcnt > 0) {
+          if (s_slot[sl].state == 1) {
+            float w[M];
+            load_w2c<NC>(s_w2c[sl], a.C, w);
+            float* zrow = a.z1 + (size_t)c.row * a.Np + s0;
+            const unsigned short* nl = e_nl + (size_t)sl * kCap;
+            const float* da = e_da + (size_t)sl * kCap;
+            const float* zn = e_zn + (size_t)sl * kCap;
+            for (int e = i0; e < c.ecnt; e += istride) {
+              zrow[nl[e]] = zn[e];
+              (void)entry_cached<ACT2, LOSS, NC, true>(a, R, w, nl[e], da[e]);
+            }
+          } else if (c.layer == 0) {
+            float* zrow = a.z1 + (size_t)c.row * a.Np;
+            float w[M];
+            load_w2c<NC>(s_w2c[sl], a.C, w);
+            for (int e = i0; e < c.ecnt; e += istride) {
+              const int n = __ldg(a.xs_n + c.ebeg + e);
+              const float x = __ldg(a.xs_v + c.ebeg + e);
+              (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
+                                                        zrow + n);
+            }
+          } else {
+            const float* zrow = a.z1 + (size_t)c.col * a.Np;
+            for (int e = i0; e < c.ecnt; e += istride)
+              (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
+          }
+        }
+        if (tid == 32) {
+          const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
+          (c.layer ? a.w2 : a.w1)[off] = c.neww;
+          const int wk = c.layer ? a.wk2 : a.wk1;
+          if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
         }
       }
+      // CTA 0 clears the buffer of batch bidx + 1, which is also that of batch bidx - 2: every CTA
+      // has added its share of batch bidx - 1, so every CTA has finished waiting on batch
+      // bidx - 2. Warp 1 fences the clearing before the barrier that precedes CTA 0's additions
+      // to batch bidx, for which every CTA waits before it adds to batch bidx + 1.
+      if (r == 0 && warp == 1) {
+        unsigned long long* z = a.accum + (size_t)((bidx + 1) % 3) * kAccStride;
+        z[lane] = 0ull;
+        z[lane + 32] = 0ull;
+        if (lane == 0) z[kArrivalWord] = 0ull;
+      }
       cons_sync();
+      if (pend >= 0) {
+        // every consumer's writes of the commit precede the new epoch that producers read
+        ++epoch;
+        if (tid == 0) st_release_cta_shared_s32(&s_epoch, epoch);
+        pend = -1;
+      }
+      if (*(volatile int*)&s_fail || !more) break;
+      if ((s_stale[0] | s_stale[1]) != 0u) {
+        // slots a commit invalidated, prepared again now that the commit is complete (rare)
+        if (warp == 0) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            unsigned int m = s_stale[h];
+            while (m) {
+              const int j = __ffs(m) - 1;
+              m &= m - 1u;
+              const int k = j + 32 * h;
+              const unsigned long long t = tau + (unsigned long long)k;
+              prepare_slot<ACT1>(a, s_slot, s_w2c, e_nl, e_da, e_zn,
+                                 (int)((sl_tau + (unsigned int)k) % (unsigned int)kWS), t, epoch,
+                                 r, s0, s1);
+              if (lane == 0) ++n_reprep;
+            }
+          }
+          batch_scan(s_slot, tau, Kb, sl_tau, s_tau_hi, r, s_bslot, s_sub0, s_nsub, s_map,
+                     &s_total, &s_bbytes, &s_bvalid, &s_nlive);
+        }
+        cons_sync();
+      }
       const unsigned long long t_s = timer ? globaltimer_ns() : 0ull;
       // ---- evaluate: warp per sub-chunk; cached slots from shared memory, the rest from global
       {
         const int total = s_total;
-        int k = 0;
         for (int it = warp; it < total; it += kConsWarps) {
-          while (s_sub0[k] + s_nsub[k] <= it) ++k;
+          const int k = s_map[it];
           const int sl = s_bslot[k];
           const Cand& c = s_slot[sl].c;
           const int q = it - s_sub0[k];
@@ -1030,7 +1179,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         }
       }
       const unsigned long long t_v = timer ? globaltimer_ns() : 0ull;
-      if (r == 0 && warp == 1) __threadfence();    // the clearing of the previous batch (below)
+      if (r == 0 && warp == 1) __threadfence();    // the clearing above
       cons_sync();
       // this range's loss change of every candidate, added into the candidate's packed 64-bit
       // word: bits 56..63 count the CTAs that have added, bits 48..55 those whose share was not
@@ -1051,6 +1200,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
           w += 1ull << 48;
         atomicAdd(acc + k, w);
       }
+      // a batch without a live candidate still synchronises (on the arrival word), so that no
+      // CTA runs more than one batch ahead of the clearing of the rotating buffers
+      if (tid == 0 && s_nlive == 0) atomicAdd(acc + kArrivalWord, 1ull << 56);
       const unsigned long long t_b = timer ? globaltimer_ns() : 0ull;
       // ---- warp 0 waits until every CTA has added to every live candidate (bounded), then
       // decides
@@ -1058,7 +1210,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         const unsigned long long need = (unsigned long long)gridDim.x;
         int ok = 1;
         unsigned long long v[2] = {0ull, 0ull};
-        bool live[2];
+        bool live[2], poll[2];
+        const unsigned long long* pa[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int k = lane + 32 * h;
@@ -1067,6 +1220,12 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
             const Cand& c = s_slot[s_bslot[k]].c;
             live[h] = c.valid && c.gcnt > 0;
           }
+          poll[h] = live[h];
+          pa[h] = acc + k;
+        }
+        if (s_nlive == 0 && lane == 0) {
+          poll[0] = true;
+          pa[0] = acc + kArrivalWord;
         }
         // the clock is read only once the wait has lasted 64 polls (and for the phase timers)
         unsigned long long w0 = kPhaseTimers ? globaltimer_ns() : 0ull;
@@ -1075,8 +1234,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
           bool mine = true;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
-            if (live[h] && (v[h] >> 56) < need) {
-              v[h] = ld_acquire_gpu_u64(acc + lane + 32 * h);
+            if (poll[h] && (v[h] >> 56) < need) {
+              v[h] = ld_acquire_gpu_u64(pa[h]);
               mine = mine && (v[h] >> 56) >= need;
             }
           }
@@ -1197,92 +1356,59 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
             }
           }
         }
+      } else if (warp <= 3) {
+        // warps 1..3 bring the published slots past the batch up to date meanwhile, one slot per
+        // lane (a few commits behind: replayed by the lane; further: warp-wide)
+        const int j = Kb + lane + 32 * (warp - 1);
+        const unsigned long long t = tau + (unsigned long long)j;
+        bool full = false;
+        int slj = 0;
+        if (j < kWS && t < end) {
+          slj = (int)((sl_tau + (unsigned int)j) % (unsigned int)kWS);
+          if (slot_ready(s_slot, t)) {
+            WSlot& o = s_slot[slj];
+            const int lag = epoch - o.epoch;
+            if (lag > 4) {
+              full = true;
+            } else {
+              for (int e = o.epoch; e < epoch; ++e)
+                if (!replay_one(o, s_w2c[slj], s_log[e % kLogLen], e + 1)) break;
+            }
+          }
+        }
+        unsigned int m = __ballot_sync(0xffffffffu, full);
+        while (m) {
+          const int jj = __ffs(m) - 1;
+          m &= m - 1u;
+          const int sj = __shfl_sync(0xffffffffu, slj, jj);
+          (void)revalidate(s_slot[sj], s_w2c[sj], s_log, epoch);
+        }
       }
       cons_sync();
       if (!s_flag) break;
       const int kstar = s_kstar;
-      const unsigned long long t_c = timer ? globaltimer_ns() : 0ull;
-      // CTA 0 clears the buffer of batch bidx + 2, which is also that of batch bidx - 1: every
-      // CTA has added its share of batch bidx, so every CTA has finished waiting on batch
-      // bidx - 1. Only the words of the first 64 candidates are used. Warp 1 fences the clearing
-      // before the barrier that precedes CTA 0's additions to batch bidx + 1, for which every CTA
-      // waits before it adds to batch bidx + 2.
-      if (r == 0 && warp == 1) {
-        unsigned long long* z = a.accum + (size_t)((bidx + 2) % 3) * kAccStride;
-        z[lane] = 0ull;
-        z[lane + 32] = 0ull;
+      if (timer) {
+        const unsigned long long t_c = globaltimer_ns();
+        ph0 += t_s - t_a;
+        ph1 += t_v - t_s;
+        ph4 += t_b - t_v;
+        ph3 += t_c - t_b;
       }
       if (kstar == -2) {
         if (stats_thread) atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
         break;
       }
       if (tid == 0) s_tau_hi = max(s_tau_hi, tau + (unsigned long long)Kb);
-
-      // ---- commit to this CTA's samples; log it for the slots prepared before it
+      const int adv = kstar >= 0 ? kstar + 1 : Kb;
       if (kstar >= 0) {
-        const int sl = s_bslot[kstar];
-        const Cand c = s_slot[sl].c;
-        if (c.gcnt > 0) {
-          if (s_slot[sl].state == 1) {
-            float w[M];
-            load_w2c<NC>(s_w2c[sl], a.C, w);
-            float* zrow = a.z1 + (size_t)c.row * a.Np + s0;
-            const unsigned short* nl = e_nl + (size_t)sl * kCap;
-            const float* da = e_da + (size_t)sl * kCap;
-            const float* zn = e_zn + (size_t)sl * kCap;
-            for (int e = tid; e < c.ecnt; e += kConsThreads) {
-              zrow[nl[e]] = zn[e];
-              (void)entry_cached<ACT2, LOSS, NC, true>(a, R, w, nl[e], da[e]);
-            }
-          } else if (c.layer == 0) {
-            float* zrow = a.z1 + (size_t)c.row * a.Np;
-            float w[M];
-            load_w2c<NC>(s_w2c[sl], a.C, w);
-            for (int e = tid; e < c.ecnt; e += kConsThreads) {
-              const int n = __ldg(a.xs_n + c.ebeg + e);
-              const float x = __ldg(a.xs_v + c.ebeg + e);
-              (void)entry_l1<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, w, n - s0, x, zrow[n],
-                                                        zrow + n);
-            }
-          } else {
-            const float* zrow = a.z1 + (size_t)c.col * a.Np;
-            for (int e = tid; e < c.ecnt; e += kConsThreads)
-              (void)entry_l2<ACT1, ACT2, LOSS, NC, true>(a, R, c.delta, c.row, e, zrow[s0 + e]);
-          }
-        }
-        if (tid == 0) {
-          const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
-          (c.layer ? a.w2 : a.w1)[off] = c.neww;
-          const int wk = c.layer ? a.wk2 : a.wk1;
-          if (wk != MCA_W_FP32) (c.layer ? a.code2 : a.code1)[off] = (signed char)c.new_code;
-          CommitLog& L = s_log[epoch % kLogLen];
-          L.idx = c.idx;
-          L.layer = c.layer;
-          L.row = c.row;
-          L.col = c.col;
-          L.neww = c.neww;
-          L.changes_z1 = c.layer == 0 && c.gcnt > 0;
-        }
-        cons_sync();
-        // every consumer's writes of this commit precede the new epoch that producers read
-        ++epoch;
-        if (tid == 0) st_release_cta_shared_s32(&s_epoch, epoch);
-        tau += (unsigned long long)(kstar + 1);
+        pend = s_bslot[kstar];
         rate_a = rate_a * kRateDecay + 1.0f;
-        rate_t = rate_t * kRateDecay + (float)(kstar + 1);
       } else {
-        tau += (unsigned long long)Kb;
         rate_a = rate_a * kRateDecay;
-        rate_t = rate_t * kRateDecay + (float)Kb;
       }
-      if (timer) {
-        const unsigned long long t_e = globaltimer_ns();
-        ph0 += t_s - t_a;
-        ph1 += t_v - t_s;
-        ph4 += t_b - t_v;
-        ph3 += t_c - t_b;
-        ph5 += t_e - t_c;
-      }
+      rate_t = rate_t * kRateDecay + (float)adv;
+      tau += (unsigned long long)adv;
+      sl_tau = (sl_tau + (unsigned int)adv) % (unsigned int)kWS;
       ++bidx;
     }
     if (tid == 0) *(volatile int*)&s_done = 1;
@@ -1293,7 +1419,6 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       atomicAdd(&st->phase_ns[2], ph2 / g);
       atomicAdd(&st->phase_ns[3], ph3 / g);
       atomicAdd(&st->phase_ns[4], ph4 / g);
-      atomicAdd(&st->phase_ns[5], ph5 / g);
     }
     if (lane == 0 && (n_starve | n_reprep)) {
       atomicAdd(&st->phase_ns[6], n_starve / (unsigned long long)gridDim.x);

@@ -104,6 +104,23 @@ def test_K_invariance(gpu_lib, Ks):
         h.close()
 
 
+def test_batches_without_live_candidates_stay_in_step(gpu_lib):
+    """Ternary proposals that keep the old code change nothing; with one candidate per batch a third
+    of the batches have nothing to exchange. The CTAs must still advance batch by batch (the
+    per-batch exchange buffers rotate), and the trajectory must equal the adaptive-width one."""
+    wl, _ = _make("ternary")
+    runs = []
+    for kw in (dict(K=1, fixed_K=True), dict(K=64)):
+        h = gpu_lib.create_from_workload(wl, trace_cap=3000, **kw)
+        gpu_lib.mca_run(h, 3000, 5)
+        runs.append((gpu_lib.mca_get_trace(h, 3000), gpu_lib.mca_get_codes(h, wl.n_params)))
+        h.close()
+    assert np.array_equal(runs[0][0], runs[1][0])
+    assert np.array_equal(runs[0][1], runs[1][1])
+    noop = runs[0][0]["old_w"] == runs[0][0]["new_w"]
+    assert noop.sum() > 500
+
+
 @pytest.mark.parametrize("grid", [1, 5, 0])
 def test_grid_choices_match_oracle(gpu_lib, traces, grid):
     """The sample ranges (one CTA each) fix the summation order of dS; every choice of their
