@@ -96,6 +96,12 @@ __host__ __device__ __forceinline__ int batch_width(float acc, float trials, flo
   return w >= (float)K ? K : (w < 1.0f ? 1 : (int)w);
 }
 
+// The same rule with one approximate division (device only; deterministic, so every CTA agrees).
+__device__ __forceinline__ int batch_width_fast(float acc, float trials, float c, int K) {
+  const float w = ceilf(__fdividef(c * (trials + 1.0f), acc + 0.5f));
+  return w >= (float)K ? K : (w < 1.0f ? 1 : (int)w);
+}
+
 // ------------------------------------------------------------------------------------------------
 // Transfer functions (Section 2) and losses (Eq. 2 with R = 0). ACT < 0 selects at run time.
 //

@@ -844,16 +844,17 @@ __device__ __forceinline__ bool replay_one(WSlot& o, float* w2c, const CommitLog
   return true;
 }
 
-// Warp 0: the batch's slots, its sub-chunks (prefix over batch positions, lane k and k + 32) and,
-// in CTA 0, the batch statistics.
-__device__ __forceinline__ void batch_scan(const WSlot* slots, unsigned long long tau, int Kb,
-                                           unsigned int sl_tau, unsigned long long tau_hi, int r,
+// Warp 0: the batch's slots and its sub-chunks (lane k and k + 32 for batch position k). The
+// prefix over batch positions is taken bit plane by bit plane of the sub-chunk counts (at most
+// kMaxSubs), with ballots, so that it costs a few dependent steps.
+__device__ __forceinline__ void batch_scan(const WSlot* slots, int Kb, unsigned int sl_tau,
                                            int* bslot, int* sub0, int* nsub, unsigned char* map,
-                                           int* total, unsigned long long* bbytes, int* bvalid,
-                                           int* nlive) {
+                                           int* total, int* bvalid, int* nlive) {
+  static_assert(kMaxSubs < 16, "sub-chunk counts fit four bit planes");
   const int lane = threadIdx.x & 31;
-  int v[2] = {0, 0}, valid = 0, live = 0;
-  unsigned long long bytes = 0ull;
+  const unsigned int lt = (1u << lane) - 1u;
+  int v[2] = {0, 0};
+  bool val[2] = {false, false}, liv[2] = {false, false};
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int k = lane + 32 * h;
@@ -862,47 +863,56 @@ __device__ __forceinline__ void batch_scan(const WSlot* slots, unsigned long lon
       bslot[k] = sl;
       const Cand& c = slots[sl].c;
       v[h] = c.nsub;
-      if (tau + (unsigned long long)k >= tau_hi) bytes += c.bytes;
-      valid += c.valid;
-      live += (c.valid && c.gcnt > 0) ? 1 : 0;
+      val[h] = c.valid != 0;
+      liv[h] = c.valid && c.gcnt > 0;
     }
   }
+  int ex[2] = {0, 0}, tot[2] = {0, 0};
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) live += __shfl_xor_sync(0xffffffffu, live, o);
-  if (lane == 0) *nlive = live;
-  int inc[2] = {v[0], v[1]};
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
+  for (int b = 0; b < 4; ++b) {
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const int y = __shfl_up_sync(0xffffffffu, inc[h], o);
-      if (lane >= o) inc[h] += y;
+      const unsigned int m = __ballot_sync(0xffffffffu, (v[h] >> b) & 1);
+      ex[h] += __popc(m & lt) << b;
+      tot[h] += __popc(m) << b;
     }
   }
-  const int tot0 = __shfl_sync(0xffffffffu, inc[0], 31);
-  const int tot1 = __shfl_sync(0xffffffffu, inc[1], 31);
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int k = lane + 32 * h;
     if (k < Kb) {
-      const int ex = (h ? tot0 : 0) + inc[h] - v[h];
-      sub0[k] = ex;
+      const int e = ex[h] + (h ? tot[0] : 0);
+      sub0[k] = e;
       nsub[k] = v[h];
-      for (int q = 0; q < v[h]; ++q) map[ex + q] = (unsigned char)k;
+      for (int q = 0; q < v[h]; ++q) map[e + q] = (unsigned char)k;
     }
   }
-  if (r == 0) {
+  const int nval = __popc(__ballot_sync(0xffffffffu, val[0])) +
+                   __popc(__ballot_sync(0xffffffffu, val[1]));
+  const int nliv = __popc(__ballot_sync(0xffffffffu, liv[0])) +
+                   __popc(__ballot_sync(0xffffffffu, liv[1]));
+  if (lane == 0) {
+    *total = tot[0] + tot[1];
+    *bvalid = nval;
+    *nlive = nliv;
+  }
+}
+
+// Compulsory bytes of the batch's candidates not evaluated before (statistics of CTA 0).
+__device__ __forceinline__ unsigned long long batch_bytes(const WSlot* slots, unsigned long long tau,
+                                                          int Kb, unsigned int sl_tau,
+                                                          unsigned long long tau_hi) {
+  const int lane = threadIdx.x & 31;
+  unsigned long long bytes = 0ull;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
-      valid += __shfl_xor_sync(0xffffffffu, valid, o);
-    }
-    if (lane == 0) {
-      *bbytes = bytes;
-      *bvalid = valid;
-    }
+  for (int h = 0; h < 2; ++h) {
+    const int k = lane + 32 * h;
+    if (k < Kb && tau + (unsigned long long)k >= tau_hi)
+      bytes += slots[(sl_tau + (unsigned int)k) % (unsigned int)kWS].c.bytes;
   }
-  if (lane == 0) *total = tot0 + tot1;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) bytes += __shfl_xor_sync(0xffffffffu, bytes, o);
+  return bytes;
 }
 
 template <int ACT1, int ACT2, int LOSS, int NC>
@@ -917,7 +927,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
   __shared__ float s_dS[kKmax];
   __shared__ unsigned char s_map[kKmax * kMaxSubs];   // sub-chunk -> batch position
   __shared__ unsigned int s_stale[2];
-  __shared__ int s_flag, s_kstar, s_total, s_bvalid, s_nlive, s_fail, s_done, s_epoch;
+  __shared__ int s_flag, s_kstar, s_total, s_bvalid, s_nlive, s_fail, s_done, s_epoch, s_redo;
   __shared__ unsigned long long s_bbytes, s_tau_hi, s_next, s_cons_tau;
   float* s_records = s_dyn;
   unsigned short* e_nl = reinterpret_cast<unsigned short*>(s_dyn + kRecFields * a.RS);
@@ -1005,28 +1015,32 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       const bool more = tau < end;
       int Kb = 0;
       if (more) {
-        const int Kw = a.fixed_K ? kmaxw : batch_width(rate_a, rate_t, kWidthMlp2, kmaxw);
+        const int Kw = a.fixed_K ? kmaxw : batch_width_fast(rate_a, rate_t, kWidthMlp2, kmaxw);
         Kb = (int)((end - tau) < (unsigned long long)Kw ? (end - tau) : Kw);
       }
       const int E = epoch + (pend >= 0 ? 1 : 0);    // commits including the pending one
       if (warp == 0) {
-        // ---- set-up: log the pending commit; the batch's slots ready (bounded wait for the
-        // producers) and replayed up to E, lane k (and k + 32) for batch position k
-        if (lane == 0) {
-          if (pend >= 0) {
-            const Cand& pc = s_slot[pend].c;
-            CommitLog& L = s_log[epoch % kLogLen];
-            L.idx = pc.idx;
-            L.layer = pc.layer;
-            L.row = pc.row;
-            L.col = pc.col;
-            L.neww = pc.neww;
-            L.changes_z1 = pc.layer == 0 && pc.gcnt > 0;
-          }
-          // producers may fill slots up to kWS trials past the oldest slot still in use
-          *(volatile unsigned long long*)&s_cons_tau = pend >= 0 ? tau - 1ull : tau;
+        // ---- set-up: the batch's slots ready (bounded wait for the producers) and brought up to
+        // E, lane k (and k + 32) for batch position k: a slot one commit behind is checked against
+        // the pending candidate itself; the log entry is written afterwards
+        CommitLog P;
+        P.idx = ~0u;
+        P.layer = P.row = P.col = -1;
+        P.neww = 0.0f;
+        P.changes_z1 = 0;
+        if (pend >= 0) {
+          const Cand& pc = s_slot[pend].c;
+          P.idx = pc.idx;
+          P.layer = pc.layer;
+          P.row = pc.row;
+          P.col = pc.col;
+          P.neww = pc.neww;
+          P.changes_z1 = pc.layer == 0 && pc.gcnt > 0;
+        } else if (E > 0) {
+          P = s_log[(E - 1) % kLogLen];      // no commit pending: commit E - 1 is logged
         }
-        __syncwarp();
+        if (lane == 0)     // producers may fill slots up to kWS trials past the oldest in use
+          *(volatile unsigned long long*)&s_cons_tau = pend >= 0 ? tau - 1ull : tau;
         bool full[2] = {false, false}, stale[2] = {false, false};
         int sl[2] = {0, 0};
 #pragma unroll
@@ -1051,21 +1065,28 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
             if (!ok) continue;
           }
           WSlot& o = s_slot[sl[h]];
-          if (o.epoch == E - 1)          // the one commit since its last check
-            stale[h] = !replay_one(o, s_w2c[sl[h]], s_log[(E - 1) % kLogLen], E);
-          else if (o.epoch != E)
+          const int oe = o.epoch;
+          if (oe == E - 1)
+            stale[h] = !replay_one(o, s_w2c[sl[h]], P, E);
+          else if (oe != E)
             full[h] = true;
         }
-        // older commits to replay (slots published after the last look): warp-wide, rare
+        if (pend >= 0 && lane == 0) s_log[epoch % kLogLen] = P;
+        const unsigned int mf0 = __ballot_sync(0xffffffffu, full[0]);
+        const unsigned int mf1 = __ballot_sync(0xffffffffu, full[1]);
+        if (mf0 | mf1) {
+          // older commits to replay (slots published after the last look): warp-wide, rare
+          __syncwarp();
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          unsigned int m = __ballot_sync(0xffffffffu, full[h]);
-          while (m) {
-            const int j = __ffs(m) - 1;
-            m &= m - 1u;
-            const int slj = __shfl_sync(0xffffffffu, sl[h], j);
-            const bool okj = revalidate(s_slot[slj], s_w2c[slj], s_log, E);
-            if (lane == j) stale[h] = !okj;
+          for (int h = 0; h < 2; ++h) {
+            unsigned int m = h ? mf1 : mf0;
+            while (m) {
+              const int j = __ffs(m) - 1;
+              m &= m - 1u;
+              const int slj = __shfl_sync(0xffffffffu, sl[h], j);
+              const bool okj = revalidate(s_slot[slj], s_w2c[slj], s_log, E);
+              if (lane == j) stale[h] = !okj;
+            }
           }
         }
         const unsigned int ms0 = __ballot_sync(0xffffffffu, stale[0]);
@@ -1073,9 +1094,11 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         if (lane == 0) {
           s_stale[0] = ms0;
           s_stale[1] = ms1;
+          s_redo = (ms0 | ms1) != 0u || *(volatile int*)&s_fail != 0;
         }
-        if ((ms0 | ms1) == 0u) batch_scan(s_slot, tau, Kb, sl_tau, s_tau_hi, r, s_bslot, s_sub0, s_nsub,
-                                          s_map, &s_total, &s_bbytes, &s_bvalid, &s_nlive);
+        if ((ms0 | ms1) == 0u)
+          batch_scan(s_slot, Kb, sl_tau, s_bslot, s_sub0, s_nsub, s_map, &s_total, &s_bvalid,
+                     &s_nlive);
       } else if (pend >= 0) {
         // ---- commit of the pending candidate to this CTA's samples (threads 32..)
         const int sl = pend;
@@ -1110,6 +1133,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
           }
         }
         if (tid == 32) {
+          if (r == 0 && c.layer == 0 && c.gcnt > 0)   // hidden-field sectors written back
+            n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
           const unsigned long long off = c.idx - (c.layer ? a.P1 : 0ull);
           (c.layer ? a.w2 : a.w1)[off] = c.neww;
           const int wk = c.layer ? a.wk2 : a.wk1;
@@ -1133,8 +1158,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
         if (tid == 0) st_release_cta_shared_s32(&s_epoch, epoch);
         pend = -1;
       }
-      if (*(volatile int*)&s_fail || !more) break;
-      if ((s_stale[0] | s_stale[1]) != 0u) {
+      if (!more) break;
+      if (s_redo) {
+        if (*(volatile int*)&s_fail) break;
         // slots a commit invalidated, prepared again now that the commit is complete (rare)
         if (warp == 0) {
 #pragma unroll
@@ -1151,8 +1177,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
               if (lane == 0) ++n_reprep;
             }
           }
-          batch_scan(s_slot, tau, Kb, sl_tau, s_tau_hi, r, s_bslot, s_sub0, s_nsub, s_map,
-                     &s_total, &s_bbytes, &s_bvalid, &s_nlive);
+          batch_scan(s_slot, Kb, sl_tau, s_bslot, s_sub0, s_nsub, s_map, &s_total, &s_bvalid,
+                     &s_nlive);
         }
         cons_sync();
       }
@@ -1341,22 +1367,22 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
               n_forced += (unsigned long long)__popc(m);
             }
             n_cand += (unsigned long long)s_bvalid;
-            n_bytes += s_bbytes;
             ++n_batch;
             if (kstar >= 0) {
-              const Cand& c = s_slot[s_bslot[kstar]].c;
               n_trials += (unsigned long long)(kstar + 1);
               ++n_acc;
               n_waste += (unsigned long long)(Kb - kstar - 1);
               S += (double)s_dS[kstar];
-              if (c.layer == 0 && c.gcnt > 0)
-                n_bytes += 32ull * (unsigned long long)a.xs_sect[c.col];
             } else if (kstar == -1) {
               n_trials += (unsigned long long)Kb;
             }
           }
         }
       } else if (warp <= 3) {
+        if (warp == 1 && r == 0) {
+          const unsigned long long bb = batch_bytes(s_slot, tau, Kb, sl_tau, s_tau_hi);
+          if (lane == 0) s_bbytes = bb;
+        }
         // warps 1..3 bring the published slots past the batch up to date meanwhile, one slot per
         // lane (a few commits behind: replayed by the lane; further: warp-wide)
         const int j = Kb + lane + 32 * (warp - 1);
@@ -1387,6 +1413,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       cons_sync();
       if (!s_flag) break;
       const int kstar = s_kstar;
+      if (stats_thread) n_bytes += s_bbytes;
       if (timer) {
         const unsigned long long t_c = globaltimer_ns();
         ph0 += t_s - t_a;
@@ -1424,6 +1451,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       atomicAdd(&st->phase_ns[6], n_starve / (unsigned long long)gridDim.x);
       atomicAdd(&st->phase_ns[7], n_reprep);
     }
+    if (r == 0 && tid == 32 && n_bytes) atomicAdd(&st->alg_bytes, n_bytes);
     if (stats_thread) {
       st->S = S;
       st->trials += n_trials;
@@ -1432,7 +1460,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
       st->batches += n_batch;
       st->wasted += n_waste;
       st->forced += n_forced;
-      st->alg_bytes += n_bytes;
+      atomicAdd(&st->alg_bytes, n_bytes);
       st->trace_written = n_trace;
       st->rate_acc = rate_a;
       st->rate_trials = rate_t;
