@@ -34,8 +34,8 @@ METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roo
 # from the ncu launch list of `python bench.py --steps 3 --warmup 3 --no-e2e --no-cpu` summarised in
 # profiles/. It is only valid for the kernel source it was measured on; any other source hash
 # reports null.
-LOOP_TRAFFIC = {"source_sha1": "af79e07dbfb98008a5f86318c55d2da3ba8d9c92",
-                "bytes_per_trial": 358196.0}
+LOOP_TRAFFIC = {"source_sha1": "c21e8feec564e69e0d2364185e9d6fbaf6417b2c",
+                "bytes_per_trial": 359457.9}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
 
@@ -381,7 +381,8 @@ def run_ours(args):
                        "K": wl.K, "trials_per_step": T,
                        "trial_range": [W_ * T, (W_ + K) * T], "seed": args.seed,
                        "resync_period": args.resync, "resync_ms": resync_ms,
-                       "l2": ("no flush: the cached hidden fields (3.9 GB) exceed L2"
+                       "l2": (f"no flush: the cached hidden fields "
+                              f"({wl.layers[0].n_out * wl.N * 4 / 1e9:.2f} GB) exceed L2"
                               if not deep else "no flush: a step's candidates recompute from "
                               "cached fields / residual streams that exceed L2 or are rewritten"),
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
