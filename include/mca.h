@@ -144,7 +144,9 @@ typedef struct {
                               prepared (summed over warps), [7] (a count) slots prepared again
                               after a commit invalidated them. Other loop, first CTA:
                               [0] proposal + evaluation, [1] grid barrier, [2] reduction +
-                              decision, [3] commit. Rest 0 */
+                              decision, [3] commit. Deep nets and the Transformer (CUDA
+                              events around each batch's launches): [0] candidate evaluation
+                              kernel, [1] decision + commit kernels. Rest 0 */
   uint64_t alg_flops;      /* deep nets: FLOPs of the evaluated candidates' recomputation (2 per
                               multiply-add: the row update, the rank-1 layer, the dense layers) */
 } mca_run_stats;

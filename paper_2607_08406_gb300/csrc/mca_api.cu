@@ -62,11 +62,21 @@ bool is_device_ptr(const void* p) {
 struct Layout {
   size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, accum, bar, st, trace,
       ex_idx, ex_new, ex_out, scratch, ell, ctl, total;
-  std::vector<size_t> w_eff, code, wfix, Z;
+  std::vector<size_t> w_eff, code, wfix, Z, whi, wlo;
 };
 
 bool is_deep(const std::vector<mca_layer>& layers) { return layers.size() > 2; }
 int deep_tiles(long long N) { return (int)((N + mca::kDeepTS - 1) / mca::kDeepTS); }
+
+// The dense chain runs on the tensor cores when every layer between the first and the output layer
+// is 256 x 256 (the kernel's fixed width).
+bool deep_tc_ok(const std::vector<mca_layer>& layers) {
+  if (layers.size() < 3) return false;
+  for (size_t l = 1; l + 1 < layers.size(); ++l)
+    if (layers[l].n_in != 256 || layers[l].n_out != 256) return false;
+  return true;
+}
+int deep_tc_tiles(long long N) { return (int)((N + mca::kTcTS - 1) / mca::kTcTS); }
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
 
@@ -100,6 +110,12 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   }
   if (deep) {
     for (const auto& ly : layers) L.Z.push_back(take(sizeof(float) * (size_t)ly.n_out * Np));
+    if (deep_tc_ok(layers)) {
+      for (size_t l = 1; l + 1 < layers.size(); ++l) {
+        L.whi.push_back(take(sizeof(float) * 256 * 256));
+        L.wlo.push_back(take(sizeof(float) * 256 * 256));
+      }
+    }
     L.ell = take(sizeof(float) * (size_t)Np);
     L.ctl = take(sizeof(mca::DeepCtl));
     L.z1 = L.srec = SIZE_MAX;
@@ -347,7 +363,10 @@ mca::DeepArgs deep_args(mca_handle* h) {
     a.code[l] = h->code[l];
     a.wfix[l] = h->wfix[l];
     a.Z[l] = h->Z[l];
+    a.whi[l] = h->tc && l >= 1 && l + 1 < a.L ? h->whi[l - 1] : nullptr;
+    a.wlo[l] = h->tc && l >= 1 && l + 1 < a.L ? h->wlo[l - 1] : nullptr;
   }
+  a.tc = h->tc ? 1 : 0;
   a.off[a.L] = h->P;
   a.XT = h->XT;
   a.ell = h->ell;
@@ -383,6 +402,10 @@ mca_status resync(mca_handle* h) {
   }
   if (h->deep) {
     const mca::DeepArgs a = deep_args(h);
+    if (a.tc) {
+      CUDA_TRY(h, mca::launch_deep_split(a, h->stream));
+      h->launches += 1;
+    }
     for (int l = 0; l < a.L; ++l) CUDA_TRY(h, mca::launch_deep_forward_layer(a, l, h->stream));
     CUDA_TRY(h, mca::launch_deep_losses(a, h->stream));
     CUDA_TRY(h, mca::launch_sum_loss(h->ell, (int)h->N, h->st, h->stream));
@@ -459,6 +482,10 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
   s->S = d.S;
   s->alg_bytes = d.alg_bytes;
   for (int q = 0; q < 8; ++q) s->phase_ns[q] = d.phase_ns[q];
+  if (h->deep || h->tfm) {           // host-timed kernels of the per-batch loop (CUDA events)
+    s->phase_ns[0] = h->eval_ns;
+    s->phase_ns[1] = h->rest_ns;
+  }
   s->alg_flops = d.alg_flops;
 }
 
@@ -684,7 +711,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   CTRY(cudaGetDevice(&h->device));
   CTRY(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
   h->deep = is_deep(ls);
-  h->ntiles = deep_tiles(h->N);
+  h->tc = h->deep && deep_tc_ok(ls);
+  h->ntiles = h->tc ? deep_tc_tiles(h->N) : deep_tiles(h->N);
   if (!h->deep) {
     long long nnz = 0;
     mca_status s = count_nnz(data, h->stream, &nnz);
@@ -737,6 +765,10 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   }
   if (h->deep) {
     for (size_t l = 0; l < ls.size(); ++l) h->Z.push_back(reinterpret_cast<float*>(base + L.Z[l]));
+    for (size_t q = 0; q < L.whi.size(); ++q) {
+      h->whi.push_back(reinterpret_cast<float*>(base + L.whi[q]));
+      h->wlo.push_back(reinterpret_cast<float*>(base + L.wlo[q]));
+    }
     h->ell = reinterpret_cast<float*>(base + L.ell);
     h->ctl = reinterpret_cast<mca::DeepCtl*>(base + L.ctl);
     CTRY(cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream));
@@ -837,23 +869,37 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
                                                        mca::kWidthDeep, h->opt.K);
       uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)Kw);
       if (R > 0) kb = std::min<uint64_t>(kb, R - h->tau % R);
+      if (!h->ev[0]) {
+        for (auto& e : h->ev) CUDA_TRY(h, cudaEventCreate(&e));
+      }
+      CUDA_TRY(h, cudaEventRecord(h->ev[0], h->stream));
       if (h->tfm) {
         ta.tau = h->tau;
         ta.Kb = (int)kb;
         CUDA_TRY(h, mca::launch_tfm_eval(ta, h->stream));
+        CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
         CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
       } else {
         a.tau = h->tau;
         a.Kb = (int)kb;
         CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
+        CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
         CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
       }
+      CUDA_TRY(h, cudaEventRecord(h->ev[2], h->stream));
       h->launches += 3;
       mca::DeepCtl ctl;
       CUDA_TRY(h, cudaMemcpyAsync(&ctl, h->ctl, sizeof(ctl), cudaMemcpyDeviceToHost, h->stream));
       CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+      {
+        float ms_eval = 0.0f, ms_rest = 0.0f;
+        CUDA_TRY(h, cudaEventElapsedTime(&ms_eval, h->ev[0], h->ev[1]));
+        CUDA_TRY(h, cudaEventElapsedTime(&ms_rest, h->ev[1], h->ev[2]));
+        h->eval_ns += (uint64_t)(ms_eval * 1e6f);
+        h->rest_ns += (uint64_t)(ms_rest * 1e6f);
+      }
       if (ctl.kstar == -2 || ctl.consumed <= 0) {
         h->broken = true;
         return fail(h, MCA_ERR_NUMERIC, "non-finite loss change");
@@ -1186,6 +1232,8 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
 void mca_destroy(mca_handle* h) {
   if (!h) return;
   cudaStreamSynchronize(h->stream);
+  for (auto& e : h->ev)
+    if (e) cudaEventDestroy(e);
   if (h->ws_owned && h->ws) cudaFree(h->ws);
   if (h->ftau) cudaFree(h->ftau);
   if (h->facc) cudaFree(h->facc);

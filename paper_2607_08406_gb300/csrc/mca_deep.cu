@@ -18,60 +18,11 @@
 #include <algorithm>
 #include <cstdio>
 
+#include "mca_deep.cuh"
 #include "mca_device.cuh"
 #include "mca_internal.h"
 
 namespace mca {
-
-__device__ __forceinline__ DeepCand deep_candidate(const DeepArgs& a, int k) {
-  unsigned int idx;
-  uint32_t r1 = 0u;
-  const bool ex = a.n_explicit > 0;
-  float exv = 0.0f;
-  const unsigned long long P = a.off[a.L];
-  if (ex) {
-    idx = a.ex_idx[k];
-    exv = a.ex_new[k];
-  } else {
-    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
-    idx = (unsigned int)(((unsigned long long)w.x * P) >> 32);
-    r1 = w.y;
-  }
-  int l = 0;
-  while (l + 1 < a.L && (unsigned long long)idx >= a.off[l + 1]) ++l;
-  const unsigned long long off = idx - a.off[l];
-  DeepCand c;
-  c.idx = idx;
-  c.layer = l;
-  c.row = (int)(off / (unsigned long long)a.n_in[l]);
-  c.col = (int)(off % (unsigned long long)a.n_in[l]);
-  const Mutation m = draw_mutation(a.wk[l], a.w[l], a.code[l], a.wfix[l], a.sc[l], off, a.op, a.lo,
-                                   a.hi, a.delta, a.bound, r1, ex, exv);
-  c.oldw = m.oldw;
-  c.neww = m.neww;
-  c.new_code = m.new_code;
-  c.valid = m.valid;
-  c.delta = __fsub_rn(c.neww, c.oldw);
-  return c;
-}
-
-// Loss change of sample n whose output fields become zz (changed: any field differs from the cached
-// one). COMMIT writes the new output fields and loss.
-template <bool COMMIT>
-__device__ __forceinline__ float out_delta(const DeepArgs& a, int n, const float (&zz)[kMaxC],
-                                           bool changed) {
-  if (!changed) return 0.0f;
-  const int Lo = a.L - 1;
-  const float ln = sample_loss<-1, -1, kMaxC>(zz, a.C, a.y[n], a.g[Lo], a.act[Lo], a.loss);
-  const float dl = ln - a.ell[n];
-  if (COMMIT) {
-#pragma unroll
-    for (int c = 0; c < kMaxC; ++c)
-      if (c < a.C) a.Z[Lo][(size_t)c * a.Np + n] = zz[c];
-    a.ell[n] = ln;
-  }
-  return dl;
-}
 
 template <bool COMMIT>
 __global__ void __launch_bounds__(kDeepThreads) deep_chain_kernel(DeepArgs a) {
@@ -401,6 +352,11 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
     const unsigned long long off = c.idx - a.off[l];
     a.w[l][off] = c.neww;
     if (a.wk[l] != MCA_W_FP32) a.code[l][off] = (signed char)c.new_code;
+    if (a.whi[l] != nullptr) {                      // split copy of the tensor-core chain
+      const float h = tf32_rna(c.neww);
+      a.whi[l][off] = h;
+      a.wlo[l][off] = tf32_rna(c.neww - h);
+    }
   } else {
     ctl->consumed = Kb;
     st->trials += (unsigned long long)Kb;
@@ -423,6 +379,7 @@ static size_t chain_smem() {
 }
 
 cudaError_t launch_deep_eval(const DeepArgs& a, cudaStream_t s) {
+  if (a.tc) return launch_deep_eval_tc(a, s);
   const int Kb = a.n_explicit > 0 ? a.n_explicit : a.Kb;
   cudaError_t e = cudaFuncSetAttribute((const void*)deep_chain_kernel<false>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -438,6 +395,7 @@ cudaError_t launch_deep_decide(const DeepArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_deep_commit(const DeepArgs& a, cudaStream_t s) {
+  if (a.tc) return launch_deep_commit_tc(a, s);
   cudaError_t e = cudaFuncSetAttribute((const void*)deep_chain_kernel<true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)chain_smem());

@@ -1,0 +1,494 @@
+// Deep MLP path on the 5th-generation tensor cores: the dense part of a candidate's chain,
+//   Z'_m = Z_m + W_m (f(Z'_{m-1}) - f(Z_{m-1})),   m = l+2 .. L-2   (Section 2.4),
+// as error-compensated 3xTF32 tcgen05 MMAs with the accumulator in tensor memory.
+//
+// One CTA per (candidate, tile of kTcTS = 128 samples), 256 threads. Per dense layer the CTA computes
+// the transposed change D^T[samples x 256] = A[samples x 256] W_m^T, where A holds the previous
+// layer's activation changes split as A = A_hi + A_lo (each rounded to tf32) and W_m = W_hi + W_lo
+// (kept split in global memory, updated with every commit):
+//   D = A_lo W_hi^T + A_hi W_lo^T + A_hi W_hi^T      (the A_lo W_lo^T term, ~2^-22 relative, dropped)
+// Tensor memory (512 columns): D in columns [0, 256) (lane = sample, column = output feature),
+// A_hi in columns [256, 512) (the A operand of two of the three MMAs). A_lo lives in shared memory
+// (128 KB) and W streams through two 32 KB stages of 16-wide K chunks (hi + lo) loaded with cp.async.
+// All operands are K-major without swizzle: 8-row x 16-byte core matrices.
+//
+// The epilogue (all 8 warps; warp w reads tensor-memory lanes 32 (w mod 4) .. + 31, half w / 4 of the
+// features) adds D to the cached fields, forms the next activation change f(z') - f(z) (exactly 0
+// where a field did not change), and writes its hi part to tensor memory and its lo part to shared
+// memory for the next layer; after the last dense layer it accumulates the output layer instead.
+// Every per-(candidate, tile) loss change depends only on that pair: the trajectory does not depend
+// on the batch width. COMMIT writes the fields exactly as the evaluation computed them.
+#include <cstdio>
+
+#include "mca_deep.cuh"
+#include "mca_device.cuh"
+#include "mca_internal.h"
+
+namespace mca {
+namespace {
+
+constexpr int kTcThreads = 256;
+constexpr int kTcW = 256;                  // width of the dense layers
+constexpr int kTcKC = 16;                  // K chunk of a W stage
+constexpr int kTcChunks = kTcW / kTcKC;
+constexpr int kAloBytes = kTcTS * kTcW * 4;          // 128 KB
+constexpr int kWHalfBytes = kTcW * kTcKC * 4;        // 16 KB: one of hi / lo of one chunk
+constexpr int kWStageBytes = 2 * kWHalfBytes;        // 32 KB
+constexpr int kTcSmem = kAloBytes + 2 * kWStageBytes;
+// core-matrix strides (bytes): A_lo: K groups 2 KB apart, sample groups 128 B apart;
+// W stage: K groups 4 KB apart, row groups 128 B apart
+constexpr uint32_t kAloLBO = (kTcTS / 8) * 128, kAloSBO = 128;
+constexpr uint32_t kWLBO = (kTcW / 8) * 128, kWSBO = 128;
+// kind::tf32, D fp32, A and B tf32 K-major, M = 128, N = 256
+constexpr uint32_t kIdesc = (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(kTcW >> 3) << 17) |
+                            ((uint32_t)(kTcTS >> 4) << 24);
+
+static_assert(kTcSmem <= 200 * 1024, "shared memory of the chain kernel");
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;                  // descriptor version; layout type 0 (no swizzle)
+  return d;
+}
+
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t acc) {
+  asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+               "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}\n"
+               ::"r"(d), "l"(a), "l"(b), "r"(kIdesc), "r"(acc));
+}
+
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t acc) {
+  asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+               "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}\n"
+               ::"r"(d), "r"(a), "l"(b), "r"(kIdesc), "r"(acc));
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+               ::"r"(smem_u32(mbar)) : "memory");
+}
+
+// Wait for phase `parity` of an mbarrier, bounded by kBarrierTimeoutNs; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint64_t* mbar, uint32_t parity) {
+  const uint32_t a = smem_u32(mbar);
+  unsigned long long t0 = 0ull;
+  for (unsigned int it = 0;; ++it) {
+    uint32_t done;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}\n" : "=r"(done) : "r"(a), "r"(parity) : "memory");
+    if (done) return true;
+    if ((it & 1023u) == 1023u) {
+      const unsigned long long now = globaltimer_ns();
+      if (t0 == 0ull)
+        t0 = now;
+      else if (now - t0 > kBarrierTimeoutNs)
+        return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+               "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+                 "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+                 "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+               : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int q = 0; q < 16; ++q) v[q] = __uint_as_float(r[q]);
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+               "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+               ::"r"(taddr), "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])),
+                 "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+                 "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+                 "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+                 "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])),
+                 "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+                 "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])),
+                 "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15]))
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+// Stage `buf` <- chunk c (K columns 16c .. 16c+15) of W_hi and W_lo of a dense layer.
+__device__ __forceinline__ void load_w_chunk(uint32_t sw, const float* whi, const float* wlo, int c,
+                                             int buf, int tid) {
+  const uint32_t dh = sw + (uint32_t)(buf * kWStageBytes), dl = dh + kWHalfBytes;
+#pragma unroll
+  for (int it = 0; it < (kTcW * 4) / kTcThreads; ++it) {
+    const int p = tid + it * kTcThreads;
+    const int r = p >> 2, kg = p & 3;
+    const size_t src = (size_t)r * kTcW + (size_t)(c * kTcKC + 4 * kg);
+    const uint32_t dst = (uint32_t)(kg * kWLBO + r * 16);
+    cp_async16(dh + dst, whi + src);
+    cp_async16(dl + dst, wlo + src);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+// A_lo element (sample s, feature k) in shared memory: 16 consecutive features of one sample as
+// four 16-byte stores.
+__device__ __forceinline__ void store_alo16(unsigned char* alo, int s, int f0, const float (&v)[16]) {
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const int k = f0 + 4 * g;
+    *reinterpret_cast<float4*>(alo + (size_t)(k >> 2) * kAloLBO + (size_t)s * 16) =
+        make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
+  }
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
+// Field rows of one layer for this tile into L2 (thread t: row t, four 128-byte lines).
+__device__ __forceinline__ void prefetch_tile(const float* Zm, int Np, int n0, int tid) {
+#pragma unroll
+  for (int p = 0; p < kTcTS / 32; ++p) prefetch_l2(Zm + (size_t)tid * Np + n0 + 32 * p);
+}
+
+// ACTH: transfer function of the hidden layers (-1: read per layer at run time).
+template <bool COMMIT, int ACTH>
+__global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a) {
+  extern __shared__ __align__(1024) unsigned char tsm[];
+  unsigned char* alo = tsm;                                   // A_lo
+  unsigned char* wst = tsm + kAloBytes;                       // W stages
+  __shared__ DeepCand s_cand;
+  __shared__ float s_da[kTcTS];
+  __shared__ float s_red[32];
+  __shared__ __align__(8) uint64_t s_mbar[2];
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int k = COMMIT ? 0 : blockIdx.x;
+  const int tile = COMMIT ? blockIdx.x : blockIdx.y;
+  const int n0 = tile * kTcTS;
+  if (COMMIT && a.ctl->kstar < 0) return;
+  if (tid == 0) {
+    s_cand = COMMIT ? a.ctl->acc : deep_candidate(a, k);
+    s_fail = 0;
+  }
+  __syncthreads();
+  const DeepCand c = s_cand;
+  float* part = a.partial + (size_t)k * a.ntiles + tile;
+  if (!c.valid || c.delta == 0.0f) {
+    if (!COMMIT && tid == 0) *part = 0.0f;
+    return;
+  }
+  const int L = a.L, l = c.layer, j = c.row, i = c.col;
+  const int Np = a.Np, N = a.N;
+  float dl = 0.0f;
+  if (l + 1 < L - 1 && a.n_out[l + 1] == kTcW) prefetch_tile(a.Z[l + 1], Np, n0, tid);
+
+  // ---- row j of layer l (thread s = sample)
+  if (tid < kTcTS) {
+    const int n = n0 + tid;
+    float da = 0.0f;
+    if (n < N) {
+      const float v = l == 0 ? a.XT[(size_t)i * Np + n]
+                             : act_rt(a.act[l - 1], a.Z[l - 1][(size_t)i * Np + n], a.g[l - 1]);
+      float* zp = a.Z[l] + (size_t)j * Np + n;
+      const float z = *zp;
+      const float zn = fmaf(c.delta, v, z);
+      if (l == L - 1) {                              // an output weight: output field j changes
+        float zz[kMaxC];
+#pragma unroll
+        for (int q = 0; q < kMaxC; ++q)
+          zz[q] = q < a.C ? a.Z[l][(size_t)q * Np + n] : 0.0f;
+#pragma unroll
+        for (int q = 0; q < kMaxC; ++q)
+          if (q == j) zz[q] = zn;
+        dl = out_delta<COMMIT>(a, n, zz, zn != z);
+      } else {
+        da = act_rt(a.act[l], zn, a.g[l]) - act_rt(a.act[l], z, a.g[l]);
+        if (COMMIT) *zp = zn;
+      }
+    }
+    s_da[tid] = da;
+  }
+  __syncthreads();
+
+  if (l == L - 2) {
+    // ---- layer l+1 is the output layer: rank-1 change of the output fields
+    if (tid < kTcTS) {
+      const int n = n0 + tid;
+      const float da = s_da[tid];
+      const float* W1 = a.w[L - 1];
+      if (n < N && da != 0.0f) {
+        float zz[kMaxC];
+        bool changed = false;
+#pragma unroll
+        for (int q = 0; q < kMaxC; ++q) {
+          if (q < a.C) {
+            const float zo = a.Z[L - 1][(size_t)q * Np + n];
+            zz[q] = fmaf(W1[(size_t)q * a.n_in[L - 1] + j], da, zo);
+            changed |= zz[q] != zo;
+          } else {
+            zz[q] = 0.0f;
+          }
+        }
+        dl = out_delta<COMMIT>(a, n, zz, changed);
+      }
+    }
+  } else if (l < L - 2) {
+    const bool dense = l + 2 <= L - 2;
+    const int qd = warp & 3, hf = warp >> 2;         // lane quarter, feature half
+    const int s = qd * 32 + lane, n = n0 + s;
+    const bool live = n < N;
+    const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+    uint32_t tmem = 0;
+    if (dense) {
+      if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;"
+                     ::"r"(smem_u32(&s_tmem)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+      }
+      if (tid == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_mbar[0])));
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_mbar[1])));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncthreads();
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      tmem = s_tmem;
+    }
+    // output-layer accumulation of this thread's feature half (after the last change matrix)
+    float outp[kMaxC];
+#pragma unroll
+    for (int q = 0; q < kMaxC; ++q) outp[q] = 0.0f;
+    const float* Wout = a.w[L - 1];
+    const int Kout = a.n_in[L - 1];
+
+    // ---- layer l+1: rank-1 change through column j of W_{l+1}; its activation change is the
+    // first A (dense) or feeds the output layer directly (l = L-3)
+    {
+      const int m1 = l + 1;
+      const float* W1 = a.w[m1];
+      const int K1 = a.n_in[m1];
+      const float da = s_da[s];
+      float* Zm = a.Z[m1];
+      const bool moves = live && da != 0.0f;
+      for (int f0 = hf * (kTcW / 2); f0 < (hf + 1) * (kTcW / 2); f0 += 16) {
+        float hi[16], lo[16], zo[16], wv[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {          // loads first (n < Np: always in the array)
+          wv[q] = W1[(size_t)(f0 + q) * K1 + j];
+          zo[q] = Zm[(size_t)(f0 + q) * Np + n];
+        }
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          const int f = f0 + q;
+          const float zn = fmaf(wv[q], da, zo[q]);
+          const bool ch = moves && zn != zo[q];
+          const float an = act<ACTH>(zn, a.g[m1], a.act[m1]);
+          const float ao = act<ACTH>(zo[q], a.g[m1], a.act[m1]);
+          const float d = ch ? an - ao : 0.0f;
+          if (COMMIT && ch) Zm[(size_t)f * Np + n] = zn;
+          if (dense) {
+            hi[q] = tf32_rna(d);
+            lo[q] = tf32_rna(d - hi[q]);
+          } else {
+#pragma unroll
+            for (int o = 0; o < kMaxC; ++o)
+              if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f], d, outp[o]);
+          }
+        }
+        if (dense) {
+          tmem_st16(tmem + lane_base + 256u + (uint32_t)f0, hi);
+          store_alo16(alo, s, f0, lo);
+        }
+      }
+    }
+
+    // ---- dense layers m = l+2 .. L-2 on the tensor cores
+    if (dense) {
+      const uint32_t sw = smem_u32(wst), salo = smem_u32(alo);
+      uint32_t phase[2] = {0u, 0u};
+      for (int m = l + 2; m <= L - 2; ++m) {
+        const float* whi = a.whi[m];
+        const float* wlo = a.wlo[m];
+        prefetch_tile(a.Z[m], Np, n0, tid);
+        // the previous step's A (tensor memory, shared memory) complete before the MMAs read it
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        load_w_chunk(sw, whi, wlo, 0, 0, tid);
+        for (int cidx = 0; cidx < kTcChunks; ++cidx) {
+          const int b = cidx & 1;
+          if (cidx + 1 < kTcChunks) {
+            const int nb = (cidx + 1) & 1;
+            if (cidx + 1 >= 2) {            // buffer nb last held chunk cidx - 1
+              if (!mbar_wait(&s_mbar[nb], phase[nb])) s_fail = 1;
+              phase[nb] ^= 1u;
+            }
+            load_w_chunk(sw, whi, wlo, cidx + 1, nb, tid);
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+          } else {
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncthreads();
+          if (tid == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+            for (int ks = 0; ks < kTcKC / 8; ++ks) {
+              const int g = cidx * (kTcKC / 8) + ks;       // K step of 8 over the layer
+              const uint64_t dalo = umma_desc(salo + (uint32_t)g * 2u * kAloLBO, kAloLBO, kAloSBO);
+              const uint32_t wb = sw + (uint32_t)(b * kWStageBytes) + (uint32_t)ks * 2u * kWLBO;
+              const uint64_t dwhi = umma_desc(wb, kWLBO, kWSBO);
+              const uint64_t dwlo = umma_desc(wb + kWHalfBytes, kWLBO, kWSBO);
+              const uint32_t tahi = tmem + 256u + (uint32_t)(g * 8);
+              mma_ss(tmem, dalo, dwhi, g > 0 ? 1u : 0u);
+              mma_ts(tmem, tahi, dwlo, 1u);
+              mma_ts(tmem, tahi, dwhi, 1u);
+            }
+            umma_commit(&s_mbar[b]);
+          }
+        }
+        // all MMAs of the layer done (the last commit of each barrier)
+        if (!mbar_wait(&s_mbar[0], phase[0])) s_fail = 1;
+        phase[0] ^= 1u;
+        if (!mbar_wait(&s_mbar[1], phase[1])) s_fail = 1;
+        phase[1] ^= 1u;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (s_fail) break;                            // the same value in every thread here
+
+        // epilogue: new fields, the next A (or the output layer after the last dense layer)
+        const bool last = m == L - 2;
+        float* Zm = a.Z[m];
+        for (int f0 = hf * (kTcW / 2); f0 < (hf + 1) * (kTcW / 2); f0 += 16) {
+          float zo[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) zo[q] = Zm[(size_t)(f0 + q) * Np + n];
+          float dv[16];
+          tmem_ld16(tmem + lane_base + (uint32_t)f0, dv);
+          float hi[16], lo[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const int f = f0 + q;
+            const float zn = zo[q] + dv[q];
+            const bool ch = live && zn != zo[q];
+            const float an = act<ACTH>(zn, a.g[m], a.act[m]);
+            const float ao = act<ACTH>(zo[q], a.g[m], a.act[m]);
+            const float d = ch ? an - ao : 0.0f;
+            if (COMMIT && ch) Zm[(size_t)f * Np + n] = zn;
+            if (!last) {
+              hi[q] = tf32_rna(d);
+              lo[q] = tf32_rna(d - hi[q]);
+            } else {
+#pragma unroll
+              for (int o = 0; o < kMaxC; ++o)
+                if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f], d, outp[o]);
+            }
+          }
+          if (!last) {
+            tmem_st16(tmem + lane_base + 256u + (uint32_t)f0, hi);
+            store_alo16(alo, s, f0, lo);
+          }
+        }
+      }
+    }
+
+    // ---- output layer: the two feature halves of each sample, in a fixed order
+    float* xo = reinterpret_cast<float*>(wst);        // W stages are free now
+    __syncthreads();
+    if (hf == 1) {
+#pragma unroll
+      for (int o = 0; o < kMaxC; ++o) xo[o * kTcTS + s] = outp[o];
+    }
+    __syncthreads();
+    if (hf == 0 && live) {
+      float zz[kMaxC];
+      bool changed = false;
+#pragma unroll
+      for (int o = 0; o < kMaxC; ++o) {
+        if (o < a.C) {
+          const float zo = a.Z[L - 1][(size_t)o * Np + n];
+          zz[o] = zo + (outp[o] + xo[o * kTcTS + s]);
+          changed |= zz[o] != zo;
+        } else {
+          zz[o] = 0.0f;
+        }
+      }
+      dl = out_delta<COMMIT>(a, n, zz, changed);
+    }
+    if (dense) {
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncthreads();
+      if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+      if (tid == 0 && s_fail) atomicCAS(&a.st->err, 0, (int)MCA_ERR_TIMEOUT);
+    }
+  }
+  if (!COMMIT) {
+    const float tot = block_sum(dl, s_red);
+    if (tid == 0) *part = tot;
+  }
+}
+
+// W_hi = tf32(W), W_lo = tf32(W - W_hi) for every dense layer.
+__global__ void deep_split_kernel(DeepArgs a) {
+  const int m = blockIdx.y + 1;
+  if (m > a.L - 2 || a.whi[m] == nullptr) return;
+  const size_t n = (size_t)a.n_out[m] * a.n_in[m];
+  for (size_t e = (size_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+       e += (size_t)gridDim.x * blockDim.x) {
+    const float w = a.w[m][e];
+    const float h = tf32_rna(w);
+    a.whi[m][e] = h;
+    a.wlo[m][e] = tf32_rna(w - h);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_deep_split(const DeepArgs& a, cudaStream_t s) {
+  if (a.L < 3) return cudaSuccess;
+  deep_split_kernel<<<dim3(64, a.L - 2), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// The hidden layers' common transfer function, if every layer 1 .. L-2 has the same one.
+static int hidden_act(const DeepArgs& a) {
+  for (int m = 1; m <= a.L - 2; ++m)
+    if (a.act[m] != a.act[1]) return -1;
+  return a.act[1] == MCA_ACT_TANH ? MCA_ACT_TANH : -1;
+}
+
+template <bool COMMIT>
+static cudaError_t launch_tc(const DeepArgs& a, dim3 grid, cudaStream_t s) {
+  const void* fn = hidden_act(a) == MCA_ACT_TANH
+                       ? (const void*)deep_chain_tc_kernel<COMMIT, MCA_ACT_TANH>
+                       : (const void*)deep_chain_tc_kernel<COMMIT, -1>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem);
+  if (e != cudaSuccess) return e;
+  DeepArgs args = a;
+  void* params[] = {&args};
+  return cudaLaunchKernel(fn, grid, dim3(kTcThreads), params, kTcSmem, s);
+}
+
+cudaError_t launch_deep_eval_tc(const DeepArgs& a, cudaStream_t s) {
+  const int Kb = a.n_explicit > 0 ? a.n_explicit : a.Kb;
+  return launch_tc<false>(a, dim3(Kb, a.ntiles), s);
+}
+
+cudaError_t launch_deep_commit_tc(const DeepArgs& a, cudaStream_t s) {
+  return launch_tc<true>(a, dim3(a.ntiles), s);
+}
+
+}  // namespace mca

@@ -96,6 +96,13 @@ __host__ __device__ __forceinline__ int batch_width(float acc, float trials, flo
   return w >= (float)K ? K : (w < 1.0f ? 1 : (int)w);
 }
 
+// Round to tf32 (10 explicit mantissa bits, nearest, ties away), kept in an fp32 register.
+__device__ __forceinline__ float tf32_rna(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return __uint_as_float(r);
+}
+
 // The same rule with one approximate division (device only; deterministic, so every CTA agrees).
 __device__ __forceinline__ int batch_width_fast(float acc, float trials, float c, int K) {
   const float w = ceilf(__fdividef(c * (trials + 1.0f), acc + 0.5f));

@@ -108,6 +108,7 @@ struct Mlp2Args {
 // ------------------------------------------------------------------------------------------------
 constexpr int kMaxLayers = 32;
 constexpr int kDeepTS = 64;        // samples per tile
+constexpr int kTcTS = 128;         // samples per tile of the tensor-core chain (one MMA M)
 constexpr int kDeepThreads = 256;
 constexpr int kDeepMaxWidth = 256; // widths of the layers inside the dense chain
 constexpr int kDeepKC = 16;        // weight-tile depth of the chain GEMM
@@ -135,6 +136,9 @@ struct DeepArgs {
   signed char* code[kMaxLayers];
   const float* wfix[kMaxLayers];
   float* Z[kMaxLayers];      // [n_out[l] x Np] fields of layer l; Z[L-1] are the output fields
+  float* whi[kMaxLayers];    // tensor-core chain: tf32(W_m) and tf32(W_m - tf32(W_m)) of the
+  float* wlo[kMaxLayers];    //   256 x 256 layers 1 .. L-2 (null otherwise)
+  int tc;                    // 1: dense chain on the tensor cores, tiles of kTcTS samples
   const float* XT;           // [D x Np]
   float* ell;                // [Np] per-sample loss
   const int* y;
@@ -163,6 +167,9 @@ cudaError_t launch_deep_decide(const DeepArgs& a, cudaStream_t s);  // one CTA
 cudaError_t launch_deep_commit(const DeepArgs& a, cudaStream_t s);  // grid ntiles
 cudaError_t launch_deep_forward_layer(const DeepArgs& a, int l, cudaStream_t s);
 cudaError_t launch_deep_losses(const DeepArgs& a, cudaStream_t s);
+cudaError_t launch_deep_split(const DeepArgs& a, cudaStream_t s);     // W_hi / W_lo of all layers
+cudaError_t launch_deep_eval_tc(const DeepArgs& a, cudaStream_t s);   // grid (Kb, ntiles)
+cudaError_t launch_deep_commit_tc(const DeepArgs& a, cudaStream_t s); // grid ntiles
 
 // ------------------------------------------------------------------------------------------------
 // Character-level Transformer path: pre-LN GPT blocks over B sequences of T tokens. All parameters
@@ -286,7 +293,9 @@ struct mca_handle {
   float* srec = nullptr;
   // deep path
   bool deep = false;
+  bool tc = false;                   // dense chain on the tensor cores
   std::vector<float*> Z;
+  std::vector<float*> whi, wlo;      // split weights of layers 1 .. L-2 (tensor-core chain)
   float* ell = nullptr;
   mca::DeepCtl* ctl = nullptr;
   int ntiles = 0;
@@ -307,6 +316,8 @@ struct mca_handle {
   // host-side counters
   unsigned long long tau = 0;
   unsigned long long launches = 0, resyncs = 0;
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};   // per-batch kernel timing (deep, Transformer)
+  unsigned long long eval_ns = 0, rest_ns = 0;
   bool broken = false;                   // a sticky CUDA error or device timeout was seen
   float rate_acc = 0.0f, rate_trials = 0.0f;   // deep path: acceptance counts (batch width)
   // transformer path
