@@ -62,7 +62,7 @@ bool is_device_ptr(const void* p) {
 struct Layout {
   size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, accum, bar, st, trace,
       ex_idx, ex_new, ex_out, scratch, ell, ctl, total;
-  std::vector<size_t> w_eff, code, wfix, Z, whi, wlo;
+  std::vector<size_t> w_eff, code, wfix, Z, whi;
 };
 
 bool is_deep(const std::vector<mca_layer>& layers) { return layers.size() > 2; }
@@ -111,10 +111,8 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   if (deep) {
     for (const auto& ly : layers) L.Z.push_back(take(sizeof(float) * (size_t)ly.n_out * Np));
     if (deep_tc_ok(layers)) {
-      for (size_t l = 1; l + 1 < layers.size(); ++l) {
-        L.whi.push_back(take(sizeof(float) * 256 * 256));
-        L.wlo.push_back(take(sizeof(float) * 256 * 256));
-      }
+      for (size_t l = 1; l + 1 < layers.size(); ++l)
+        L.whi.push_back(take(sizeof(float) * 2 * 256 * 256));   // hi and lo stage images
     }
     L.ell = take(sizeof(float) * (size_t)Np);
     L.ctl = take(sizeof(mca::DeepCtl));
@@ -364,7 +362,6 @@ mca::DeepArgs deep_args(mca_handle* h) {
     a.wfix[l] = h->wfix[l];
     a.Z[l] = h->Z[l];
     a.whi[l] = h->tc && l >= 1 && l + 1 < a.L ? h->whi[l - 1] : nullptr;
-    a.wlo[l] = h->tc && l >= 1 && l + 1 < a.L ? h->wlo[l - 1] : nullptr;
   }
   a.tc = h->tc ? 1 : 0;
   a.off[a.L] = h->P;
@@ -765,10 +762,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   }
   if (h->deep) {
     for (size_t l = 0; l < ls.size(); ++l) h->Z.push_back(reinterpret_cast<float*>(base + L.Z[l]));
-    for (size_t q = 0; q < L.whi.size(); ++q) {
+    for (size_t q = 0; q < L.whi.size(); ++q)
       h->whi.push_back(reinterpret_cast<float*>(base + L.whi[q]));
-      h->wlo.push_back(reinterpret_cast<float*>(base + L.wlo[q]));
-    }
     h->ell = reinterpret_cast<float*>(base + L.ell);
     h->ctl = reinterpret_cast<mca::DeepCtl*>(base + L.ctl);
     CTRY(cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream));

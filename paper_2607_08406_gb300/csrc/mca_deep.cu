@@ -352,10 +352,11 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
     const unsigned long long off = c.idx - a.off[l];
     a.w[l][off] = c.neww;
     if (a.wk[l] != MCA_W_FP32) a.code[l][off] = (signed char)c.new_code;
-    if (a.whi[l] != nullptr) {                      // split copy of the tensor-core chain
+    if (a.whi[l] != nullptr) {                      // split image of the tensor-core chain
       const float h = tf32_rna(c.neww);
-      a.whi[l][off] = h;
-      a.wlo[l][off] = tf32_rna(c.neww - h);
+      const size_t o = deep_tc_image_index(c.row, c.col);
+      a.whi[l][o] = h;
+      a.whi[l][o + 4096] = tf32_rna(c.neww - h);
     }
   } else {
     ctl->consumed = Kb;

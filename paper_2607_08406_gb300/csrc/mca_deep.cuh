@@ -7,6 +7,13 @@
 
 namespace mca {
 
+// Float index of W[r][k] (256 x 256 layer) inside the split-weight image of the tensor-core chain:
+// 16 chunks of 16 columns, each chunk 32 KB (hi 16 KB, then lo), core-matrix order inside
+// (columns 4g .. 4g+3 of 256 rows form a 4 KB block). The lo part is 4096 floats further on.
+__host__ __device__ __forceinline__ size_t deep_tc_image_index(int r, int k) {
+  return (size_t)(k >> 4) * 8192 + (size_t)((k >> 2) & 3) * 1024 + (size_t)r * 4 + (size_t)(k & 3);
+}
+
 __device__ __forceinline__ DeepCand deep_candidate(const DeepArgs& a, int k) {
   unsigned int idx;
   uint32_t r1 = 0u;

@@ -34,16 +34,19 @@ constexpr int kTcChunks = kTcW / kTcKC;
 constexpr int kAloBytes = kTcTS * kTcW * 4;          // 128 KB
 constexpr int kWHalfBytes = kTcW * kTcKC * 4;        // 16 KB: one of hi / lo of one chunk
 constexpr int kWStageBytes = 2 * kWHalfBytes;        // 32 KB
-constexpr int kTcSmem = kAloBytes + 2 * kWStageBytes;
+constexpr int kStages = 3;
+constexpr int kTcSmem = kAloBytes + kStages * kWStageBytes;
 // core-matrix strides (bytes): A_lo: K groups 2 KB apart, sample groups 128 B apart;
-// W stage: K groups 4 KB apart, row groups 128 B apart
+// W stage: K groups 4 KB apart, row groups 128 B apart. The split weights of a layer are kept in
+// global memory as kTcChunks consecutive 32 KB stage images (hi then lo), so that one bulk copy
+// fills a stage.
 constexpr uint32_t kAloLBO = (kTcTS / 8) * 128, kAloSBO = 128;
 constexpr uint32_t kWLBO = (kTcW / 8) * 128, kWSBO = 128;
 // kind::tf32, D fp32, A and B tf32 K-major, M = 128, N = 256
 constexpr uint32_t kIdesc = (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(kTcW >> 3) << 17) |
                             ((uint32_t)(kTcTS >> 4) << 24);
 
-static_assert(kTcSmem <= 200 * 1024, "shared memory of the chain kernel");
+static_assert(kTcSmem + 2048 <= 227 * 1024, "shared memory of the chain kernel");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -120,24 +123,12 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) 
                : "memory");
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-
-// Stage `buf` <- chunk c (K columns 16c .. 16c+15) of W_hi and W_lo of a dense layer.
-__device__ __forceinline__ void load_w_chunk(uint32_t sw, const float* whi, const float* wlo, int c,
-                                             int buf, int tid) {
-  const uint32_t dh = sw + (uint32_t)(buf * kWStageBytes), dl = dh + kWHalfBytes;
-#pragma unroll
-  for (int it = 0; it < (kTcW * 4) / kTcThreads; ++it) {
-    const int p = tid + it * kTcThreads;
-    const int r = p >> 2, kg = p & 3;
-    const size_t src = (size_t)r * kTcW + (size_t)(c * kTcKC + 4 * kg);
-    const uint32_t dst = (uint32_t)(kg * kWLBO + r * 16);
-    cp_async16(dh + dst, whi + src);
-    cp_async16(dl + dst, wlo + src);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
+// One thread: stage st <- the 32 KB image of one chunk, completion counted on mbarrier full.
+__device__ __forceinline__ void load_stage(uint32_t dst, const void* src, uint64_t* full) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
+               ::"r"(smem_u32(full)), "r"((uint32_t)kWStageBytes) : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(dst), "l"(src), "r"((uint32_t)kWStageBytes), "r"(smem_u32(full)) : "memory");
 }
 
 // A_lo element (sample s, feature k) in shared memory: 16 consecutive features of one sample as
@@ -170,7 +161,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
   __shared__ DeepCand s_cand;
   __shared__ float s_da[kTcTS];
   __shared__ float s_red[32];
-  __shared__ __align__(8) uint64_t s_mbar[2];
+  __shared__ __align__(8) uint64_t s_full[kStages], s_empty[kStages];
   __shared__ uint32_t s_tmem;
   __shared__ int s_fail;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -258,9 +249,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
       }
       if (tid == 0) {
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_mbar[0])));
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_mbar[1])));
+        for (int q = 0; q < kStages; ++q) {
+          asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_full[q])));
+          asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_empty[q])));
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        // the first two chunks of the first dense layer load during the rank-1 step
+        const unsigned char* w0 = reinterpret_cast<const unsigned char*>(a.whi[l + 2]);
+        const uint32_t sw0 = smem_u32(wst);
+        for (int q = 0; q < kStages - 1 && q < (L - 2 - (l + 2) + 1) * kTcChunks; ++q)
+          load_stage(sw0 + (uint32_t)(q * kWStageBytes), w0 + (size_t)q * kWStageBytes, &s_full[q]);
       }
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       __syncthreads();
@@ -318,38 +316,29 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
     // ---- dense layers m = l+2 .. L-2 on the tensor cores
     if (dense) {
       const uint32_t sw = smem_u32(wst), salo = smem_u32(alo);
-      uint32_t phase[2] = {0u, 0u};
+      const int nchunks = (L - 2 - (l + 2) + 1) * kTcChunks;   // chunks of all dense layers
       for (int m = l + 2; m <= L - 2; ++m) {
-        const float* whi = a.whi[m];
-        const float* wlo = a.wlo[m];
+        const int li = m - (l + 2);
         prefetch_tile(a.Z[m], Np, n0, tid);
         // the previous step's A (tensor memory, shared memory) complete before the MMAs read it
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        load_w_chunk(sw, whi, wlo, 0, 0, tid);
-        for (int cidx = 0; cidx < kTcChunks; ++cidx) {
-          const int b = cidx & 1;
-          if (cidx + 1 < kTcChunks) {
-            const int nb = (cidx + 1) & 1;
-            if (cidx + 1 >= 2) {            // buffer nb last held chunk cidx - 1
-              if (!mbar_wait(&s_mbar[nb], phase[nb])) s_fail = 1;
-              phase[nb] ^= 1u;
+        __syncthreads();
+        if (tid == 0) {
+          // one thread: wait for a chunk, issue its MMAs, release its stage, refill two ahead
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          for (int cidx = 0; cidx < kTcChunks; ++cidx) {
+            const int gc = li * kTcChunks + cidx, st = gc % kStages;
+            if (!mbar_wait(&s_full[st], (uint32_t)(gc / kStages) & 1u)) {
+              s_fail = 1;
+              break;
             }
-            load_w_chunk(sw, whi, wlo, cidx + 1, nb, tid);
-            asm volatile("cp.async.wait_group 1;" ::: "memory");
-          } else {
-            asm volatile("cp.async.wait_group 0;" ::: "memory");
-          }
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          __syncthreads();
-          if (tid == 0) {
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
             for (int ks = 0; ks < kTcKC / 8; ++ks) {
               const int g = cidx * (kTcKC / 8) + ks;       // K step of 8 over the layer
               const uint64_t dalo = umma_desc(salo + (uint32_t)g * 2u * kAloLBO, kAloLBO, kAloSBO);
-              const uint32_t wb = sw + (uint32_t)(b * kWStageBytes) + (uint32_t)ks * 2u * kWLBO;
+              const uint32_t wb = sw + (uint32_t)(st * kWStageBytes) + (uint32_t)ks * 2u * kWLBO;
               const uint64_t dwhi = umma_desc(wb, kWLBO, kWSBO);
               const uint64_t dwlo = umma_desc(wb + kWHalfBytes, kWLBO, kWSBO);
               const uint32_t tahi = tmem + 256u + (uint32_t)(g * 8);
@@ -357,14 +346,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
               mma_ts(tmem, tahi, dwlo, 1u);
               mma_ts(tmem, tahi, dwhi, 1u);
             }
-            umma_commit(&s_mbar[b]);
+            umma_commit(&s_empty[st]);
+            // chunk gc + 2 goes to the stage chunk gc - 1 used, once its MMAs are done
+            const int nc = gc + kStages - 1;
+            if (nc < nchunks) {
+              const int ns = nc % kStages;
+              if (gc >= 1 && !mbar_wait(&s_empty[ns], (uint32_t)((gc - 1) / kStages) & 1u)) {
+                s_fail = 1;
+                break;
+              }
+              const int nl = l + 2 + nc / kTcChunks, nci = nc % kTcChunks;
+              load_stage(sw + (uint32_t)(ns * kWStageBytes),
+                         reinterpret_cast<const unsigned char*>(a.whi[nl]) +
+                             (size_t)nci * kWStageBytes,
+                         &s_full[ns]);
+            }
           }
         }
-        // all MMAs of the layer done (the last commit of each barrier)
-        if (!mbar_wait(&s_mbar[0], phase[0])) s_fail = 1;
-        phase[0] ^= 1u;
-        if (!mbar_wait(&s_mbar[1], phase[1])) s_fail = 1;
-        phase[1] ^= 1u;
+        // every MMA of the layer done: the last chunk's commit (commits complete in order)
+        {
+          const int gl = li * kTcChunks + kTcChunks - 1;
+          if (!mbar_wait(&s_empty[gl % kStages], (uint32_t)(gl / kStages) & 1u)) s_fail = 1;
+        }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         __syncthreads();
         if (s_fail) break;                            // the same value in every thread here
@@ -441,17 +444,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
   }
 }
 
-// W_hi = tf32(W), W_lo = tf32(W - W_hi) for every dense layer.
+// W_hi = tf32(W), W_lo = tf32(W - W_hi) for every dense layer, stored as the stage images the
+// chain kernel copies (chunk c: hi then lo, core-matrix order).
 __global__ void deep_split_kernel(DeepArgs a) {
   const int m = blockIdx.y + 1;
   if (m > a.L - 2 || a.whi[m] == nullptr) return;
-  const size_t n = (size_t)a.n_out[m] * a.n_in[m];
-  for (size_t e = (size_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-       e += (size_t)gridDim.x * blockDim.x) {
+  const int n = kTcW * kTcW;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
+    const int r = e / kTcW, k = e % kTcW;
     const float w = a.w[m][e];
     const float h = tf32_rna(w);
-    a.whi[m][e] = h;
-    a.wlo[m][e] = tf32_rna(w - h);
+    const size_t o = deep_tc_image_index(r, k);
+    a.whi[m][o] = h;
+    a.whi[m][o + kWHalfBytes / 4] = tf32_rna(w - h);
   }
 }
 

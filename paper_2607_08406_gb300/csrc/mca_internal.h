@@ -137,7 +137,7 @@ struct DeepArgs {
   const float* wfix[kMaxLayers];
   float* Z[kMaxLayers];      // [n_out[l] x Np] fields of layer l; Z[L-1] are the output fields
   float* whi[kMaxLayers];    // tensor-core chain: tf32(W_m) and tf32(W_m - tf32(W_m)) of the
-  float* wlo[kMaxLayers];    //   256 x 256 layers 1 .. L-2 (null otherwise)
+                             //   256 x 256 layers 1 .. L-2 as stage images (null otherwise)
   int tc;                    // 1: dense chain on the tensor cores, tiles of kTcTS samples
   const float* XT;           // [D x Np]
   float* ell;                // [Np] per-sample loss
@@ -295,7 +295,7 @@ struct mca_handle {
   bool deep = false;
   bool tc = false;                   // dense chain on the tensor cores
   std::vector<float*> Z;
-  std::vector<float*> whi, wlo;      // split weights of layers 1 .. L-2 (tensor-core chain)
+  std::vector<float*> whi;           // split-weight images of layers 1 .. L-2 (tensor-core chain)
   float* ell = nullptr;
   mca::DeepCtl* ctl = nullptr;
   int ntiles = 0;
