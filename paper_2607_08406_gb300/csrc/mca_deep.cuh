@@ -14,6 +14,20 @@ __host__ __device__ __forceinline__ size_t deep_tc_image_index(int r, int k) {
   return (size_t)(k >> 4) * 8192 + (size_t)((k >> 2) & 3) * 1024 + (size_t)r * 4 + (size_t)(k & 3);
 }
 
+// Layer of candidate k's weight (proposal only, no memory reads besides the layer offsets).
+__device__ __forceinline__ int deep_candidate_layer(const DeepArgs& a, int k) {
+  unsigned int idx;
+  if (a.n_explicit > 0) {
+    idx = a.ex_idx[k];
+  } else {
+    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
+    idx = (unsigned int)(((unsigned long long)w.x * a.off[a.L]) >> 32);
+  }
+  int l = 0;
+  while (l + 1 < a.L && (unsigned long long)idx >= a.off[l + 1]) ++l;
+  return l;
+}
+
 __device__ __forceinline__ DeepCand deep_candidate(const DeepArgs& a, int k) {
   unsigned int idx;
   uint32_t r1 = 0u;

@@ -164,11 +164,31 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
   __shared__ __align__(8) uint64_t s_full[kStages], s_empty[kStages];
   __shared__ uint32_t s_tmem;
   __shared__ int s_fail;
+  __shared__ int s_k;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int k = COMMIT ? 0 : blockIdx.x;
-  const int tile = COMMIT ? blockIdx.x : blockIdx.y;
-  const int n0 = tile * kTcTS;
+  int k = 0, tile = COMMIT ? blockIdx.x : 0;
   if (COMMIT && a.ctl->kstar < 0) return;
+  if (!COMMIT) {
+    // Longest chains first: CTAs start in linear block order, so the linear index is mapped to
+    // (candidate rank, tile) with the candidates ranked by the depth of their dense chain (the
+    // mutated layer, from the proposal alone), ties by index. Every CTA computes the same ranking.
+    const int Kb = gridDim.x;
+    const int lid = blockIdx.x + blockIdx.y * gridDim.x;
+    const int rank = lid / a.ntiles;
+    tile = lid - rank * a.ntiles;
+    if (tid < Kb) {
+      const int my = deep_candidate_layer(a, tid);
+      int rk = 0;
+      for (int q = 0; q < Kb; ++q) {
+        const int lq = deep_candidate_layer(a, q);
+        rk += (lq < my || (lq == my && q < tid)) ? 1 : 0;     // shallower layer = longer chain
+      }
+      if (rk == rank) s_k = tid;
+    }
+    __syncthreads();
+    k = s_k;
+  }
+  const int n0 = tile * kTcTS;
   if (tid == 0) {
     s_cand = COMMIT ? a.ctl->acc : deep_candidate(a, k);
     s_fail = 0;
