@@ -27,8 +27,10 @@
 namespace mca {
 namespace {
 
-constexpr int kTcThreads = 256;
+constexpr int kTcThreads = 512;
+constexpr int kParts = kTcThreads / 128;     // feature parts per sample (warps sharing a lane quarter)
 constexpr int kTcW = 256;                  // width of the dense layers
+constexpr int kPartW = kTcW / kParts;
 constexpr int kTcKC = 16;                  // K chunk of a W stage
 constexpr int kTcChunks = kTcW / kTcKC;
 constexpr int kAloBytes = kTcTS * kTcW * 4;          // 128 KB
@@ -203,7 +205,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
   const int L = a.L, l = c.layer, j = c.row, i = c.col;
   const int Np = a.Np, N = a.N;
   float dl = 0.0f;
-  if (l + 1 < L - 1 && a.n_out[l + 1] == kTcW) prefetch_tile(a.Z[l + 1], Np, n0, tid);
+  if (l + 1 < L - 1 && a.n_out[l + 1] == kTcW && tid < kTcW)
+    prefetch_tile(a.Z[l + 1], Np, n0, tid);
 
   // ---- row j of layer l (thread s = sample)
   if (tid < kTcTS) {
@@ -257,7 +260,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
     }
   } else if (l < L - 2) {
     const bool dense = l + 2 <= L - 2;
-    const int qd = warp & 3, hf = warp >> 2;         // lane quarter, feature half
+    const int qd = warp & 3, hf = warp >> 2;         // lane quarter, feature part
     const int s = qd * 32 + lane, n = n0 + s;
     const bool live = n < N;
     const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
@@ -301,7 +304,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
       const float da = s_da[s];
       float* Zm = a.Z[m1];
       const bool moves = live && da != 0.0f;
-      for (int f0 = hf * (kTcW / 2); f0 < (hf + 1) * (kTcW / 2); f0 += 16) {
+      for (int f0 = hf * kPartW; f0 < (hf + 1) * kPartW; f0 += 16) {
         float hi[16], lo[16], zo[16], wv[16];
 #pragma unroll
         for (int q = 0; q < 16; ++q) {          // loads first (n < Np: always in the array)
@@ -339,7 +342,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
       const int nchunks = (L - 2 - (l + 2) + 1) * kTcChunks;   // chunks of all dense layers
       for (int m = l + 2; m <= L - 2; ++m) {
         const int li = m - (l + 2);
-        prefetch_tile(a.Z[m], Np, n0, tid);
+        if (tid < kTcW) prefetch_tile(a.Z[m], Np, n0, tid);
         // the previous step's A (tensor memory, shared memory) complete before the MMAs read it
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -395,7 +398,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
         // epilogue: new fields, the next A (or the output layer after the last dense layer)
         const bool last = m == L - 2;
         float* Zm = a.Z[m];
-        for (int f0 = hf * (kTcW / 2); f0 < (hf + 1) * (kTcW / 2); f0 += 16) {
+        for (int f0 = hf * kPartW; f0 < (hf + 1) * kPartW; f0 += 16) {
           float zo[16];
 #pragma unroll
           for (int q = 0; q < 16; ++q) zo[q] = Zm[(size_t)(f0 + q) * Np + n];
@@ -428,14 +431,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
       }
     }
 
-    // ---- output layer: the two feature halves of each sample, in a fixed order
+    // ---- output layer: the feature parts of each sample, in a fixed order
     float* xo = reinterpret_cast<float*>(wst);        // W stages are free now
     __syncthreads();
-    if (hf == 1) {
+    if (hf >= 1) {
 #pragma unroll
-      for (int o = 0; o < kMaxC; ++o) xo[o * kTcTS + s] = outp[o];
+      for (int o = 0; o < kMaxC; ++o) xo[((hf - 1) * kMaxC + o) * kTcTS + s] = outp[o];
     }
     __syncthreads();
+    if (hf == 0) {
+#pragma unroll
+      for (int p = 1; p < kParts; ++p)
+#pragma unroll
+        for (int o = 0; o < kMaxC; ++o) outp[o] += xo[((p - 1) * kMaxC + o) * kTcTS + s];
+    }
     if (hf == 0 && live) {
       float zz[kMaxC];
       bool changed = false;
@@ -443,7 +452,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
       for (int o = 0; o < kMaxC; ++o) {
         if (o < a.C) {
           const float zo = a.Z[L - 1][(size_t)o * Np + n];
-          zz[o] = zo + (outp[o] + xo[o * kTcTS + s]);
+          zz[o] = zo + outp[o];
           changed |= zz[o] != zo;
         } else {
           zz[o] = 0.0f;
