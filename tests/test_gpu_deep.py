@@ -30,6 +30,11 @@ CASES = {
     "ce_w40_d3": dict(),
     "mse_sigmoid_w33_d4": dict(width=33, depth=4, loss="mse_onehot", out_act="sigmoid"),
     "gauss_w64_d2": dict(N=513, width=64, depth=2, hidden="gaussian"),
+    # 256-wide inner layers: the dense chain runs on the tensor cores (3xTF32); 1100 samples leave a
+    # ragged last tile of 76; Gaussian hidden layers take the kernel's run-time transfer function
+    "tc_ce_w256_d5": dict(N=1100, width=256, depth=5),
+    "tc_gauss_mse_w256_d4": dict(N=1100, width=256, depth=4, loss="mse_onehot", out_act="sigmoid",
+                                 hidden="gaussian"),
 }
 
 
@@ -50,8 +55,11 @@ def test_deep_initial_loss_and_trajectory(gpu_lib, case):
     assert st["accepts"] > 20
 
 
-def test_deep_K_invariance(gpu_lib):
-    wl = _deep()
+@pytest.mark.parametrize("width", [40, 256])
+def test_deep_K_invariance(gpu_lib, width):
+    """Trajectories and weights do not depend on the batch width K (SIMT chain at width 40, the
+    tensor-core chain at width 256, whose CTAs are ordered by chain length within each batch)."""
+    wl = _deep(N=700 if width == 40 else 1100, width=width, depth=3 if width == 40 else 5)
     ref = None
     for K in (1, 5, 32, 128):
         h = gpu_lib.create_from_workload(wl, K=K, trace_cap=400)
@@ -84,8 +92,9 @@ def _idx_per_layer(wl, rng, per_layer):
                            for l in range(len(wl.layers))]).astype(np.uint32)
 
 
-def test_deep_eval_candidates_every_layer(gpu_lib):
-    wl = _deep(width=40, depth=4)
+@pytest.mark.parametrize("width", [40, 256])
+def test_deep_eval_candidates_every_layer(gpu_lib, width):
+    wl = _deep(width=width, depth=4, N=700 if width == 40 else 1100)
     h = gpu_lib.create_from_workload(wl)
     gpu_lib.mca_run(h, 300, 5)
     params = O.Params(wl.layers, gpu_lib.mca_get_params(h, wl.n_params))
