@@ -208,6 +208,20 @@ def cpu_oracle_rate(wl, n_trials, warm=0):
     return trials
 
 
+def job_totals(local_ms: float, local_units: float, device=None):
+    """Whole-job aggregate over the ranks of an initialised process group: the slowest rank's time
+    (MAX) and the units every rank processed (SUM). A single process returns its own figures."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return local_ms, local_units
+    mx = torch.tensor([local_ms], dtype=torch.float64, device=device)
+    sm = torch.tensor([local_units], dtype=torch.float64, device=device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx.item()), float(sm.item())
+
+
 def run_reference(args):
     rank, local_rank, world = dist_env()
     if rank != 0:
@@ -292,12 +306,8 @@ def run_ours(args):
     barrier()
     st1 = mca.mca_get_stats(h)
     step_ms = [evs[k].elapsed_time(evs[k + 1]) for k in range(K)]
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    trials_timed = (st1["trials"] - st0["trials"]) * world
+    total_ms, trials_timed = job_totals(sum(step_ms), float(st1["trials"] - st0["trials"]),
+                                        device="cuda")
     value = trials_timed / (total_ms / 1e3)
     launches = st1["launches"] - st0["launches"]
     # dominant kernel: single hidden layer -- the trial loop (one launch per step when no resync
@@ -372,12 +382,9 @@ def run_ours(args):
         for _ in range(args.e2e_steps):
             job()
         torch.cuda.synchronize()
-        dt = time.perf_counter() - t0
-        if world > 1:
-            t = torch.tensor([dt], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            dt = float(t.item())
-        e2e = {"value": e2e_trials * args.e2e_steps * world / dt, "unit": UNIT,
+        dt, e2e_units = job_totals(time.perf_counter() - t0, float(e2e_trials * args.e2e_steps),
+                                   device="cuda")
+        e2e = {"value": e2e_units / dt, "unit": UNIT,
                "h2d_bytes_per_step": int(sum(a.nbytes for a in host_arrays(wl))),
                "d2h_bytes_per_step": int(out.numel() * 4 + 8),
                "step": f"create from pinned host arrays + {e2e_trials} trials + params to host"}
