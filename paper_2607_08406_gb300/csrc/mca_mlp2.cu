@@ -652,7 +652,7 @@ struct CommitLog {
 constexpr bool kPhaseTimers = MCA_PHASE_TIMERS != 0;
 constexpr int kLogLen = 128;
 static_assert(kLogLen > kWS, "a slot is used at most kWS commits after its preparation began");
-constexpr int kProdWarps = 4;
+constexpr int kProdWarps = 3;
 constexpr int kConsWarps = kLoopWarps - kProdWarps;
 constexpr int kConsThreads = kConsWarps * 32;
 
