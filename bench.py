@@ -34,8 +34,8 @@ METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roo
 # from the ncu launch list of `python bench.py --steps 3 --warmup 3 --no-e2e --no-cpu` summarised in
 # profiles/. It is only valid for the kernel source it was measured on; any other source hash
 # reports null.
-LOOP_TRAFFIC = {"source_sha1": "c21e8feec564e69e0d2364185e9d6fbaf6417b2c",
-                "bytes_per_trial": 359457.9}
+LOOP_TRAFFIC = {"source_sha1": "4e88068a1e68ea52e4b82a19ac9993baaf728611",
+                "bytes_per_trial": 359559.0}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
 
