@@ -352,7 +352,7 @@ def run_ours(args):
         if LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and LOOP_TRAFFIC["bytes_per_trial"]:
             traffic = LOOP_TRAFFIC["bytes_per_trial"] * (st1["trials"] - st0["trials"]) / K
         roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                    "frac": achieved / peak, "traffic": traffic, "kernel": "mlp2_trial_loop",
+                    "frac": achieved / peak, "traffic": traffic, "kernel": "mlp2_window_loop",
                     "peak_kind": peak_kind,
                     "bytes": "compulsory DRAM bytes of the distinct candidates evaluated, "
                              "counted by the kernel (per launch)"}

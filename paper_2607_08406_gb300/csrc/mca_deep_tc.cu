@@ -2,18 +2,19 @@
 //   Z'_m = Z_m + W_m (f(Z'_{m-1}) - f(Z_{m-1})),   m = l+2 .. L-2   (Section 2.4),
 // as error-compensated 3xTF32 tcgen05 MMAs with the accumulator in tensor memory.
 //
-// One CTA per (candidate, tile of kTcTS = 128 samples), 256 threads. Per dense layer the CTA computes
+// One CTA per (candidate, tile of kTcTS = 128 samples), 512 threads. Per dense layer the CTA computes
 // the transposed change D^T[samples x 256] = A[samples x 256] W_m^T, where A holds the previous
 // layer's activation changes split as A = A_hi + A_lo (each rounded to tf32) and W_m = W_hi + W_lo
 // (kept split in global memory, updated with every commit):
 //   D = A_lo W_hi^T + A_hi W_lo^T + A_hi W_hi^T      (the A_lo W_lo^T term, ~2^-22 relative, dropped)
 // Tensor memory (512 columns): D in columns [0, 256) (lane = sample, column = output feature),
 // A_hi in columns [256, 512) (the A operand of two of the three MMAs). A_lo lives in shared memory
-// (128 KB) and W streams through two 32 KB stages of 16-wide K chunks (hi + lo) loaded with cp.async.
-// All operands are K-major without swizzle: 8-row x 16-byte core matrices.
+// (128 KB); W streams through three 32 KB stages of 16-wide K chunks (hi + lo), each filled by one
+// bulk copy, in a ring run by one thread (full / empty mbarriers) that reaches across layer
+// boundaries. All operands are K-major without swizzle: 8-row x 16-byte core matrices.
 //
-// The epilogue (all 8 warps; warp w reads tensor-memory lanes 32 (w mod 4) .. + 31, half w / 4 of the
-// features) adds D to the cached fields, forms the next activation change f(z') - f(z) (exactly 0
+// The epilogue (all 16 warps; warp w reads tensor-memory lanes 32 (w mod 4) .. + 31 and a quarter of
+// the features) adds D to the cached fields, forms the next activation change f(z') - f(z) (exactly 0
 // where a field did not change), and writes its hi part to tensor memory and its lo part to shared
 // memory for the next layer; after the last dense layer it accumulates the output layer instead.
 // Every per-(candidate, tile) loss change depends only on that pair: the trajectory does not depend
