@@ -21,7 +21,7 @@ Two evaluation modes, which must agree (the invariant the incremental GPU path r
   mutated neuron's activation change times one weight column (rank-1 in l+1), and the layers from
   l+2 on are recomputed densely.
 
-Readings of points the paper leaves open (each listed in the design doc):
+Readings of points the paper leaves open (the paper is silent on each):
 
 * Proposal stream: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), key = (seed_lo, seed_hi),
   counter = (tau_lo, tau_hi, 0, 0); words r0 (index) and r1 (value) are used.
