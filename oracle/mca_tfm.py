@@ -5,9 +5,8 @@ TEST INFRASTRUCTURE ONLY -- imported by tests/, __graft_entry__.smoke() and benc
 The model (a reading of the paper's sparse description): token + learned position embeddings; per
 block a pre-LN causal multi-head self-attention and a pre-LN feed-forward network (exact-erf GELU, or
 the Gaussian exp(-gamma x^2)), both with residual connections; a final LN and an untied linear head.
-The loss of a
-sequence is the sum of the next-character cross-entropies of its positions; the trial loop decides on
-the sum S over all sequences (Eq. 2 with R = 0, Eq. 6) and reports S / (B * T).
+The loss of a sequence is the sum of the next-character cross-entropies of its positions; the trial
+loop decides on the sum S over all sequences (Eq. 2 with R = 0, Eq. 6) and reports S / (B * T).
 
 The trial loop is the definition: a full forward pass of every sequence after every mutation.
 """
