@@ -24,7 +24,7 @@ constexpr int kRangeTarget = 64;
 // Batch width: ceil(c / p) candidates, p = (A + 0.5) / (T + 1) from counts decayed per batch.
 constexpr float kRateDecay = 0.95f;
 constexpr float kWidthMlp2 = 2.0f;
-constexpr float kWidthDeep = 1.5f;  // samples per range below which fewer CTAs are used
+constexpr float kWidthDeep = 1.0f;   // deep nets and the Transformer (host-driven batches)
 constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
 // Window of the trial loop: kWS candidate slots per CTA, each caching up to kCap entries of the
 // candidate's segment (range-local sample, activation change, new hidden field), prepared ahead of
