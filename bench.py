@@ -423,8 +423,8 @@ def run_ours(args):
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
                                     for q, nm in enumerate(
                                         ["eval_kernel", "decide_commit_kernels"] if deep else
-                                        ["setup", "evaluate", "wait_decide", "wait_cta",
-                                         "add_shares", "commit", "slot_wait"])},
+                                        ["setup_and_commit", "evaluate", "wait_decide",
+                                         "wait_cta", "add_shares", "unused", "slot_wait"])},
                        "slots_reprepared": 0 if deep else st1["phase_ns"][7] - st0["phase_ns"][7],
                        "candidates_timed": st1["candidates"] - st0["candidates"],
                        "loss_end": loss_end},

@@ -136,13 +136,15 @@ typedef struct {
                               candidate 4 B per sample (one hidden-field row); per accepted
                               first-layer candidate the sectors written back */
   uint64_t phase_ns[8];    /* two-layer nets, device time per phase of the trial loop. Windowed
-                              loop (used when its shared-memory window fits), mean over CTAs:
-                              [0] batch set-up, [1] evaluation, [2] the waiting warp's wait for
-                              every CTA's shares + decision, [3] the whole CTA's wait (including
-                              the preparation of later candidates), [4] adding the CTA's shares,
-                              [5] commit, [6] the consumer warps' wait for slots still being
-                              prepared (summed over warps), [7] (a count) slots prepared again
-                              after a commit invalidated them. Other loop, first CTA:
+                              loop (used when its shared-memory window fits), mean over CTAs, [0]
+                              to [6] only in a build with MCA_PHASE_TIMERS=1: [0] batch set-up
+                              together with the previous batch's commit (overlapped), [1]
+                              evaluation, [2] the waiting warp's wait for every CTA's shares +
+                              decision, [3] the whole CTA's wait (including bringing later slots up
+                              to date), [4] adding the CTA's shares, [5] 0, [6] the consumer warps'
+                              wait for slots still being prepared (summed over warps); [7] (a count,
+                              always) slots prepared again after a commit invalidated them. Other
+                              loop, first CTA:
                               [0] proposal + evaluation, [1] grid barrier, [2] reduction +
                               decision, [3] commit. Deep nets and the Transformer (CUDA
                               events around each batch's launches): [0] candidate evaluation
