@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -11,6 +12,7 @@
 
 #include "mca_device.cuh"
 #include "mca_internal.h"
+#include "mca_tc_layout.h"
 
 using mca::DevState;
 using mca::GridBarrier;
@@ -392,6 +394,10 @@ mca::TfmArgs tfm_args(mca_handle* h);
 mca_status resync(mca_handle* h) {
   if (h->tfm) {
     const mca::TfmArgs a = tfm_args(h);
+    if (a.tc) {
+      CUDA_TRY(h, mca::launch_tfm_tc_split(a, h->stream));
+      h->launches += 1;
+    }
     CUDA_TRY(h, mca::launch_tfm_forward(a, h->stream));
     CUDA_TRY(h, mca::launch_sum_loss(h->ell, a.B, h->st, h->stream));
     h->launches += 2;
@@ -536,8 +542,17 @@ mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
 }
 
 struct TfmMem {
-  size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, scratch, total;
+  size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, scratch, wimg,
+      total;
 };
+
+// The tensor-core Transformer kernels (mca_tfm_tc.cu) run a handle's sequences when the process
+// sets MCA_TFM_TENSOR_CORES=1 and the shape is one they handle; otherwise the SIMT kernels do.
+bool tfm_use_tc(const mca_tfm_spec& t, long long B) {
+  const char* e = std::getenv("MCA_TFM_TENSOR_CORES");
+  if (!e || std::strcmp(e, "1") != 0) return false;
+  return mca::tfm_tc_shape_ok(t.ctx, t.d_model, t.n_head, t.d_ff, t.vocab, B);
+}
 
 TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap) {
   TfmMem M;
@@ -560,6 +575,7 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap) {
   M.ex_new = take(sizeof(float) * mca::kKmax);
   M.ex_out = take(sizeof(double) * mca::kKmax);
   M.scratch = take(sizeof(int) * 8);
+  M.wimg = tfm_use_tc(t, B) ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
   M.total = o;
   return M;
 }
@@ -612,6 +628,8 @@ mca::TfmArgs tfm_args(mca_handle* h) {
   a.ftau = h->ftau;
   a.facc = h->facc;
   a.nforce = h->nforce;
+  a.tc = h->tc ? 1 : 0;
+  a.wimg = h->tfm_img;
   return a;
 }
 
@@ -875,6 +893,10 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
         CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
         CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
+        if (ta.tc) {
+          CUDA_TRY(h, mca::launch_tfm_tc_image_update(ta, h->stream));
+          h->launches += 1;
+        }
       } else {
         a.tau = h->tau;
         a.Kb = (int)kb;
@@ -1196,6 +1218,8 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->ex_idx = reinterpret_cast<unsigned int*>(base + M.ex_idx);
   h->ex_new = reinterpret_cast<float*>(base + M.ex_new);
   h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
+  h->tc = tfm_use_tc(*spec, n_seq);
+  h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
   e = cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream);
   if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));

@@ -24,6 +24,7 @@
 #include "mca_deep.cuh"
 #include "mca_device.cuh"
 #include "mca_internal.h"
+#include "mca_tc.cuh"
 
 namespace mca {
 namespace {
@@ -46,92 +47,13 @@ constexpr int kTcSmem = kAloBytes + kStages * kWStageBytes;
 constexpr uint32_t kAloLBO = (kTcTS / 8) * 128, kAloSBO = 128;
 constexpr uint32_t kWLBO = (kTcW / 8) * 128, kWSBO = 128;
 // kind::tf32, D fp32, A and B tf32 K-major, M = 128, N = 256
-constexpr uint32_t kIdesc = (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(kTcW >> 3) << 17) |
-                            ((uint32_t)(kTcTS >> 4) << 24);
+constexpr uint32_t kIdesc = tc_idesc_tf32(kTcTS, kTcW);
 
 static_assert(kTcSmem + 2048 <= 227 * 1024, "shared memory of the chain kernel");
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-
-__device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;                  // descriptor version; layout type 0 (no swizzle)
-  return d;
-}
-
-__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t acc) {
-  asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-               "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}\n"
-               ::"r"(d), "l"(a), "l"(b), "r"(kIdesc), "r"(acc));
-}
-
-__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t acc) {
-  asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-               "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n\t}\n"
-               ::"r"(d), "r"(a), "l"(b), "r"(kIdesc), "r"(acc));
-}
-
-__device__ __forceinline__ void umma_commit(uint64_t* mbar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-               ::"r"(smem_u32(mbar)) : "memory");
-}
-
-// Wait for phase `parity` of an mbarrier, bounded by kBarrierTimeoutNs; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t* mbar, uint32_t parity) {
-  const uint32_t a = smem_u32(mbar);
-  unsigned long long t0 = 0ull;
-  for (unsigned int it = 0;; ++it) {
-    uint32_t done;
-    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-                 "selp.u32 %0, 1, 0, p;\n\t}\n" : "=r"(done) : "r"(a), "r"(parity) : "memory");
-    if (done) return true;
-    if ((it & 1023u) == 1023u) {
-      const unsigned long long now = globaltimer_ns();
-      if (t0 == 0ull)
-        t0 = now;
-      else if (now - t0 > kBarrierTimeoutNs)
-        return false;
-    }
-  }
-}
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[16];
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-               "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-                 "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
-                 "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-               : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int q = 0; q < 16; ++q) v[q] = __uint_as_float(r[q]);
-}
-
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-               "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
-               ::"r"(taddr), "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])),
-                 "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
-                 "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
-                 "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
-                 "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])),
-                 "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
-                 "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])),
-                 "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15]))
-               : "memory");
-}
-
 // One thread: stage st <- the 32 KB image of one chunk, completion counted on mbarrier full.
 __device__ __forceinline__ void load_stage(uint32_t dst, const void* src, uint64_t* full) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
-               ::"r"(smem_u32(full)), "r"((uint32_t)kWStageBytes) : "memory");
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-               ::"r"(dst), "l"(src), "r"((uint32_t)kWStageBytes), "r"(smem_u32(full)) : "memory");
+  bulk_load(dst, src, (uint32_t)kWStageBytes, full);
 }
 
 // A_lo element (sample s, feature k) in shared memory: 16 consecutive features of one sample as
@@ -366,9 +288,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
               const uint64_t dwhi = umma_desc(wb, kWLBO, kWSBO);
               const uint64_t dwlo = umma_desc(wb + kWHalfBytes, kWLBO, kWSBO);
               const uint32_t tahi = tmem + 256u + (uint32_t)(g * 8);
-              mma_ss(tmem, dalo, dwhi, g > 0 ? 1u : 0u);
-              mma_ts(tmem, tahi, dwlo, 1u);
-              mma_ts(tmem, tahi, dwhi, 1u);
+              mma_ss(tmem, dalo, dwhi, kIdesc, g > 0 ? 1u : 0u);
+              mma_ts(tmem, tahi, dwlo, kIdesc, 1u);
+              mma_ts(tmem, tahi, dwhi, kIdesc, 1u);
             }
             umma_commit(&s_empty[st]);
             // chunk gc + 2 goes to the stage chunk gc - 1 used, once its MMAs are done

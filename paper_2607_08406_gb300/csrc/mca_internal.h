@@ -220,6 +220,8 @@ struct TfmArgs {
   const unsigned int* ex_idx;
   const float* ex_new;
   double* ex_out;
+  int tc;                    // 1: the tensor-core kernels (mca_tfm_tc.cu) run the sequences
+  float* wimg;               // their split-weight images (mca_tc_layout.h), tc = 1 only
 };
 
 size_t tfm_smem_bytes(int T, int d, int dh, int V);
@@ -227,6 +229,13 @@ cudaError_t launch_tfm_eval(const TfmArgs& a, cudaStream_t s);      // grid (Kb,
 cudaError_t launch_tfm_decide(const TfmArgs& a, cudaStream_t s);    // one CTA
 cudaError_t launch_tfm_commit(const TfmArgs& a, cudaStream_t s);    // grid B
 cudaError_t launch_tfm_forward(const TfmArgs& a, cudaStream_t s);   // grid B, writes every stage
+// Tensor-core Transformer kernels (two sequences per CTA): the split-weight images from the
+// parameters, the three sequence modes, and the image entry of the accepted parameter after a commit.
+cudaError_t launch_tfm_tc_split(const TfmArgs& a, cudaStream_t s);
+cudaError_t launch_tfm_tc_eval(const TfmArgs& a, cudaStream_t s);      // grid (Kb, B / 2)
+cudaError_t launch_tfm_tc_commit(const TfmArgs& a, cudaStream_t s);    // grid B / 2
+cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s);   // grid B / 2
+cudaError_t launch_tfm_tc_image_update(const TfmArgs& a, cudaStream_t s);
 
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
 cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
@@ -293,7 +302,8 @@ struct mca_handle {
   float* srec = nullptr;
   // deep path
   bool deep = false;
-  bool tc = false;                   // dense chain on the tensor cores
+  bool tc = false;                   // deep: dense chain on the tensor cores; Transformer: the
+                                     // tensor-core sequence kernels
   std::vector<float*> Z;
   std::vector<float*> whi;           // split-weight images of layers 1 .. L-2 (tensor-core chain)
   float* ell = nullptr;
@@ -326,4 +336,5 @@ struct mca_handle {
   float* params = nullptr;               // [P] flat parameters
   int* tokens = nullptr;                 // [B x (ctx + 1)]
   float* X = nullptr;                    // cached residual stream at every stage
+  float* tfm_img = nullptr;              // split-weight images of the tensor-core kernels (tc)
 };

@@ -18,6 +18,7 @@
 
 #include "mca_device.cuh"
 #include "mca_internal.h"
+#include "mca_tfm.cuh"
 
 namespace mca {
 
@@ -35,41 +36,6 @@ size_t tfm_smem_bytes(int T, int d, int dh, int V) {
 __device__ __forceinline__ float ldp(const TfmArgs& a, unsigned long long i,
                                      unsigned long long midx, float mval) {
   return i == midx ? mval : a.params[i];
-}
-
-// Stage of parameter idx: -1 embeddings, b in [0, nL) block b, nL the final LN and head.
-__device__ __forceinline__ int tfm_stage(const TfmArgs& a, unsigned long long idx) {
-  if (idx < a.o_blk0) return -1;
-  if (idx < a.o_lnf_g) return (int)((idx - a.o_blk0) / a.blk_size);
-  return a.nL;
-}
-
-__device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {
-  unsigned int idx;
-  uint32_t r1 = 0u;
-  const bool ex = a.n_explicit > 0;
-  float exv = 0.0f;
-  if (ex) {
-    idx = a.ex_idx[k];
-    exv = a.ex_new[k];
-  } else {
-    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
-    idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
-    r1 = w.y;
-  }
-  const Mutation m = draw_mutation(MCA_W_FP32, a.params, nullptr, nullptr, 1.0f, idx, a.op, a.lo,
-                                   a.hi, a.delta, a.bound, r1, ex, exv);
-  DeepCand c;
-  c.idx = idx;
-  c.layer = tfm_stage(a, idx);
-  c.row = idx < a.o_pos ? (int)(idx / (unsigned long long)a.d) : -1;   // token of a tok_emb entry
-  c.col = 0;
-  c.oldw = m.oldw;
-  c.neww = m.neww;
-  c.new_code = 0;
-  c.valid = m.valid;
-  c.delta = __fsub_rn(c.neww, c.oldw);
-  return c;
 }
 
 // Row-wise layer norm of x [T][d] into h (warp per row).
@@ -577,15 +543,18 @@ static cudaError_t launch_seq(const TfmArgs& a, dim3 grid, cudaStream_t s) {
 }
 
 cudaError_t launch_tfm_eval(const TfmArgs& a, cudaStream_t s) {
+  if (a.tc) return launch_tfm_tc_eval(a, s);
   const int Kb = a.n_explicit > 0 ? a.n_explicit : a.Kb;
   return launch_seq<kTfmEval>(a, dim3(Kb, a.B), s);
 }
 
 cudaError_t launch_tfm_commit(const TfmArgs& a, cudaStream_t s) {
+  if (a.tc) return launch_tfm_tc_commit(a, s);
   return launch_seq<kTfmCommit>(a, dim3(a.B), s);
 }
 
 cudaError_t launch_tfm_forward(const TfmArgs& a, cudaStream_t s) {
+  if (a.tc) return launch_tfm_tc_forward(a, s);
   return launch_seq<kTfmForward>(a, dim3(a.B), s);
 }
 

@@ -1,0 +1,45 @@
+// Pieces of the Transformer trial loop shared by the SIMT kernels (mca_tfm.cu) and the tensor-core
+// kernels (mca_tfm_tc.cu): the stage a parameter feeds and the candidate of trial tau + k.
+#pragma once
+
+#include "mca_device.cuh"
+#include "mca_internal.h"
+
+namespace mca {
+
+// Stage of parameter idx: -1 embeddings, b in [0, nL) block b, nL the final LN and head.
+__device__ __forceinline__ int tfm_stage(const TfmArgs& a, unsigned long long idx) {
+  if (idx < a.o_blk0) return -1;
+  if (idx < a.o_lnf_g) return (int)((idx - a.o_blk0) / a.blk_size);
+  return a.nL;
+}
+
+__device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {
+  unsigned int idx;
+  uint32_t r1 = 0u;
+  const bool ex = a.n_explicit > 0;
+  float exv = 0.0f;
+  if (ex) {
+    idx = a.ex_idx[k];
+    exv = a.ex_new[k];
+  } else {
+    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
+    idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
+    r1 = w.y;
+  }
+  const Mutation m = draw_mutation(MCA_W_FP32, a.params, nullptr, nullptr, 1.0f, idx, a.op, a.lo,
+                                   a.hi, a.delta, a.bound, r1, ex, exv);
+  DeepCand c;
+  c.idx = idx;
+  c.layer = tfm_stage(a, idx);
+  c.row = idx < a.o_pos ? (int)(idx / (unsigned long long)a.d) : -1;   // token of a tok_emb entry
+  c.col = 0;
+  c.oldw = m.oldw;
+  c.neww = m.neww;
+  c.new_code = 0;
+  c.valid = m.valid;
+  c.delta = __fsub_rn(c.neww, c.oldw);
+  return c;
+}
+
+}  // namespace mca
