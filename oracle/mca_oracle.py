@@ -11,7 +11,9 @@ Networks", Section 2 Eq. 1 and Section 3.1 Eq. 6):
         reject without evaluating if the new value leaves the domain |w| < Delta   (Eq. 1)
         W' = W with that one parameter changed
         S' = sum over all N samples of the per-sample loss of f_W'   (full batch, Eq. 2 with R = 0)
-        keep W' iff S' <= S, else keep W   (greedy rule, Eq. 6)
+        keep W' iff S' <= S, else keep W   (greedy rule, Eq. 6; or Eq. 7's Metropolis rule with
+                                             a finite selection intensity beta, as a per-trial
+                                             threshold S' - S <= theta_tau, metropolis_threshold)
 
 Two evaluation modes, which must agree (the invariant the incremental GPU path relies on):
 
@@ -46,7 +48,7 @@ from scipy.special import erf as _erf
 __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
     "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
-    "candidate_dS_two_layer",
+    "candidate_dS_two_layer", "metropolis_threshold",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -308,8 +310,29 @@ class Trace:
         return {f: np.asarray(c, dtype=dt[f]) for f, c in zip(self.FIELDS, cols)}
 
 
-def _decide(dS: float, strict: bool) -> bool:
-    return (dS < 0.0) if strict else (dS <= 0.0)
+def metropolis_threshold(seed: int, tau, beta: float, N: int):
+    """Acceptance threshold of trial tau on the loss-sum change dS (Section 3.1, Eq. 7).
+
+    Eq. 7 keeps a mutation with probability A = min{1, exp(-beta dL)}, dL the change of the mean
+    loss L = S / N. The trial's uniform number is u = (r3 + 1/2) 2^-32, r3 the fourth Philox word
+    of its counter (words r0, r1 draw the proposal), and the trial is kept iff u < exp(-beta dL),
+    i.e. iff dS <= theta = -(N / beta) ln u (theta > 0 since u < 1). beta = inf gives theta = 0,
+    the greedy rule of Eq. 6. Every trial's decision depends only on its own dS and counter, so
+    evaluating several trials against the same state and keeping the lowest-index accepted one
+    reproduces the sequential chain, as for the greedy rule."""
+    if beta == float("inf"):
+        return np.zeros(np.shape(tau)) if np.ndim(tau) else 0.0
+    r3 = draw_words(seed, tau)[..., 3].astype(np.float64)
+    u = (r3 + 0.5) * 2.0 ** -32
+    return -(float(N) / beta) * np.log(u)
+
+
+def _decide(dS: float, strict: bool, theta: float = 0.0) -> bool:
+    return (dS < theta) if strict else (dS <= theta)
+
+
+def _threshold(seed: int, tau: int, domain, N: int) -> float:
+    return float(metropolis_threshold(seed, tau, getattr(domain, "beta", float("inf")), N))
 
 
 def run_full(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials: int, seed: int,
@@ -329,7 +352,7 @@ def run_full(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials: in
         apply_proposal(params, p)
         S_new = total_loss(params, XT, y, loss)
         dS = S_new - S
-        acc = S_new < S if domain.strict else S_new <= S
+        acc = _decide(dS, domain.strict, _threshold(seed, tau0 + t, domain, XT.shape[1]))
         tr.add(p, S, dS, acc)
         if acc:
             S = S_new
@@ -398,7 +421,7 @@ def run_incremental(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_tri
             tr.add(p, S, float("nan"), False)
             continue
         dS, updates, ell_new = _candidate(params, cache, XT, y, loss, p)
-        acc = _decide(dS, domain.strict)
+        acc = _decide(dS, domain.strict, _threshold(seed, tau0 + t, domain, XT.shape[1]))
         tr.add(p, S, dS, acc)
         if acc:
             apply_proposal(params, p)

@@ -151,6 +151,8 @@ def _layers(layers) -> "ctypes.Array":
 
 
 def _domain(d) -> mca_domain:
+    if getattr(d, "beta", float("inf")) != float("inf"):
+        raise ValueError("the Metropolis rule (finite beta) is not part of the C ABI yet")
     return mca_domain(OP[d.op], d.lo, d.hi, d.delta, d.bound, int(bool(d.strict)))
 
 

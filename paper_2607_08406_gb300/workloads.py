@@ -54,6 +54,7 @@ class Domain:
     delta: float = 0.01
     bound: float = 0.0          # > 0: a proposal with |w'| >= bound is rejected unevaluated
     strict: bool = False        # False: accept iff dS <= 0 (Eq. 1, Eq. 6); True: dS < 0
+    beta: float = float("inf")  # selection intensity of the Metropolis rule (Eq. 7); inf: greedy
 
 
 @dataclass
