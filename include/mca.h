@@ -205,7 +205,12 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
 /* Build a trial loop for the Transformer `spec` on n_seq fixed sequences. tokens: [n_seq x (ctx+1)]
  * int32, host or device (inputs tokens[:, :ctx], targets tokens[:, 1:]); init_params: [P] fp32,
  * host or device, in the flat order above. Every parameter is an fp32 weight (Eq. 1 replacement or
- * perturbation). mca_loss reports S / (n_seq * ctx). Errors as for mca_create. */
+ * perturbation). mca_loss reports S / (n_seq * ctx). Errors as for mca_create.
+ * Kernels: SIMT fp32 by default. With MCA_TFM_TENSOR_CORES=1 in the process environment (read by this
+ * call and by mca_tfm_workspace_size, which then includes their weight images) and ctx 64, d_model 128,
+ * 4 heads, d_ff a multiple of 64 up to 1024, vocab <= 128 and an even n_seq, the sequences run on the
+ * tensor-core kernels instead (3xTF32 tcgen05, two sequences per CTA); they have not yet been validated
+ * on a GPU. */
 mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
                                   const int32_t* tokens, int64_t n_seq, const float* init_params,
                                   const mca_options* opt, mca_handle** out);
