@@ -140,25 +140,8 @@ def make_workload(args, rank):
     return wl
 
 
-def deep_tc_shape(wl) -> bool:
-    """The library runs a deep net's dense chain on the tensor cores when every layer between the
-    first and the output layer is 256 x 256."""
-    return len(wl.layers) > 2 and all(ly.n_in == 256 and ly.n_out == 256 for ly in wl.layers[1:-1])
-
-
 def is_tfm(wl) -> bool:
     return hasattr(wl, "spec")
-
-
-def tfm_tc_active(wl) -> bool:
-    """The library runs the Transformer's sequences on its tensor-core kernels when the process sets
-    MCA_TFM_TENSOR_CORES=1 and the shape qualifies (T 64, d 128, 4 heads, d_ff a multiple of 64 up
-    to 1024, vocabulary <= 128, an even number of sequences)."""
-    if not is_tfm(wl) or os.environ.get("MCA_TFM_TENSOR_CORES") != "1":
-        return False
-    sp = wl.spec
-    return (sp.ctx == 64 and sp.d_model == 128 and sp.n_head == 4 and sp.d_ff % 64 == 0
-            and 64 <= sp.d_ff <= 1024 and 2 <= sp.vocab <= 128 and wl.tokens.shape[0] % 2 == 0)
 
 
 def host_arrays(wl):
@@ -334,7 +317,7 @@ def run_ours(args):
         flops_timed = st1["alg_flops"] - st0["alg_flops"]
         eval_s = (st1["phase_ns"][0] - st0["phase_ns"][0]) / 1e9
         achieved = flops_timed / eval_s / 1e12 if eval_s > 0 else 0.0
-        if (not is_tfm(wl) and deep_tc_shape(wl)) or tfm_tc_active(wl):
+        if st1["tensor_cores"]:         # the library reports which kernels the handle runs
             bf16 = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["bf16_tflops"] \
                 if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) else 1900.0
             peak = bf16 * 0.5 / 3.0

@@ -151,6 +151,13 @@ typedef struct {
                               kernel, [1] decision + commit kernels. Rest 0 */
   uint64_t alg_flops;      /* deep nets: FLOPs of the evaluated candidates' recomputation (2 per
                               multiply-add: the row update, the rank-1 layer, the dense layers) */
+  uint32_t tensor_cores;   /* 1: this handle's dense recomputation runs on the tcgen05 tensor-core
+                              kernels (3xTF32): a deep net whose hidden layers are all 256 x 256,
+                              or a Transformer with ctx 64, d_model 128, 4 heads, d_ff a multiple
+                              of 64 up to 1024, vocab <= 128 and an even number of sequences
+                              (unless the process sets MCA_TFM_TENSOR_CORES=0 before creating
+                              the handle); 0: the SIMT fp32 kernels */
+  uint32_t reserved;       /* 0 */
 } mca_run_stats;
 
 typedef struct {
@@ -206,11 +213,12 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
  * int32, host or device (inputs tokens[:, :ctx], targets tokens[:, 1:]); init_params: [P] fp32,
  * host or device, in the flat order above. Every parameter is an fp32 weight (Eq. 1 replacement or
  * perturbation). mca_loss reports S / (n_seq * ctx). Errors as for mca_create.
- * Kernels: SIMT fp32 by default. With MCA_TFM_TENSOR_CORES=1 in the process environment (read by this
- * call and by mca_tfm_workspace_size, which then includes their weight images) and ctx 64, d_model 128,
- * 4 heads, d_ff a multiple of 64 up to 1024, vocab <= 128 and an even n_seq, the sequences run on the
- * tensor-core kernels instead (3xTF32 tcgen05, two sequences per CTA); they have not yet been validated
- * on a GPU. */
+ * Kernels: with ctx 64, d_model 128, 4 heads, d_ff a multiple of 64 up to 1024, vocab <= 128 and an
+ * even n_seq the sequences run on the tensor-core kernels (3xTF32 tcgen05, two sequences per CTA);
+ * for other shapes, or when the process environment has MCA_TFM_TENSOR_CORES=0, on the SIMT fp32
+ * kernels. The variable is read by this call and by mca_tfm_workspace_size (the tensor-core kernels'
+ * weight images are part of the workspace), so it must not change between the two. mca_run_stats
+ * .tensor_cores reports the choice. */
 mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
                                   const int32_t* tokens, int64_t n_seq, const float* init_params,
                                   const mca_options* opt, mca_handle** out);

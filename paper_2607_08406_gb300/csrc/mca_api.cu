@@ -490,6 +490,8 @@ void fill_stats(mca_handle* h, const DevState& d, mca_run_stats* s) {
     s->phase_ns[1] = h->rest_ns;
   }
   s->alg_flops = d.alg_flops;
+  s->tensor_cores = h->tc ? 1u : 0u;
+  s->reserved = 0u;
 }
 
 // ---------------------------------------------------------------- Transformer handles
@@ -546,15 +548,16 @@ struct TfmMem {
       total;
 };
 
-// The tensor-core Transformer kernels (mca_tfm_tc.cu) run a handle's sequences when the process
-// sets MCA_TFM_TENSOR_CORES=1 and the shape is one they handle; otherwise the SIMT kernels do.
+// The tensor-core Transformer kernels (mca_tfm_tc.cu) run a handle's sequences when the shape is
+// one they handle, unless the process sets MCA_TFM_TENSOR_CORES=0 (then, and for every other shape,
+// the SIMT kernels do). Read once per mca_create_transformer / mca_tfm_workspace_size call.
 bool tfm_use_tc(const mca_tfm_spec& t, long long B) {
   const char* e = std::getenv("MCA_TFM_TENSOR_CORES");
-  if (!e || std::strcmp(e, "1") != 0) return false;
+  if (e && std::strcmp(e, "0") == 0) return false;
   return mca::tfm_tc_shape_ok(t.ctx, t.d_model, t.n_head, t.d_ff, t.vocab, B);
 }
 
-TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap) {
+TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc) {
   TfmMem M;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -575,7 +578,7 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap) {
   M.ex_new = take(sizeof(float) * mca::kKmax);
   M.ex_out = take(sizeof(double) * mca::kKmax);
   M.scratch = take(sizeof(int) * 8);
-  M.wimg = tfm_use_tc(t, B) ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
+  M.wimg = tc ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
   M.total = o;
   return M;
 }
@@ -1139,7 +1142,7 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
   if (rc != MCA_OK) return rc;
   if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
   const mca_options o = opt ? *opt : default_options();
-  *bytes = tfm_plan(*spec, n_seq, o.trace_cap).total;
+  *bytes = tfm_plan(*spec, n_seq, o.trace_cap, tfm_use_tc(*spec, n_seq)).total;
   return MCA_OK;
 }
 
@@ -1188,7 +1191,8 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   if (e == cudaSuccess)
     e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
   if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
-  const TfmMem M = tfm_plan(*spec, n_seq, o.trace_cap);
+  h->tc = tfm_use_tc(*spec, n_seq);
+  const TfmMem M = tfm_plan(*spec, n_seq, o.trace_cap, h->tc);
   if (o.workspace) {
     if (o.workspace_bytes < M.total)
       return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
@@ -1218,7 +1222,6 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->ex_idx = reinterpret_cast<unsigned int*>(base + M.ex_idx);
   h->ex_new = reinterpret_cast<float*>(base + M.ex_new);
   h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
-  h->tc = tfm_use_tc(*spec, n_seq);
   h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
   e = cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream);

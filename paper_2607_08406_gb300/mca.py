@@ -55,7 +55,8 @@ class mca_run_stats(Structure):
     _fields_ = [("trials", c_uint64), ("accepts", c_uint64), ("candidates", c_uint64),
                 ("batches", c_uint64), ("wasted", c_uint64), ("forced", c_uint64),
                 ("resyncs", c_uint64), ("launches", c_uint64), ("tau", c_uint64), ("S", c_double),
-                ("alg_bytes", c_uint64), ("phase_ns", c_uint64 * 8), ("alg_flops", c_uint64)]
+                ("alg_bytes", c_uint64), ("phase_ns", c_uint64 * 8), ("alg_flops", c_uint64),
+                ("tensor_cores", c_uint32), ("reserved", c_uint32)]
 
     def asdict(self):
         d = {f: getattr(self, f) for f, _ in self._fields_ if f != "phase_ns"}

@@ -49,6 +49,7 @@ def test_deep_initial_loss_and_trajectory(gpu_lib, case):
     gpu_lib.mca_force_decisions(h, *forced_from_oracle(tr))
     st = gpu_lib.mca_run(h, n, wl.seed)
     assert st["trials"] == n
+    assert st["tensor_cores"] == int(case.startswith("tc_"))
     compare(gpu_lib.mca_get_trace(h, n), tr)
     assert np.array_equal(gpu_lib.mca_get_params(h, wl.n_params), params.flat_eff32())
     assert gpu_lib.mca_loss(h) == pytest.approx(S / wl.N, rel=TIE_REL)
@@ -133,7 +134,7 @@ def test_deep_full_size_24x256(gpu_lib):
     assert np.all(np.abs(d - want) <= TIE_REL * S0), (d, want)
     st = gpu_lib.mca_run(h, 256, wl.seed)
     g = gpu_lib.mca_get_trace(h, 256)
-    assert st["trials"] == 256 and len(g) == 256
+    assert st["trials"] == 256 and len(g) == 256 and st["tensor_cores"] == 1
     params = O.Params(wl.layers, wl.init)
     for t in range(256):
         p = O.propose(wl.seed, t, params, wl.domain)

@@ -1,8 +1,9 @@
 """Parity of the CUDA Transformer path with the CPU oracle (needs a GPU).
 
 Small specs check trajectories (proposals bit for bit, decisions with the tie band replayed, final
-parameters); the config-sized spec (vocab 65, context 64, d_model 128, 2 blocks of 4 heads, FFN 512,
-256 sequences) is checked on candidates of every stage and on a short run.
+parameters) on the SIMT kernels; the config-sized spec (vocab 65, context 64, d_model 128, 2 blocks
+of 4 heads, FFN 512, 256 sequences) is checked on candidates of every stage and on a short run, on
+the tensor-core kernels and on the SIMT kernels.
 """
 import numpy as np
 import pytest
@@ -98,13 +99,17 @@ def test_tfm_resync_keeps_loss(gpu_lib):
     assert gpu_lib.mca_loss(h) == pytest.approx(L, rel=1e-5)
 
 
-def test_tfm_full_size(gpu_lib):
-    """vocab 65, context 64, d_model 128, 2 blocks x 4 heads, FFN 512, 256 sequences: the initial
-    loss and candidates of every stage against the oracle, then 64 trials replayed through the
-    oracle's proposal rule with the final loss."""
+@pytest.mark.parametrize("tensor_cores", ["1", "0"])
+def test_tfm_full_size(gpu_lib, monkeypatch, tensor_cores):
+    """vocab 65, context 64, d_model 128, 2 blocks x 4 heads, FFN 512, 256 sequences, on the
+    tensor-core kernels (the default at this shape) and on the SIMT kernels: the initial loss and
+    candidates of every stage against the oracle, then 64 trials replayed through the oracle's
+    proposal rule with the final loss."""
+    monkeypatch.setenv("MCA_TFM_TENSOR_CORES", tensor_cores)
     wl = W.char_transformer()
     spec = wl.spec
     h = gpu_lib.create_from_tfm_workload(wl, trace_cap=64)
+    assert gpu_lib.mca_get_stats(h)["tensor_cores"] == int(tensor_cores)
     rng = np.random.default_rng(9)
     idx = _stage_indices(spec, rng)[[0, 1, 3, 6, 9, 12]]
     new = rng.uniform(-1, 1, len(idx)).astype(np.float32)
