@@ -7,6 +7,8 @@ block a pre-LN causal multi-head self-attention and a pre-LN feed-forward networ
 the Gaussian exp(-gamma x^2)), both with residual connections; a final LN and an untied linear head.
 The loss of a sequence is the sum of the next-character cross-entropies of its positions; the trial
 loop decides on the sum S over all sequences (Eq. 2 with R = 0, Eq. 6) and reports S / (B * T).
+With a finite selection intensity beta the decision is Eq. 7's Metropolis rule on the mean loss
+L = S / (B * T), i.e. the threshold of metropolis_threshold with N = B * T predicted tokens.
 
 The trial loop is the definition: a full forward pass of every sequence after every mutation.
 """
@@ -14,7 +16,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from .mca_oracle import Trace, act_fn, draw_words
+from .mca_oracle import Trace, act_fn, draw_words, metropolis_threshold
 
 __all__ = ["tfm_views", "tfm_forward", "tfm_seq_losses", "tfm_propose", "run_full_tfm"]
 
@@ -116,7 +118,9 @@ def run_full_tfm(spec, tokens_full, init, n_trials, seed, domain, tau0=0):
         flat[idx] = np.float32(new)
         S_new = float(tfm_seq_losses(spec, flat.astype(np.float64), tokens_full).sum())
         dS = S_new - S
-        acc = S_new < S if domain.strict else S_new <= S
+        theta = float(metropolis_threshold(seed, tau0 + t, getattr(domain, "beta", float("inf")),
+                                           tokens_full.shape[0] * spec.ctx))
+        acc = dS < theta if domain.strict else dS <= theta
         tr.add(p, S, dS, acc)
         if acc:
             S = S_new

@@ -125,3 +125,71 @@ def test_planted_wrong_counter_is_caught(monkeypatch):
     monkeypatch.setattr(O, "_threshold", lambda s, t, d, N: orig(s, t + 1, d, N))
     with pytest.raises(AssertionError):
         test_metropolis_trajectory_matches_enumeration()
+
+
+# ---- the Transformer oracle under Eq. 7 (N = predicted tokens, B sequences x T positions)
+
+from oracle import mca_tfm as T  # noqa: E402
+
+TFM_TINY = W.TfmSpec(vocab=11, ctx=6, d_model=8, n_layer=1, n_head=2, d_ff=16)
+
+
+def _tfm_run(beta, n=400, tokens=None):
+    wl = W.char_transformer(seed=1, batch=4, text_len=4000, spec=TFM_TINY, n_trials=n, K=8)
+    tok = wl.tokens if tokens is None else tokens
+    dom = dataclasses.replace(wl.domain, beta=beta)
+    return wl, T.run_full_tfm(TFM_TINY, tok, wl.init, n, wl.seed, dom)
+
+
+def test_tfm_metropolis_limits():
+    """A huge beta takes the greedy trajectory (Eq. 6); a tiny beta (theta above any loss change)
+    keeps every valid proposal, so the final parameters are the initial ones with every valid
+    proposal applied in order."""
+    wl, (tg, fg, Sg) = _tfm_run(float("inf"), n=150)
+    _, (tb, fb, Sb) = _tfm_run(1e30, n=150)
+    assert (tg["accept"] == tb["accept"]).all() and (fg == fb).all() and Sg == Sb
+    assert 0 < tg["accept"].sum() < tg["valid"].sum()
+    _, (tt, ft, St) = _tfm_run(1e-30, n=150)
+    assert (tt["accept"] == tt["valid"]).all()
+    want = np.array(wl.init, dtype=np.float32)
+    for i, v, ok in zip(tt["idx"], tt["new"], tt["valid"]):
+        if ok:
+            want[int(i)] = np.float32(v)
+    assert (ft == want).all()
+
+
+def test_tfm_metropolis_acceptance_probability():
+    """Eq. 7 on the mean loss per predicted token (L = S / (B T)): given the chain's past, trial t
+    is kept with probability p_t = min{1, exp(-beta dS_t / (B T))}. The number of kept trials must
+    match sum p_t within 5 standard deviations of the Poisson-binomial sum, and uphill moves must
+    be among them."""
+    beta = 400.0
+    wl, (tr, _, _) = _tfm_run(beta)
+    v = tr["valid"]
+    n_tok = wl.tokens.shape[0] * TFM_TINY.ctx
+    p = np.minimum(1.0, np.exp(-beta * tr["dS"][v] / n_tok))
+    kept = tr["accept"][v].sum()
+    sig = math.sqrt(float((p * (1.0 - p)).sum()))
+    assert abs(kept - p.sum()) <= 5.0 * sig + 1.0, (kept, p.sum(), sig)
+    uphill = (tr["dS"] > 0) & tr["accept"]
+    assert uphill.sum() > 10
+    assert ((p > 0.05) & (p < 0.95)).sum() > 50       # the test is not decided by the limits
+
+
+def test_tfm_metropolis_batch_duplication_invariance():
+    """Repeating every sequence doubles S, each dS and the token count B T, so Eq. 7's decisions
+    do not change (trials within 1e-9 of their threshold excepted)."""
+    wl, (t1, f1, S1) = _tfm_run(400.0, n=200)
+    tok2 = np.concatenate([wl.tokens, wl.tokens])
+    _, (t2, f2, S2) = _tfm_run(400.0, n=200, tokens=tok2)
+    assert S2 == pytest.approx(2.0 * S1, rel=1e-12)
+    assert (t1["accept"] == t2["accept"]).all() and (f1 == f2).all()
+
+
+def test_planted_sequence_count_for_token_count_is_caught(monkeypatch):
+    """Taking N = B sequences instead of B T predicted tokens fails the probability pin."""
+    orig = T.metropolis_threshold
+    monkeypatch.setattr(T, "metropolis_threshold",
+                        lambda s, t, b, N: orig(s, t, b, N // TFM_TINY.ctx))
+    with pytest.raises(AssertionError):
+        test_tfm_metropolis_acceptance_probability()
