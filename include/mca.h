@@ -79,13 +79,21 @@ typedef struct {
   float scale;             /* TERNARY_I8: effective weight = scale * code; ignored otherwise */
 } mca_layer;
 
-/* Weight domain and acceptance rule (Eq. 1, Eq. 6). */
+/* Weight domain and acceptance rule (Eq. 1; Eq. 6, or Eq. 7 with temperature > 0). */
 typedef struct {
   int32_t op;              /* mca_op */
   float lo, hi;            /* REPLACE range [lo, hi) */
   float delta;             /* PERTURB amplitude */
   float bound;             /* > 0: a proposal with !(|w'| < bound) is rejected unevaluated */
-  int32_t strict;          /* 0: accept iff dS <= 0 (Eq. 1, Eq. 6); 1: accept iff dS < 0 */
+  int32_t strict;          /* 0: accept iff dS <= theta; 1: accept iff dS < theta */
+  float temperature;       /* 1 / beta of the Metropolis rule (Section 3.1, Eq. 7), finite, >= 0.
+                              0: the greedy rule (Eq. 6), theta = 0. > 0: Eq. 7's acceptance
+                              probability min{1, exp(-beta dS / N)} as a per-trial threshold
+                              theta = -(N / beta) ln u on the loss-sum change, with the trial's
+                              own uniform number u = (r3 + 1/2) 2^-32, r3 the fourth word of
+                              Philox4x32-10(key = seed, counter = tau); N = samples (MLP) or
+                              n_seq * ctx predicted tokens (Transformer). theta depends only on
+                              the trial, so speculative batches keep the sequential chain */
 } mca_domain;
 
 /* Training set. x: [n x d] fp32, sample-major (sample n's features at x + n * d); y: [n] int32

@@ -327,6 +327,8 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.delta = h->dom.delta;
   a.bound = h->dom.bound;
   a.strict = h->dom.strict;
+  a.metro = h->dom.temperature > 0.0f ? 1 : 0;
+  a.msc = (double)h->N * (double)h->dom.temperature;
   a.K = h->opt.K;
   a.fixed_K = h->opt.fixed_K;
   a.partial = h->partial;
@@ -377,6 +379,8 @@ mca::DeepArgs deep_args(mca_handle* h) {
   a.delta = h->dom.delta;
   a.bound = h->dom.bound;
   a.strict = h->dom.strict;
+  a.metro = h->dom.temperature > 0.0f ? 1 : 0;
+  a.msc = (double)h->N * (double)h->dom.temperature;
   a.partial = h->partial;
   a.st = h->st;
   a.ctl = h->ctl;
@@ -622,6 +626,8 @@ mca::TfmArgs tfm_args(mca_handle* h) {
   a.delta = h->dom.delta;
   a.bound = h->dom.bound;
   a.strict = h->dom.strict;
+  a.metro = h->dom.temperature > 0.0f ? 1 : 0;
+  a.msc = (double)h->N * (double)h->dom.temperature;
   a.smem = mca::tfm_smem_bytes(a.T, a.d, a.dh, a.V);
   a.partial = h->partial;
   a.st = h->st;
@@ -688,6 +694,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     return fail(nullptr, MCA_ERR_INVALID, "unknown op %d", d.op);
   if (!std::isfinite(d.lo) || !std::isfinite(d.hi) || !std::isfinite(d.delta) || !(d.hi > d.lo))
     return fail(nullptr, MCA_ERR_INVALID, "bad domain");
+  if (!std::isfinite(d.temperature) || d.temperature < 0.0f)
+    return fail(nullptr, MCA_ERR_INVALID, "temperature %g: must be finite and >= 0", d.temperature);
 
   mca_handle* h = new (std::nothrow) mca_handle();
   if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
@@ -1163,6 +1171,8 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
     return fail(nullptr, MCA_ERR_INVALID, "unknown op %d", d.op);
   if (!std::isfinite(d.lo) || !std::isfinite(d.hi) || !std::isfinite(d.delta) || !(d.hi > d.lo))
     return fail(nullptr, MCA_ERR_INVALID, "bad domain");
+  if (!std::isfinite(d.temperature) || d.temperature < 0.0f)
+    return fail(nullptr, MCA_ERR_INVALID, "temperature %g: must be finite and >= 0", d.temperature);
   mca_handle* h = new (std::nothrow) mca_handle();
   if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
   auto bail = [&](mca_status st) {

@@ -12,8 +12,9 @@
 //   deep_eval     grid (K, tiles): CTA (k, t) runs candidate k's chain over tile t's kDeepTS samples,
 //                 the change matrix staying in shared memory from layer to layer, and writes one
 //                 partial loss change per (candidate, tile) -- a fixed computation, independent of K
-//   deep_decide   one CTA: fixed-order (compensated fp32) sums, lowest-index candidate with dS <= 0
-//                 (Eq. 6), trace, statistics, weight update
+//   deep_decide   one CTA: fixed-order (compensated fp32) sums, lowest-index candidate with
+//                 dS <= theta (Eq. 6: theta = 0; Eq. 7: the trial's Metropolis threshold), trace,
+//                 statistics, weight update
 //   deep_commit   grid (tiles): the accepted candidate's chain with writes
 #include <algorithm>
 #include <cstdio>
@@ -271,7 +272,7 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
         acc = facc;
       } else {
         bad = !isfinite(d);
-        acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
+        acc = accept_change(d, a.strict, a.metro, a.seed, tk, a.msc);
       }
     }
   }

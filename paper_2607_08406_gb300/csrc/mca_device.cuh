@@ -33,6 +33,24 @@ __device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
                        make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
 }
 
+// Threshold of the Metropolis rule (Section 3.1, Eq. 7) on the loss-sum change of trial tau. Eq. 7
+// keeps a mutation with probability min{1, exp(-beta dS / N)}; with the trial's own uniform number
+// u = (r3 + 1/2) 2^-32, r3 the fourth Philox word of its counter, that is u < exp(-beta dS / N),
+// i.e. dS <= -(N / beta) ln u. msc = N / beta > 0. Evaluated in fp64 (once per candidate and
+// batch) and rounded to the fp32 of the candidate's dS.
+__device__ __forceinline__ float metropolis_theta(uint64_t seed, uint64_t tau, double msc) {
+  const uint32_t r3 = trial_words(seed, tau).w;
+  const double u = ((double)r3 + 0.5) * 0x1p-32;
+  return (float)(-msc * log(u));
+}
+
+// Acceptance of a candidate with loss-sum change d (Eq. 6, or Eq. 7 when metro != 0).
+__device__ __forceinline__ bool accept_change(float d, int strict, int metro, uint64_t seed,
+                                              uint64_t tau, double msc) {
+  const float th = metro ? metropolis_theta(seed, tau, msc) : 0.0f;
+  return strict ? (d < th) : (d <= th);
+}
+
 // u = (r >> 8) * 2^-24: exact, in [0, 1)
 __device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >> 8) * 0x1p-24f; }
 

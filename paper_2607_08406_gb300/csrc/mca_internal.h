@@ -83,6 +83,8 @@ struct Mlp2Args {
   int op;
   float lo, hi, delta, bound;
   int strict;
+  int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
+  double msc;
   unsigned long long seed, tau0, n_trials;
   int K;
   int fixed_K;
@@ -146,6 +148,8 @@ struct DeepArgs {
   int op;
   float lo, hi, delta, bound;
   int strict;
+  int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
+  double msc;
   unsigned long long seed, tau;
   int Kb;
   float* partial;            // [kKmax x ntiles]
@@ -204,6 +208,8 @@ struct TfmArgs {
   int op;
   float lo, hi, delta, bound;
   int strict;
+  int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
+  double msc;
   unsigned long long seed, tau;
   int Kb;
   int mode;

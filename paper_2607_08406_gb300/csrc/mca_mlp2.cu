@@ -18,7 +18,8 @@
 //             (warp per sub-chunk, fixed lane order), and writes one partial per (candidate, range)
 //   barrier   the only grid-wide synchronisation of a batch
 //   decide    every CTA sums each candidate's NR partials in the same fixed order and takes the
-//             lowest-index candidate with dS <= 0 (Eq. 6): the same answer in every CTA
+//             lowest-index candidate with dS <= theta (Eq. 6: theta = 0; Eq. 7: the trial's
+//             Metropolis threshold): the same answer in every CTA
 //   commit    each CTA applies the accepted candidate to its own samples (no barrier needed: no
 //             other CTA reads them) and writes the new weight value (the same value from all CTAs)
 // Every partial depends only on (candidate, range), so dS and the trajectory do not depend on K.
@@ -443,7 +444,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
       break;
     }
 
-    // ---- decide (the same in every CTA): lowest-index candidate with dS <= 0 (Eq. 6)
+    // ---- decide (the same in every CTA): lowest-index candidate with dS <= theta (Eq. 6 / 7)
     if (warp < kKmax / 32) {
       bool acc = false, bad = false, forced = false;
       const int k = tid;
@@ -469,7 +470,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
           acc = facc;
         } else {
           bad = !isfinite(d);
-          acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
+          acc = accept_change(d, a.strict, a.metro, a.seed, tk, a.msc);
         }
       }
       const unsigned int ma = __ballot_sync(0xffffffffu, acc);
@@ -1282,9 +1283,9 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
             break;
           }
         }
-        // decide in the same warp (the same in every CTA): lowest-index candidate with dS <= 0
-        // (Eq. 6); decisions forced by the caller take precedence; a non-finite dS at or before
-        // the first acceptance stops the run
+        // decide in the same warp (the same in every CTA): lowest-index candidate with
+        // dS <= theta (Eq. 6 / Eq. 7); decisions forced by the caller take precedence; a
+        // non-finite dS at or before the first acceptance stops the run
         unsigned int mask_a[2], mask_b[2], mask_f[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -1323,7 +1324,7 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_window_loop(Mlp2Args a) 
                 accept = facc;
               } else {
                 bad = !isfinite(d);
-                accept = a.strict ? (d < 0.0f) : (d <= 0.0f);
+                accept = accept_change(d, a.strict, a.metro, a.seed, tk, a.msc);
               }
             }
           }

@@ -12,7 +12,8 @@
 // cached per sequence; a rejected candidate writes nothing.
 //
 // Per batch: tfm_eval (grid K x B, one partial loss change per candidate and sequence), tfm_decide
-// (one CTA, fixed-order sums, Eq. 6), tfm_commit (grid B: the accepted candidate with writes).
+// (one CTA, fixed-order sums, Eq. 6 or Eq. 7), tfm_commit (grid B: the accepted candidate with
+// writes).
 #include <algorithm>
 #include <cstdio>
 
@@ -456,7 +457,7 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
         acc = facc;
       } else {
         bad = !isfinite(d);
-        acc = a.strict ? (d < 0.0f) : (d <= 0.0f);
+        acc = accept_change(d, a.strict, a.metro, a.seed, tk, a.msc);
       }
     }
   }

@@ -32,7 +32,7 @@ class mca_layer(Structure):
 
 class mca_domain(Structure):
     _fields_ = [("op", c_int32), ("lo", c_float), ("hi", c_float), ("delta", c_float),
-                ("bound", c_float), ("strict", c_int32)]
+                ("bound", c_float), ("strict", c_int32), ("temperature", c_float)]
 
 
 class mca_dataset(Structure):
@@ -152,9 +152,11 @@ def _layers(layers) -> "ctypes.Array":
 
 
 def _domain(d) -> mca_domain:
-    if getattr(d, "beta", float("inf")) != float("inf"):
-        raise ValueError("the Metropolis rule (finite beta) is not part of the C ABI yet")
-    return mca_domain(OP[d.op], d.lo, d.hi, d.delta, d.bound, int(bool(d.strict)))
+    beta = float(getattr(d, "beta", float("inf")))
+    if not beta > 0.0:
+        raise ValueError(f"beta = {beta}: the selection intensity must be > 0 (inf: greedy rule)")
+    return mca_domain(OP[d.op], d.lo, d.hi, d.delta, d.bound, int(bool(d.strict)),
+                      0.0 if beta == float("inf") else 1.0 / beta)
 
 
 class Handle:

@@ -13,14 +13,16 @@ def oracle_trace(wl, n_trials, seed=0, mode="incremental", domain=None):
     return tr, params, S
 
 
-def tie_band(tr):
-    """Trials where the oracle's |dS| < TIE_REL * S and dS != 0 (exact zeros must match)."""
-    d = np.abs(tr["dS"])
+def tie_band(tr, theta=0.0):
+    """Trials where the oracle's dS lies within TIE_REL * S of the acceptance threshold theta (0 for
+    the greedy rule, Eq. 6; per trial for the Metropolis rule, Eq. 7) and dS != 0 (exact zeros,
+    the no-op proposals, must match)."""
+    d = np.abs(tr["dS"] - theta)
     return tr["valid"] & (d < TIE_REL * np.abs(tr["S"])) & (tr["dS"] != 0.0)
 
 
-def forced_from_oracle(tr):
-    m = tie_band(tr)
+def forced_from_oracle(tr, theta=0.0):
+    m = tie_band(tr, theta)
     return tr["tau"][m].astype(np.uint64), tr["accept"][m]
 
 

@@ -105,6 +105,12 @@ def test_invalid_specs_rejected_without_gpu(lib):
     rc = lib.mca_create(big, 2, 0, None, ctypes.byref(ds), wl.init.ctypes.data, None,
                         ctypes.byref(h))
     assert rc == mca.MCA_ERR_UNSUPPORTED
+    # Metropolis temperature (1 / beta, Eq. 7) must be finite and >= 0
+    for t in (-1.0, float("nan"), float("inf")):
+        d = mca.mca_domain(0, -1.0, 1.0, 0.01, 0.0, 0, t)
+        rc = lib.mca_create(L, n, 0, ctypes.byref(d), ctypes.byref(ds), wl.init.ctypes.data,
+                            None, ctypes.byref(h))
+        assert rc == mca.MCA_ERR_INVALID and b"temperature" in lib.mca_last_error(None)
     # NULL handle calls
     assert lib.mca_run(None, 1, 0, None) == mca.MCA_ERR_INVALID
     lib.mca_destroy(None)
@@ -116,3 +122,14 @@ def test_binding_names_match_c_abi():
         if n == "mca_last_error":
             continue
         assert callable(getattr(mca, n)), n
+
+
+def test_binding_maps_beta_to_temperature():
+    """The binding passes Eq. 7's beta as temperature = 1 / beta (0 for the greedy rule, beta = inf)
+    and refuses beta <= 0."""
+    assert mca._domain(W.Domain()).temperature == 0.0
+    d = mca._domain(W.Domain(beta=250.0, strict=True))
+    assert d.temperature == pytest.approx(1.0 / 250.0) and d.strict == 1
+    for bad in (0.0, -3.0, float("nan")):
+        with pytest.raises(ValueError):
+            mca._domain(W.Domain(beta=bad))
