@@ -28,7 +28,9 @@ Readings of points the paper leaves open (the paper is silent on each):
 * Proposal stream: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), key = (seed_lo, seed_hi),
   counter = (tau_lo, tau_hi, 0, 0); words r0 (index) and r1 (value) are used.
 * Index: idx = floor(r0 * P / 2^32) over the flat parameter space (layers in forward order,
-  each weight matrix [out x in] row-major).
+  each weight matrix [out x in] row-major). With the current-layer schedule of Section 2.1
+  (domain.layer_stretch = M > 0), stretches of M trials each mutate one layer chosen uniformly at
+  random, the index uniform inside it (proposal_index, stretch_layer).
 * Replacement value: u = (r1 >> 8) * 2^-24 in fp32, w' = lo + (hi - lo) * u with two fp32
   roundings (for [lo, hi) = [-1, 1) this is exact). Perturbation: r = 2u - 1 (exact),
   w' = w + delta * r in fp32.
@@ -48,7 +50,7 @@ from scipy.special import erf as _erf
 __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
     "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
-    "candidate_dS_two_layer", "metropolis_threshold",
+    "candidate_dS_two_layer", "metropolis_threshold", "stretch_layer", "proposal_index",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -174,11 +176,36 @@ class Proposal:
     valid: bool         # False: outside the weight domain, rejected without evaluation
 
 
+def stretch_layer(seed: int, s, n_layers: int):
+    """Layer of stretch s under the current-layer schedule (Section 2.1): a layer chosen uniformly at
+    random, l_s = floor(q * n_layers / 2^32), q the first word of Philox4x32-10 under the proposal
+    key at counter (s_lo, s_hi, 1, 0) -- the third counter word keeps these draws apart from the
+    trials' own words (counter (tau_lo, tau_hi, 0, 0))."""
+    s = np.asarray(s, dtype=np.uint64)
+    ctr = np.stack([s & _M32, s >> _S32, np.ones_like(s), np.zeros_like(s)], axis=-1)
+    k = np.uint64(seed)
+    key = np.broadcast_to(np.array([k & _M32, k >> _S32], dtype=np.uint64), ctr.shape[:-1] + (2,))
+    q = philox4x32_10(ctr, key)[..., 0]
+    return (q * np.uint64(n_layers)) >> _S32
+
+
+def proposal_index(seed: int, tau: int, r0: int, offsets: Sequence[int], stretch: int) -> int:
+    """Flat index of trial tau's parameter; offsets: the first index of every layer, then P.
+    stretch = 0: uniform over all P parameters (Eq. 1),
+    floor(r0 P / 2^32). stretch = M > 0, the current-layer schedule of Section 2.1: the trials of
+    stretch s = floor(tau / M) mutate only layer l_s (stretch_layer), each trial's index uniform
+    inside that layer, offsets[l_s] + floor(r0 P_l / 2^32)."""
+    if stretch <= 0:
+        return (r0 * offsets[-1]) >> 32
+    l = int(stretch_layer(seed, tau // stretch, len(offsets) - 1))
+    return offsets[l] + ((r0 * (offsets[l + 1] - offsets[l])) >> 32)
+
+
 def propose(seed: int, tau: int, params: Params, domain) -> Proposal:
     r = draw_words(seed, tau)
     r0, r1 = int(r[0]), int(r[1])
-    P = params.n_params
-    idx = (r0 * P) >> 32
+    idx = proposal_index(seed, tau, r0, list(params.offsets) + [params.n_params],
+                         getattr(domain, "layer_stretch", 0))
     l = 0
     while l + 1 < len(params.layers) and idx >= params.offsets[l + 1]:
         l += 1

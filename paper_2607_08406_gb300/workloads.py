@@ -55,6 +55,8 @@ class Domain:
     bound: float = 0.0          # > 0: a proposal with |w'| >= bound is rejected unevaluated
     strict: bool = False        # False: accept iff dS <= 0 (Eq. 1, Eq. 6); True: dS < 0
     beta: float = float("inf")  # selection intensity of the Metropolis rule (Eq. 7); inf: greedy
+    layer_stretch: int = 0      # > 0: current-layer schedule (Section 2.1), stretches of this many
+                                #   trials each mutating one randomly chosen layer; 0: uniform
 
 
 @dataclass
