@@ -94,6 +94,14 @@ typedef struct {
                               Philox4x32-10(key = seed, counter = tau); N = samples (MLP) or
                               n_seq * ctx predicted tokens (Transformer). theta depends only on
                               the trial, so speculative batches keep the sequential chain */
+  int32_t layer_stretch;   /* 0: each trial's parameter is uniform over all P parameters (Eq. 1).
+                              M > 0 (MLPs; the current-layer schedule of Section 2.1): trials come
+                              in stretches of M, stretch s = tau / M mutating only layer l_s,
+                              l_s = floor(q * n_layers / 2^32) with q the first word of
+                              Philox4x32-10(key = seed, counter = (s_lo, s_hi, 1, 0)); the index
+                              is uniform inside that layer: first index of l_s +
+                              floor(r0 * (size of l_s) / 2^32). The Transformer takes 0 only
+                              (MCA_ERR_UNSUPPORTED otherwise) */
 } mca_domain;
 
 /* Training set. x: [n x d] fp32, sample-major (sample n's features at x + n * d); y: [n] int32

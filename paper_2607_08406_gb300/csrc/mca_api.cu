@@ -329,6 +329,7 @@ mca::Mlp2Args mlp2_args(mca_handle* h) {
   a.strict = h->dom.strict;
   a.metro = h->dom.temperature > 0.0f ? 1 : 0;
   a.msc = (double)h->N * (double)h->dom.temperature;
+  a.stretch = h->dom.layer_stretch;
   a.K = h->opt.K;
   a.fixed_K = h->opt.fixed_K;
   a.partial = h->partial;
@@ -381,6 +382,7 @@ mca::DeepArgs deep_args(mca_handle* h) {
   a.strict = h->dom.strict;
   a.metro = h->dom.temperature > 0.0f ? 1 : 0;
   a.msc = (double)h->N * (double)h->dom.temperature;
+  a.stretch = h->dom.layer_stretch;
   a.partial = h->partial;
   a.st = h->st;
   a.ctl = h->ctl;
@@ -628,6 +630,7 @@ mca::TfmArgs tfm_args(mca_handle* h) {
   a.strict = h->dom.strict;
   a.metro = h->dom.temperature > 0.0f ? 1 : 0;
   a.msc = (double)h->N * (double)h->dom.temperature;
+  a.stretch = h->dom.layer_stretch;
   a.smem = mca::tfm_smem_bytes(a.T, a.d, a.dh, a.V);
   a.partial = h->partial;
   a.st = h->st;
@@ -696,6 +699,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     return fail(nullptr, MCA_ERR_INVALID, "bad domain");
   if (!std::isfinite(d.temperature) || d.temperature < 0.0f)
     return fail(nullptr, MCA_ERR_INVALID, "temperature %g: must be finite and >= 0", d.temperature);
+  if (d.layer_stretch < 0)
+    return fail(nullptr, MCA_ERR_INVALID, "layer_stretch = %d < 0", d.layer_stretch);
 
   mca_handle* h = new (std::nothrow) mca_handle();
   if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
@@ -1173,6 +1178,10 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
     return fail(nullptr, MCA_ERR_INVALID, "bad domain");
   if (!std::isfinite(d.temperature) || d.temperature < 0.0f)
     return fail(nullptr, MCA_ERR_INVALID, "temperature %g: must be finite and >= 0", d.temperature);
+  if (d.layer_stretch < 0)
+    return fail(nullptr, MCA_ERR_INVALID, "layer_stretch = %d < 0", d.layer_stretch);
+  if (d.layer_stretch > 0)
+    return fail(nullptr, MCA_ERR_UNSUPPORTED, "the current-layer schedule is for MLPs");
   mca_handle* h = new (std::nothrow) mca_handle();
   if (!h) return fail(nullptr, MCA_ERR_OOM, "host allocation failed");
   auto bail = [&](mca_status st) {

@@ -14,6 +14,15 @@ __host__ __device__ __forceinline__ size_t deep_tc_image_index(int r, int k) {
   return (size_t)(k >> 4) * 8192 + (size_t)((k >> 2) & 3) * 1024 + (size_t)r * 4 + (size_t)(k & 3);
 }
 
+// Flat index of trial tau's weight from its first Philox word r0 (Eq. 1): uniform over all
+// weights, or, under the current-layer schedule, uniform inside its stretch's layer.
+__device__ __forceinline__ unsigned int deep_trial_index(const DeepArgs& a, unsigned long long tau,
+                                                         uint32_t r0) {
+  if (a.stretch <= 0) return (unsigned int)(((unsigned long long)r0 * a.off[a.L]) >> 32);
+  const int l = stretch_layer(a.seed, tau / (unsigned long long)a.stretch, a.L);
+  return (unsigned int)(a.off[l] + (((unsigned long long)r0 * (a.off[l + 1] - a.off[l])) >> 32));
+}
+
 // Layer of candidate k's weight (proposal only, no memory reads besides the layer offsets).
 __device__ __forceinline__ int deep_candidate_layer(const DeepArgs& a, int k) {
   unsigned int idx;
@@ -21,7 +30,7 @@ __device__ __forceinline__ int deep_candidate_layer(const DeepArgs& a, int k) {
     idx = a.ex_idx[k];
   } else {
     const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
-    idx = (unsigned int)(((unsigned long long)w.x * a.off[a.L]) >> 32);
+    idx = deep_trial_index(a, a.tau + (unsigned long long)k, w.x);
   }
   int l = 0;
   while (l + 1 < a.L && (unsigned long long)idx >= a.off[l + 1]) ++l;
@@ -33,13 +42,12 @@ __device__ __forceinline__ DeepCand deep_candidate(const DeepArgs& a, int k) {
   uint32_t r1 = 0u;
   const bool ex = a.n_explicit > 0;
   float exv = 0.0f;
-  const unsigned long long P = a.off[a.L];
   if (ex) {
     idx = a.ex_idx[k];
     exv = a.ex_new[k];
   } else {
     const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
-    idx = (unsigned int)(((unsigned long long)w.x * P) >> 32);
+    idx = deep_trial_index(a, a.tau + (unsigned long long)k, w.x);
     r1 = w.y;
   }
   int l = 0;

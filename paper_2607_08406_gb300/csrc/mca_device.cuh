@@ -51,6 +51,15 @@ __device__ __forceinline__ bool accept_change(float d, int strict, int metro, ui
   return strict ? (d < th) : (d <= th);
 }
 
+// Layer of stretch s under the current-layer schedule (Section 2.1: a layer chosen at random, many
+// mutations inside it, then the next random layer): uniform over nl layers, from the first word of
+// Philox4x32-10 at counter (s_lo, s_hi, 1, 0) -- apart from every trial's counter (tau, 0, 0).
+__device__ __forceinline__ int stretch_layer(uint64_t seed, uint64_t s, int nl) {
+  const uint4 w = philox4x32_10(make_uint4((uint32_t)s, (uint32_t)(s >> 32), 1u, 0u),
+                                make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+  return (int)(((unsigned long long)w.x * (unsigned int)nl) >> 32);
+}
+
 // u = (r >> 8) * 2^-24: exact, in [0, 1)
 __device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >> 8) * 0x1p-24f; }
 

@@ -85,6 +85,7 @@ struct Mlp2Args {
   int strict;
   int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
   double msc;
+  int stretch;               // > 0: current-layer schedule, trials per stretch; 0: uniform index
   unsigned long long seed, tau0, n_trials;
   int K;
   int fixed_K;
@@ -150,6 +151,7 @@ struct DeepArgs {
   int strict;
   int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
   double msc;
+  int stretch;               // > 0: current-layer schedule, trials per stretch; 0: uniform index
   unsigned long long seed, tau;
   int Kb;
   float* partial;            // [kKmax x ntiles]
@@ -210,6 +212,7 @@ struct TfmArgs {
   int strict;
   int metro;                 // 1: Metropolis rule (Eq. 7) with msc = N / beta; 0: greedy (Eq. 6)
   double msc;
+  int stretch;               // > 0: current-layer schedule, trials per stretch; 0: uniform index
   unsigned long long seed, tau;
   int Kb;
   int mode;

@@ -32,7 +32,8 @@ class mca_layer(Structure):
 
 class mca_domain(Structure):
     _fields_ = [("op", c_int32), ("lo", c_float), ("hi", c_float), ("delta", c_float),
-                ("bound", c_float), ("strict", c_int32), ("temperature", c_float)]
+                ("bound", c_float), ("strict", c_int32), ("temperature", c_float),
+                ("layer_stretch", c_int32)]
 
 
 class mca_dataset(Structure):
@@ -156,7 +157,8 @@ def _domain(d) -> mca_domain:
     if not beta > 0.0:
         raise ValueError(f"beta = {beta}: the selection intensity must be > 0 (inf: greedy rule)")
     return mca_domain(OP[d.op], d.lo, d.hi, d.delta, d.bound, int(bool(d.strict)),
-                      0.0 if beta == float("inf") else 1.0 / beta)
+                      0.0 if beta == float("inf") else 1.0 / beta,
+                      int(getattr(d, "layer_stretch", 0)))
 
 
 class Handle:

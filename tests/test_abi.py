@@ -111,6 +111,19 @@ def test_invalid_specs_rejected_without_gpu(lib):
         rc = lib.mca_create(L, n, 0, ctypes.byref(d), ctypes.byref(ds), wl.init.ctypes.data,
                             None, ctypes.byref(h))
         assert rc == mca.MCA_ERR_INVALID and b"temperature" in lib.mca_last_error(None)
+    # a negative current-layer stretch
+    d = mca.mca_domain(0, -1.0, 1.0, 0.01, 0.0, 0, 0.0, -1)
+    rc = lib.mca_create(L, n, 0, ctypes.byref(d), ctypes.byref(ds), wl.init.ctypes.data, None,
+                        ctypes.byref(h))
+    assert rc == mca.MCA_ERR_INVALID and b"layer_stretch" in lib.mca_last_error(None)
+    # the current-layer schedule is for MLPs: a Transformer handle refuses it
+    sp = W.TfmSpec(vocab=17, ctx=8, d_model=16, n_layer=1, n_head=2, d_ff=32)
+    tok = np.zeros((4, 9), np.int32)
+    init = np.zeros(sp.n_params, np.float32)
+    d = mca.mca_domain(0, -1.0, 1.0, 0.01, 0.0, 0, 0.0, 10)
+    rc = lib.mca_create_transformer(ctypes.byref(mca._tfm_spec(sp)), ctypes.byref(d),
+                                    tok.ctypes.data, 4, init.ctypes.data, None, ctypes.byref(h))
+    assert rc == mca.MCA_ERR_UNSUPPORTED and h.value is None
     # NULL handle calls
     assert lib.mca_run(None, 1, 0, None) == mca.MCA_ERR_INVALID
     lib.mca_destroy(None)
