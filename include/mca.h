@@ -297,6 +297,16 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
 mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t* flat_idx,
                                        const float* new_w, size_t n, double* dS);
 
+/* Failure-detection self-test (the library's own check; the paper has no counterpart). Runs the
+ * bounded grid barrier of the trial loop in one CTA that waits for a second CTA which is never
+ * launched: a peer that never arrives. The wait must give up after its 2 s limit, record
+ * MCA_ERR_TIMEOUT and let the kernel return, leaving the CUDA context usable. *status receives the
+ * status the kernel recorded (MCA_ERR_TIMEOUT when the limit works); *waited_ms (nullable) the
+ * host wall time of the kernel. Runs on the legacy default stream and allocates 256 bytes of
+ * device memory for its barrier. Returns MCA_OK when the kernel ran and returned, MCA_ERR_CUDA
+ * otherwise. */
+mca_status mca_selftest_wait_timeout(int32_t* status, double* waited_ms);
+
 void mca_destroy(mca_handle* h);
 
 /* Message of the last failed call on h (h may be NULL: then the last failed mca_create or

@@ -1,6 +1,7 @@
 // C ABI of the MCA trial loop (include/mca.h): argument checks, device memory layout, the
 // creation-time full forward pass, and the host side of mca_run.
 #include <algorithm>
+#include <chrono>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -10,6 +11,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "mca_device.cuh"
 #include "mca_internal.h"
 #include "mca_tc_layout.h"
@@ -18,6 +21,16 @@ using mca::DevState;
 using mca::GridBarrier;
 
 namespace {
+
+// NVTX range for profilers (nsys, ncu --nvtx): creation, each mca_run call, each host-driven batch
+// of the deep and Transformer paths, each persistent trial-loop segment, each resync. Without an
+// attached tool a push / pop is a check of one function pointer.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 thread_local std::string g_create_err;
 
@@ -198,6 +211,14 @@ long long host_nnz(const float* x, size_t n) {
   long long c = 0;
   for (size_t i = 0; i < n; ++i) c += x[i] != 0.0f;
   return c;
+}
+
+// One CTA waits in the trial loop's grid barrier for a second CTA that is never launched
+// (mca_selftest_wait_timeout): the bounded wait must give up and record MCA_ERR_TIMEOUT in *err.
+__global__ void wait_selftest_kernel(GridBarrier* bar, int* err) {
+  __shared__ int s_flag;
+  unsigned int gen = 0u;
+  mca::grid_sync(bar, 2u, gen, err, &s_flag);
 }
 
 __global__ void count_nonzero_kernel(const float* __restrict__ p, size_t n,
@@ -398,6 +419,7 @@ mca::DeepArgs deep_args(mca_handle* h) {
 mca::TfmArgs tfm_args(mca_handle* h);
 
 mca_status resync(mca_handle* h) {
+  NvtxRange nv("mca resync");
   if (h->tfm) {
     const mca::TfmArgs a = tfm_args(h);
     if (a.tc) {
@@ -681,6 +703,7 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
 mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
                       const mca_domain* dom, const mca_dataset* data, const float* init_params,
                       const mca_options* opt, mca_handle** out) {
+  NvtxRange nv("mca_create");
   if (!out) return fail(nullptr, MCA_ERR_INVALID, "out is NULL");
   *out = nullptr;
   std::vector<mca_layer> ls;
@@ -883,6 +906,7 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
 
 mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stats* stats) {
   if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  NvtxRange nv_run("mca_run");
   if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
   uint64_t remaining = n_trials;
   if (h->deep || h->tfm) {
@@ -893,6 +917,7 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     ta.seed = seed;
     const uint64_t R = (uint64_t)h->opt.resync_period;
     while (remaining > 0) {
+      NvtxRange nv_batch(h->tfm ? "mca batch (transformer)" : "mca batch (deep)");
       const int Kw = h->opt.fixed_K ? h->opt.K
                                     : mca::batch_width(h->rate_acc, h->rate_trials,
                                                        mca::kWidthDeep, h->opt.K);
@@ -949,6 +974,7 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     }
   }
   while (remaining > 0) {
+    NvtxRange nv_seg("mca trial-loop segment");
     uint64_t seg = remaining;
     const uint64_t R = (uint64_t)h->opt.resync_period;
     if (R > 0) seg = std::min<uint64_t>(seg, R - h->tau % R);
@@ -1162,6 +1188,7 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
 mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
                                   const int32_t* tokens, int64_t n_seq, const float* init_params,
                                   const mca_options* opt, mca_handle** out) {
+  NvtxRange nv("mca_create_transformer");
   if (!out) return fail(nullptr, MCA_ERR_INVALID, "out is NULL");
   *out = nullptr;
   mca_status rc = tfm_check(spec, n_seq);
@@ -1267,6 +1294,33 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   if (rc != MCA_OK) return bail(rc);
   if (!std::isfinite(ds.S)) return bail(fail(h, MCA_ERR_NUMERIC, "initial loss is not finite"));
   *out = h;
+  return MCA_OK;
+}
+
+mca_status mca_selftest_wait_timeout(int32_t* status, double* waited_ms) {
+  if (!status) return fail(nullptr, MCA_ERR_INVALID, "status is NULL");
+  NvtxRange nv("mca wait self-test");
+  void* mem = nullptr;
+  cudaError_t e = cudaMalloc(&mem, 256);
+  if (e != cudaSuccess) return fail(nullptr, MCA_ERR_CUDA, "%s", cudaGetErrorString(e));
+  GridBarrier* bar = static_cast<GridBarrier*>(mem);
+  int* err = reinterpret_cast<int*>(static_cast<char*>(mem) + 64);
+  e = cudaMemset(mem, 0, 256);
+  const auto t0 = std::chrono::steady_clock::now();
+  if (e == cudaSuccess) {
+    wait_selftest_kernel<<<1, 32, 0, 0>>>(bar, err);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(0);
+  const double ms =
+      std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+  int h_err = -1;
+  if (e == cudaSuccess) e = cudaMemcpy(&h_err, err, sizeof(int), cudaMemcpyDeviceToHost);
+  const cudaError_t ef = cudaFree(mem);
+  if (e == cudaSuccess) e = ef;
+  if (e != cudaSuccess) return fail(nullptr, MCA_ERR_CUDA, "%s", cudaGetErrorString(e));
+  *status = h_err;
+  if (waited_ms) *waited_ms = ms;
   return MCA_OK;
 }
 

@@ -99,6 +99,7 @@ SIGNATURES = {
     "mca_get_stats": (c_int32, [c_void_p, POINTER(mca_run_stats)]),
     "mca_eval_candidates": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "mca_eval_candidates_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "mca_selftest_wait_timeout": (c_int32, [POINTER(c_int32), POINTER(c_double)]),
     "mca_destroy": (None, [c_void_p]),
     "mca_last_error": (c_char_p, [c_void_p]),
 }
@@ -336,6 +337,14 @@ def mca_eval_candidates_noalloc(h: Handle, flat_idx, new_w, dS):
     _check(load_library().mca_eval_candidates_noalloc(h.ptr, flat_idx.data_ptr(), new_w.data_ptr(),
                                                       n, dS.data_ptr()), h.ptr)
     return dS
+
+
+def mca_selftest_wait_timeout():
+    """(status recorded by the kernel, host milliseconds): the trial loop's bounded grid barrier
+    waiting for a peer CTA that never arrives must give up with MCA_ERR_TIMEOUT."""
+    st, ms = ctypes.c_int32(-1), ctypes.c_double(0.0)
+    _check(load_library().mca_selftest_wait_timeout(ctypes.byref(st), ctypes.byref(ms)))
+    return st.value, ms.value
 
 
 def mca_destroy(h: Handle):
