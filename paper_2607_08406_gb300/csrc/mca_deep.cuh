@@ -16,8 +16,9 @@ __host__ __device__ __forceinline__ size_t deep_tc_image_index(int r, int k) {
 
 // Flat index of trial tau's weight from its first Philox word r0 (Eq. 1): uniform over all
 // weights, or, under the current-layer schedule, uniform inside its stretch's layer.
-__device__ __forceinline__ unsigned int deep_trial_index(const DeepArgs& a, unsigned long long tau,
-                                                         uint32_t r0) {
+__host__ __device__ __forceinline__ unsigned int deep_trial_index(const DeepArgs& a,
+                                                                  unsigned long long tau,
+                                                                  uint32_t r0) {
   if (a.stretch <= 0) return (unsigned int)(((unsigned long long)r0 * a.off[a.L]) >> 32);
   const int l = stretch_layer(a.seed, tau / (unsigned long long)a.stretch, a.L);
   return (unsigned int)(a.off[l] + (((unsigned long long)r0 * (a.off[l + 1] - a.off[l])) >> 32));

@@ -13,22 +13,32 @@ namespace mca {
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11, Section 3.2): ten rounds of two 32x32->64
 // multiplies and xors over a 128-bit counter, the 64-bit key bumped by the Weyl constants between
 // rounds. Counter = (tau_lo, tau_hi, 0, 0), key = (seed_lo, seed_hi).
+// The proposal-stream helpers below are also compiled for the host, so that a CPU test can check
+// their arithmetic against the oracle.
 // ------------------------------------------------------------------------------------------------
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+__host__ __device__ __forceinline__ uint32_t mulhi32(uint32_t a, uint32_t b) {
+#ifdef __CUDA_ARCH__
+  return __umulhi(a, b);
+#else
+  return (uint32_t)(((uint64_t)a * b) >> 32);
+#endif
+}
+
+__host__ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
     if (r) {
       k.x += 0x9E3779B9u;
       k.y += 0xBB67AE85u;
     }
-    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
-    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
+    const uint32_t hi0 = mulhi32(0xD2511F53u, c.x), lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = mulhi32(0xCD9E8D57u, c.z), lo1 = 0xCD9E8D57u * c.z;
     c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
   }
   return c;
 }
 
-__device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
+__host__ __device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
   return philox4x32_10(make_uint4((uint32_t)tau, (uint32_t)(tau >> 32), 0u, 0u),
                        make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
 }
@@ -38,15 +48,16 @@ __device__ __forceinline__ uint4 trial_words(uint64_t seed, uint64_t tau) {
 // u = (r3 + 1/2) 2^-32, r3 the fourth Philox word of its counter, that is u < exp(-beta dS / N),
 // i.e. dS <= -(N / beta) ln u. msc = N / beta > 0. Evaluated in fp64 (once per candidate and
 // batch) and rounded to the fp32 of the candidate's dS.
-__device__ __forceinline__ float metropolis_theta(uint64_t seed, uint64_t tau, double msc) {
+__host__ __device__ __forceinline__ float metropolis_theta(uint64_t seed, uint64_t tau,
+                                                             double msc) {
   const uint32_t r3 = trial_words(seed, tau).w;
   const double u = ((double)r3 + 0.5) * 0x1p-32;
   return (float)(-msc * log(u));
 }
 
 // Acceptance of a candidate with loss-sum change d (Eq. 6, or Eq. 7 when metro != 0).
-__device__ __forceinline__ bool accept_change(float d, int strict, int metro, uint64_t seed,
-                                              uint64_t tau, double msc) {
+__host__ __device__ __forceinline__ bool accept_change(float d, int strict, int metro,
+                                                       uint64_t seed, uint64_t tau, double msc) {
   const float th = metro ? metropolis_theta(seed, tau, msc) : 0.0f;
   return strict ? (d < th) : (d <= th);
 }
@@ -54,10 +65,23 @@ __device__ __forceinline__ bool accept_change(float d, int strict, int metro, ui
 // Layer of stretch s under the current-layer schedule (Section 2.1: a layer chosen at random, many
 // mutations inside it, then the next random layer): uniform over nl layers, from the first word of
 // Philox4x32-10 at counter (s_lo, s_hi, 1, 0) -- apart from every trial's counter (tau, 0, 0).
-__device__ __forceinline__ int stretch_layer(uint64_t seed, uint64_t s, int nl) {
+__host__ __device__ __forceinline__ int stretch_layer(uint64_t seed, uint64_t s, int nl) {
   const uint4 w = philox4x32_10(make_uint4((uint32_t)s, (uint32_t)(s >> 32), 1u, 0u),
                                 make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
   return (int)(((unsigned long long)w.x * (unsigned int)nl) >> 32);
+}
+
+// Flat index of trial tau's weight in a two-layer net (P weights, the first P1 in W1) from the
+// trial's first Philox word r0 (Eq. 1): uniform over the P weights, or, under the current-layer
+// schedule (stretch = M > 0), uniform inside the stretch's layer.
+__host__ __device__ __forceinline__ unsigned int mlp2_trial_index(unsigned long long P,
+                                                                  unsigned long long P1,
+                                                                  uint64_t seed, uint64_t tau,
+                                                                  uint32_t r0, int stretch) {
+  if (stretch <= 0) return (unsigned int)(((unsigned long long)r0 * P) >> 32);
+  const int l = stretch_layer(seed, tau / (unsigned long long)stretch, 2);
+  const unsigned long long lo = l ? P1 : 0ull, n = l ? P - P1 : P1;
+  return (unsigned int)(lo + (((unsigned long long)r0 * n) >> 32));
 }
 
 // u = (r >> 8) * 2^-24: exact, in [0, 1)

@@ -43,16 +43,6 @@ struct Cand {
   int sub0, nsub;            // this CTA's sub-chunks
 };
 
-// Flat index of trial tau's weight from its first Philox word r0 (Eq. 1): uniform over the P
-// weights, or, under the current-layer schedule, uniform inside its stretch's layer (W1 or W2).
-__device__ __forceinline__ unsigned int mlp2_trial_index(const Mlp2Args& a, unsigned long long tau,
-                                                         uint32_t r0) {
-  if (a.stretch <= 0) return (unsigned int)(((unsigned long long)r0 * a.P) >> 32);
-  const int l = stretch_layer(a.seed, tau / (unsigned long long)a.stretch, 2);
-  const unsigned long long lo = l ? a.P1 : 0ull, n = l ? a.P - a.P1 : a.P1;
-  return (unsigned int)(lo + (((unsigned long long)r0 * n) >> 32));
-}
-
 __device__ __forceinline__ void fill_candidate(const Mlp2Args& a, unsigned int idx, uint32_t r1,
                                                bool explicit_value, float ex_new, int r, int s0,
                                                int s1, Cand& c) {
@@ -318,7 +308,8 @@ __global__ void __launch_bounds__(kLoopThreads, 1) mlp2_trial_loop(Mlp2Args a) {
         fill_candidate(a, a.ex_idx[k], 0u, true, a.ex_new[k], r, s0, s1, c);
       } else {
         const uint4 w = trial_words(a.seed, tau + (unsigned long long)k);
-        const unsigned int idx = mlp2_trial_index(a, tau + (unsigned long long)k, w.x);
+        const unsigned int idx =
+            mlp2_trial_index(a.P, a.P1, a.seed, tau + (unsigned long long)k, w.x, a.stretch);
         fill_candidate(a, idx, w.y, false, 0.0f, r, s0, s1, c);
       }
       if (c.layer == 0 && c.gcnt > 0) {
@@ -749,7 +740,7 @@ __device__ __forceinline__ void prepare_slot(const Mlp2Args& a, WSlot* slots, fl
   const int lane = threadIdx.x & 31;
   if (lane == 0) {
     const uint4 w = trial_words(a.seed, t);
-    const unsigned int idx = mlp2_trial_index(a, t, w.x);
+    const unsigned int idx = mlp2_trial_index(a.P, a.P1, a.seed, t, w.x, a.stretch);
     Cand c;
     fill_candidate(a, idx, w.y, false, 0.0f, r, s0, s1, c);
     slots[sl].c = c;
