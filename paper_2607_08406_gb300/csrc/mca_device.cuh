@@ -25,7 +25,9 @@ __host__ __device__ __forceinline__ uint32_t mulhi32(uint32_t a, uint32_t b) {
 }
 
 __host__ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#ifdef __CUDA_ARCH__
 #pragma unroll
+#endif
   for (int r = 0; r < 10; ++r) {
     if (r) {
       k.x += 0x9E3779B9u;

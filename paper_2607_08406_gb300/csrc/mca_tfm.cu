@@ -23,7 +23,7 @@
 
 namespace mca {
 
-__host__ __device__ inline int tfm_region_floats(int T, int d, int dh, int V) {
+__host__ __device__ inline int tfm_region_floats(int T, int /*d*/, int dh, int V) {
   const int att = T * dh + T * (dh + 1) + T * dh + T * T;
   const int ffn = T * kTfmFC;
   const int head = T * V;
