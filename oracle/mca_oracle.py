@@ -15,6 +15,9 @@ Networks", Section 2 Eq. 1 and Section 3.1 Eq. 6):
                                              a finite selection intensity beta, as a per-trial
                                              threshold S' - S <= theta_tau, metropolis_threshold)
 
+Multi-parameter channel mutations (Section 2.3) have their own loop, ``run_channel``: every weight on
+one input-to-output path changes at once and a full forward pass decides.
+
 Two evaluation modes, which must agree (the invariant the incremental GPU path relies on):
 
 * ``run_full``: a full forward pass of all N samples after every mutation -- the definition.
@@ -51,6 +54,7 @@ __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
     "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
     "candidate_dS_two_layer", "metropolis_threshold", "stretch_layer", "proposal_index",
+    "channel_words", "propose_channel", "run_channel",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -505,3 +509,80 @@ def candidate_dS_two_layer(params: Params, XT: np.ndarray, y: np.ndarray, loss: 
         Z2n[o] += delta * a
     ell_new = loss_per_sample(loss, act_fn(L2.act, Z2n, L2.act_param), y)
     return float((ell_new - ell).sum())
+
+
+# ------------------------------------------------------------------------------------------------
+# Multi-parameter channel mutations (Section 2.3). A channel is a path from one input node through
+# one node of every hidden layer to one output node; a mutation changes the one weight of every
+# layer that lies on it, either redrawing each with He-normalised amplitude or setting all to zero
+# (the Dropout-like scheme), and is kept iff the loss does not increase. fp32 layers only.
+# ------------------------------------------------------------------------------------------------
+
+def channel_words(seed: int, tau: int, n: int) -> np.ndarray:
+    """n Philox words for trial tau's channel: counters (tau_lo, tau_hi, 2, q), q = 0, 1, ..., four
+    words each -- apart from the trial's own counter (tau, 0, 0, 0) and the schedule's (s, 0, 1, 0)."""
+    q = np.arange((n + 3) // 4, dtype=np.uint64)
+    t = np.uint64(tau)
+    ctr = np.stack([np.full_like(q, t & _M32), np.full_like(q, t >> _S32),
+                    np.full_like(q, 2), q], axis=-1)
+    s = np.uint64(seed)
+    key = np.broadcast_to(np.array([s & _M32, s >> _S32], dtype=np.uint64), ctr.shape[:-1] + (2,))
+    return philox4x32_10(ctr, key).reshape(-1)[:n]
+
+
+def propose_channel(seed: int, tau: int, params: Params, scheme: str):
+    """The channel of trial tau and its new weights: a list of (layer m, row, col, old, new) with
+    W_m[c_{m+1}, c_m] for m = 0 .. L-1. Nodes: c_m = floor(v_m n_m / 2^32) over the L + 1 node
+    counts (inputs, every hidden width, outputs), v_m the channel words. scheme "he": the new
+    weight of layer m is a_m (2 u_m - 1) in fp32, u_m = (v_{L+1+m} >> 8) 2^-24 and
+    a_m = fp32(sqrt(6 / fan_in_m)) (He's uniform amplitude); scheme "zero": 0."""
+    layers = params.layers
+    L = len(layers)
+    sizes = [layers[0].n_in] + [ly.n_out for ly in layers]
+    v = channel_words(seed, tau, 2 * L + 1)
+    nodes = [int((int(v[m]) * sizes[m]) >> 32) for m in range(L + 1)]
+    f32 = np.float32
+    out = []
+    for m, ly in enumerate(layers):
+        if ly.wkind != "fp32":
+            raise ValueError("channel mutations take fp32 layers")
+        row, col = nodes[m + 1], nodes[m]
+        old = f32(params.vals[m][row, col])
+        if scheme == "he":
+            a = f32(np.sqrt(6.0 / ly.n_in))
+            u = f32(int(v[L + 1 + m]) >> 8) * f32(2.0 ** -24)
+            new = f32(a * f32(f32(f32(2.0) * u) - f32(1.0)))
+        elif scheme == "zero":
+            new = f32(0.0)
+        else:
+            raise ValueError(scheme)
+        out.append((m, row, col, float(old), float(new)))
+    return out
+
+
+def run_channel(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials: int, seed: int,
+                scheme: str, strict: bool = False, beta: float = float("inf"), tau0: int = 0,
+                params: Optional[Params] = None):
+    """Channel-mutation trial loop, by definition: apply every weight of the channel, run a full
+    forward pass, keep iff dS <= theta (Eq. 6; Eq. 7 for a finite beta), else restore every weight.
+    Returns (list of (tau, channel, S before, dS, accepted), final Params, final S)."""
+    XT = np.ascontiguousarray(np.asarray(X, dtype=np.float64).T)
+    y = np.asarray(y)
+    params = Params(layers, init) if params is None else params
+    S = total_loss(params, XT, y, loss)
+    rows = []
+    for t in range(n_trials):
+        tau = tau0 + t
+        ch = propose_channel(seed, tau, params, scheme)
+        for m, r, c, old, new in ch:
+            params.vals[m][r, c] = np.float32(new)
+        S_new = total_loss(params, XT, y, loss)
+        dS = S_new - S
+        acc = _decide(dS, strict, float(metropolis_threshold(seed, tau, beta, XT.shape[1])))
+        rows.append((tau, ch, S, dS, acc))
+        if acc:
+            S = S_new
+        else:
+            for m, r, c, old, new in reversed(ch):
+                params.vals[m][r, c] = np.float32(old)
+    return rows, params, S
