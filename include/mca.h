@@ -297,6 +297,25 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
 mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t* flat_idx,
                                        const float* new_w, size_t n, double* dS);
 
+/* Multi-parameter channel mutations (Section 2.3) on an MLP handle whose layers are all
+ * MCA_W_FP32. Trial tau draws a channel -- one node of every layer, input c_0, hidden c_1 ..
+ * c_{L-1}, output c_L, each uniform: c_m = floor(v_m * n_m / 2^32) -- and changes the L weights
+ * W_m[c_{m+1}][c_m] at once: scheme MCA_CHANNEL_HE redraws weight m as a_m * (2u - 1) in fp32,
+ * a_m = fp32(sqrt(6 / n_in of layer m)) (He's uniform amplitude), u = (v_{L+1+m} >> 8) * 2^-24;
+ * MCA_CHANNEL_ZERO sets them to 0 (the Dropout-like scheme). The words v_0, v_1, ... are those of
+ * Philox4x32-10(key = seed, counter = (tau_lo, tau_hi, 2, q)), q = 0, 1, ..., four per counter.
+ * Every layer changes, so each trial recomputes every cached field with the full forward pass
+ * (the kernels of creation and mca_resync), then keeps the channel iff dS <= theta (Eq. 6, or Eq.
+ * 7 with the domain's temperature; forced decisions apply); a rejected channel is restored and
+ * the fields recomputed again. Trials run one at a time (no speculation) from the handle's trial
+ * counter tau, which advances by n_trials; mca_run_stats and the trace count single-weight trials
+ * only. accepted [n_trials] (uint8, 1 kept) and dS [n_trials] (S' - S) are nullable HOST arrays.
+ * Errors: INVALID (NULL handle, unknown scheme), UNSUPPORTED (a Transformer handle or a ternary /
+ * masked layer), NUMERIC (a non-finite loss change), CUDA. */
+typedef enum { MCA_CHANNEL_HE = 0, MCA_CHANNEL_ZERO = 1 } mca_channel_scheme;
+mca_status mca_run_channels(mca_handle* h, uint64_t n_trials, uint64_t seed, int32_t scheme,
+                            uint8_t* accepted, double* dS);
+
 /* Failure-detection self-test (the library's own check; the paper has no counterpart). Runs the
  * bounded grid barrier of the trial loop in one CTA that waits for a second CTA which is never
  * launched: a peer that never arrives. The wait must give up after its 2 s limit, record

@@ -1297,6 +1297,104 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   return MCA_OK;
 }
 
+mca_status mca_run_channels(mca_handle* h, uint64_t n_trials, uint64_t seed, int32_t scheme,
+                            uint8_t* accepted, double* dS) {
+  if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (scheme != MCA_CHANNEL_HE && scheme != MCA_CHANNEL_ZERO)
+    return fail(h, MCA_ERR_INVALID, "unknown channel scheme %d", scheme);
+  if (h->tfm) return fail(h, MCA_ERR_UNSUPPORTED, "channel mutations are for MLPs");
+  const int L = (int)h->layers.size();
+  for (int m = 0; m < L; ++m)
+    if (h->layers[m].wkind != MCA_W_FP32)
+      return fail(h, MCA_ERR_UNSUPPORTED, "layer %d is not fp32", m);
+  NvtxRange nv("mca_run_channels");
+  // forced decisions, as a host copy of the device lists
+  std::vector<unsigned long long> ftau(h->nforce);
+  std::vector<unsigned char> facc(h->nforce);
+  if (h->nforce > 0) {
+    CUDA_TRY(h, cudaMemcpyAsync(ftau.data(), h->ftau, sizeof(unsigned long long) * h->nforce,
+                                cudaMemcpyDeviceToHost, h->stream));
+    CUDA_TRY(h, cudaMemcpyAsync(facc.data(), h->facc, h->nforce, cudaMemcpyDeviceToHost,
+                                h->stream));
+    CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  }
+  std::vector<int> node(L + 1);
+  std::vector<float> oldw(L), neww(L);
+  std::vector<float*> at(L);
+  std::vector<uint32_t> v(2 * L + 4);
+  DevState ds;
+  mca_status rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  double S = ds.S;
+  for (uint64_t t = 0; t < n_trials; ++t) {
+    const uint64_t tau = h->tau;
+    for (int q = 0; 4 * q < 2 * L + 1; ++q) {          // channel words: counters (tau, 2, q)
+      const uint4 w = mca::philox4x32_10(
+          make_uint4((uint32_t)tau, (uint32_t)(tau >> 32), 2u, (uint32_t)q),
+          make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+      v[4 * q] = w.x;
+      v[4 * q + 1] = w.y;
+      v[4 * q + 2] = w.z;
+      v[4 * q + 3] = w.w;
+    }
+    for (int m = 0; m <= L; ++m) {
+      const unsigned long long n_m =
+          m == 0 ? (unsigned long long)h->layers[0].n_in : (unsigned long long)h->layers[m - 1].n_out;
+      node[m] = (int)(((unsigned long long)v[m] * n_m) >> 32);
+    }
+    for (int m = 0; m < L; ++m) {
+      const mca_layer& ly = h->layers[m];
+      at[m] = h->w_eff[m] + (size_t)node[m + 1] * ly.n_in + node[m];
+      if (scheme == MCA_CHANNEL_HE) {
+        const float a = (float)std::sqrt(6.0 / (double)ly.n_in);
+        const float u = (float)(v[L + 1 + m] >> 8) * 0x1p-24f;
+        const float r = 2.0f * u;                       // exact
+        neww[m] = a * (r - 1.0f);
+      } else {
+        neww[m] = 0.0f;
+      }
+      CUDA_TRY(h, cudaMemcpyAsync(&oldw[m], at[m], sizeof(float), cudaMemcpyDeviceToHost,
+                                  h->stream));
+    }
+    CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+    for (int m = 0; m < L; ++m)
+      CUDA_TRY(h, cudaMemcpyAsync(at[m], &neww[m], sizeof(float), cudaMemcpyHostToDevice,
+                                  h->stream));
+    rc = resync(h);
+    if (rc != MCA_OK) return rc;
+    rc = read_state(h, &ds);
+    if (rc != MCA_OK) return rc;
+    const double d = ds.S - S;
+    if (!std::isfinite(d)) {
+      h->broken = true;
+      return fail(h, MCA_ERR_NUMERIC, "non-finite loss change");
+    }
+    bool acc;
+    const auto it = std::lower_bound(ftau.begin(), ftau.end(), (unsigned long long)tau);
+    if (it != ftau.end() && *it == tau) {
+      acc = facc[it - ftau.begin()] != 0;
+    } else {
+      acc = mca::accept_change((float)d, h->dom.strict, h->dom.temperature > 0.0f ? 1 : 0, seed,
+                               tau, (double)h->N * (double)h->dom.temperature);
+    }
+    if (accepted) accepted[t] = acc ? 1 : 0;
+    if (dS) dS[t] = d;
+    if (acc) {
+      S = ds.S;
+    } else {
+      for (int m = L - 1; m >= 0; --m)
+        CUDA_TRY(h, cudaMemcpyAsync(at[m], &oldw[m], sizeof(float), cudaMemcpyHostToDevice,
+                                    h->stream));
+      rc = resync(h);
+      if (rc != MCA_OK) return rc;
+      CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+    }
+    h->tau = tau + 1;
+  }
+  return MCA_OK;
+}
+
 mca_status mca_selftest_wait_timeout(int32_t* status, double* waited_ms) {
   if (!status) return fail(nullptr, MCA_ERR_INVALID, "status is NULL");
   NvtxRange nv("mca wait self-test");

@@ -99,6 +99,7 @@ SIGNATURES = {
     "mca_get_stats": (c_int32, [c_void_p, POINTER(mca_run_stats)]),
     "mca_eval_candidates": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "mca_eval_candidates_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "mca_run_channels": (c_int32, [c_void_p, c_uint64, c_uint64, c_int32, c_void_p, c_void_p]),
     "mca_selftest_wait_timeout": (c_int32, [POINTER(c_int32), POINTER(c_double)]),
     "mca_destroy": (None, [c_void_p]),
     "mca_last_error": (c_char_p, [c_void_p]),
@@ -337,6 +338,18 @@ def mca_eval_candidates_noalloc(h: Handle, flat_idx, new_w, dS):
     _check(load_library().mca_eval_candidates_noalloc(h.ptr, flat_idx.data_ptr(), new_w.data_ptr(),
                                                       n, dS.data_ptr()), h.ptr)
     return dS
+
+
+CHANNEL = {"he": 0, "zero": 1}
+
+
+def mca_run_channels(h: Handle, n_trials: int, seed: int, scheme: str):
+    """Channel-mutation trials (Section 2.3); returns (accepted [n] bool, dS [n] float64)."""
+    acc = np.zeros(n_trials, np.uint8)
+    dS = np.zeros(n_trials, np.float64)
+    _check(load_library().mca_run_channels(h.ptr, n_trials, seed, CHANNEL[scheme],
+                                           acc.ctypes.data, dS.ctypes.data), h.ptr)
+    return acc.astype(bool), dS
 
 
 def mca_selftest_wait_timeout():

@@ -126,6 +126,7 @@ def test_invalid_specs_rejected_without_gpu(lib):
     assert rc == mca.MCA_ERR_UNSUPPORTED and h.value is None
     # NULL handle calls
     assert lib.mca_run(None, 1, 0, None) == mca.MCA_ERR_INVALID
+    assert lib.mca_run_channels(None, 1, 0, 0, None, None) == mca.MCA_ERR_INVALID
     lib.mca_destroy(None)
 
 
