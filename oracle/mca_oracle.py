@@ -54,7 +54,7 @@ __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
     "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
     "candidate_dS_two_layer", "metropolis_threshold", "stretch_layer", "proposal_index",
-    "channel_words", "propose_channel", "run_channel",
+    "channel_words", "propose_channel", "run_channel", "run_batches",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -586,3 +586,25 @@ def run_channel(layers, loss: str, X: np.ndarray, y: np.ndarray, init, n_trials:
             for m, r, c, old, new in reversed(ch):
                 params.vals[m][r, c] = np.float32(old)
     return rows, params, S
+
+
+# ------------------------------------------------------------------------------------------------
+# Mini-batch schedules (Sections 2.2 and 2.5: a batch of 30,000 of the 60,000 samples; a batch size
+# that grows during training). The trials of stretch s = tau // stretch decide on the loss summed
+# over batch s only (Eq. 2 over the batch's samples); the weights and the trial counter carry over
+# from batch to batch. Which samples form each batch is an input (the paper gives no rule).
+# ------------------------------------------------------------------------------------------------
+
+def run_batches(layers, loss: str, X: np.ndarray, y: np.ndarray, init, batches, stretch: int,
+                seed: int, domain, params: Optional[Params] = None):
+    """Trials 0 .. len(batches) * stretch - 1; batch s (an index array into X, y) serves trials
+    s * stretch .. (s + 1) * stretch - 1 through the cached-field mode on its samples. Returns
+    (concatenated trace arrays, final Params, loss sum of the last batch)."""
+    params = Params(layers, init) if params is None else params
+    traces, S = [], 0.0
+    for s, b in enumerate(batches):
+        b = np.asarray(b)
+        tr, params, S = run_incremental(layers, loss, X[b], y[b], None, stretch, seed, domain,
+                                        tau0=s * stretch, params=params)
+        traces.append(tr)
+    return {k: np.concatenate([t[k] for t in traces]) for k in traces[0]}, params, S

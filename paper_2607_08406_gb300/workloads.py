@@ -203,6 +203,15 @@ MLP_WORKLOADS = {
 }
 
 
+def minibatches(n_samples: int, batch: int, n_batches: int, seed: int = 0) -> List[np.ndarray]:
+    """Sample indices of n_batches mini-batches of ``batch`` samples each, every batch drawn without
+    replacement (ascending indices) from the n_samples of a workload; consecutive batches are
+    independent. Input generation only: which batch a trial uses is the caller's schedule."""
+    rng = np.random.default_rng([7, seed, 9])
+    return [np.sort(rng.choice(n_samples, size=batch, replace=False)).astype(np.int64)
+            for _ in range(n_batches)]
+
+
 def make(name: str, **kw) -> MLPWorkload:
     return MLP_WORKLOADS[name](**kw)
 
