@@ -137,6 +137,9 @@ def make_workload(args, rank):
     wl.seed = args.seed + rank
     if args.K:
         wl.K = args.K
+    if args.beta != float("inf") or args.layer_stretch:
+        import dataclasses
+        wl.domain = dataclasses.replace(wl.domain, beta=args.beta, layer_stretch=args.layer_stretch)
     return wl
 
 
@@ -160,6 +163,7 @@ def create_handle(mca, wl, arrays, **kw):
 def cpu_oracle_rate(wl, n_trials, warm=0):
     """A function running oracle trials t0 .. t0+n: the incremental mode (after an untimed cache
     build) for the MLPs, the full-recompute loop for the Transformer."""
+    from oracle import mca_oracle as O
     if is_tfm(wl):
         from oracle import mca_tfm as T
         flat = np.array(wl.init, dtype=np.float32)
@@ -172,12 +176,13 @@ def cpu_oracle_rate(wl, n_trials, warm=0):
                     continue
                 flat[idx] = np.float32(new)
                 S_new = float(T.tfm_seq_losses(wl.spec, flat.astype(np.float64), wl.tokens).sum())
-                if S_new <= state["S"]:
+                theta = float(O.metropolis_threshold(wl.seed, t, wl.domain.beta,
+                                                     wl.tokens.shape[0] * wl.spec.ctx))
+                if S_new - state["S"] <= theta:
                     state["S"] = S_new
                 else:
                     flat[idx] = np.float32(old)
         return tfm_trials
-    from oracle import mca_oracle as O
     XT = np.ascontiguousarray(wl.X.astype(np.float64).T)
     params = O.Params(wl.layers, wl.init)
     cache = O._Cache(params, XT, wl.y, wl.loss)
@@ -190,7 +195,8 @@ def cpu_oracle_rate(wl, n_trials, warm=0):
             if not p.valid:
                 continue
             dS, updates, ell_new = O._candidate(params, cache, XT, wl.y, wl.loss, p)
-            if dS <= 0.0:
+            theta = O._threshold(wl.seed, t, wl.domain, XT.shape[1])
+            if O._decide(dS, wl.domain.strict, theta):
                 O.apply_proposal(params, p)
                 for m, upd in updates:
                     if upd[0] == "row":
@@ -413,6 +419,11 @@ def run_ours(args):
                               if not deep else "no flush: a step's candidates recompute from "
                               "cached fields / residual streams that exceed L2 or are rewritten"),
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+                       "acceptance": ("greedy (Eq. 6)" if wl.domain.beta == float("inf")
+                                      else f"Metropolis (Eq. 7), beta = {wl.domain.beta:g}"),
+                       "proposals": ("uniform over all parameters" if not wl.domain.layer_stretch
+                                     else f"current-layer schedule, {wl.domain.layer_stretch} "
+                                          "trials per layer"),
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
@@ -456,6 +467,10 @@ def main():
     ap.add_argument("--e2e-trials", dest="e2e_trials", type=int, default=0)
     ap.add_argument("--no-e2e", dest="no_e2e", action="store_true")
     ap.add_argument("--no-cpu", dest="no_cpu", action="store_true")
+    ap.add_argument("--beta", type=float, default=float("inf"),
+                    help="Metropolis selection intensity (Eq. 7); inf: the greedy rule")
+    ap.add_argument("--layer-stretch", dest="layer_stretch", type=int, default=0,
+                    help="current-layer schedule: trials per randomly chosen layer (MLPs)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
