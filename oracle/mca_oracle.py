@@ -16,7 +16,9 @@ Networks", Section 2 Eq. 1 and Section 3.1 Eq. 6):
                                              threshold S' - S <= theta_tau, metropolis_threshold)
 
 Multi-parameter channel mutations (Section 2.3) have their own loop, ``run_channel``: every weight on
-one input-to-output path changes at once and a full forward pass decides.
+one input-to-output path changes at once and a full forward pass decides. Mini-batch schedules
+(Sections 2.2 and 2.5) run the cached-field loop on one given batch of samples per stretch of
+trials, ``run_batches``.
 
 Two evaluation modes, which must agree (the invariant the incremental GPU path relies on):
 
