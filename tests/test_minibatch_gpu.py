@@ -47,3 +47,29 @@ def test_minibatch_schedule_through_the_abi(gpu_lib, case):
         h.close()
     assert np.array_equal(flat, params.flat_eff32())
     assert tr["accept"].sum() > 30
+
+
+def test_growing_batch_of_sequences_transformer(gpu_lib):
+    """Section 2.5's adaptive batch size: the Transformer trains on 4, then 8, then 16 sequences
+    (each batch a handle created with the previous batch's weights), against the oracle's
+    full-recompute loop on the same batches."""
+    from oracle import mca_tfm as T
+    import dataclasses
+    spec = W.TfmSpec(vocab=17, ctx=8, d_model=16, n_layer=2, n_head=2, d_ff=32)
+    wl = W.char_transformer(seed=0, batch=16, text_len=20000, spec=spec, n_trials=300, K=8)
+    M = 100
+    flat_o = wl.init.copy()
+    flat = wl.init.copy()
+    for s, B in enumerate((4, 8, 16)):
+        tok = np.ascontiguousarray(wl.tokens[:B])
+        tr, flat_o, S = T.run_full_tfm(spec, tok, flat_o, M, wl.seed, wl.domain, tau0=s * M)
+        sub = dataclasses.replace(wl, tokens=tok, init=flat)
+        h = gpu_lib.create_from_tfm_workload(sub, trace_cap=M)
+        gpu_lib.mca_set_params(h, flat, tau=s * M)
+        gpu_lib.mca_force_decisions(h, *forced_from_oracle(tr))
+        gpu_lib.mca_run(h, M, wl.seed)
+        compare(gpu_lib.mca_get_trace(h, M), tr)
+        flat = gpu_lib.mca_get_params(h, wl.n_params)
+        assert gpu_lib.mca_loss(h) * B * spec.ctx == pytest.approx(S, rel=TIE_REL)
+        h.close()
+    assert np.array_equal(flat, flat_o)
