@@ -56,7 +56,7 @@ __all__ = [
     "philox4x32_10", "draw_words", "propose", "Proposal", "Params", "act_fn", "loss_per_sample",
     "forward", "total_loss", "run_full", "run_incremental", "Trace", "output_fields_blocked",
     "candidate_dS_two_layer", "metropolis_threshold", "stretch_layer", "proposal_index",
-    "channel_words", "propose_channel", "run_channel", "run_batches",
+    "channel_words", "propose_channel", "run_channel", "run_batches", "conditional_dS_two_layer",
 ]
 
 # ------------------------------------------------------------------------------------------------
@@ -610,3 +610,44 @@ def run_batches(layers, loss: str, X: np.ndarray, y: np.ndarray, init, batches, 
                                         tau0=s * stretch, params=params)
         traces.append(tr)
     return {k: np.concatenate([t[k] for t in traces]) for k in traces[0]}, params, S
+
+
+# ------------------------------------------------------------------------------------------------
+# Loss change of a later first-layer candidate given that an earlier one is kept (two-layer nets).
+# A speculative batch whose decision keeps candidate c1 can decide a later candidate c2 in the same
+# pass if it knows dS(c2 | c1). When both change first-layer weights of different hidden rows
+# (j1 != j2), c2's output-field change is unaffected by c1, so dS(c2 | c1) differs from dS(c2) only
+# on the samples where both input features are non-zero:
+#   dS(c2 | c1) = dS(c2) + sum_{n: x[n,i1] != 0 != x[n,i2]}
+#                 [l(z + d1 + d2) - l(z + d1) - l(z + d2) + l(z)]_n
+# with z the cached output fields and d_k = W2[:, j_k] (f(z1[j_k] + D_k x[i_k]) - f(z1[j_k])).
+# ------------------------------------------------------------------------------------------------
+
+def conditional_dS_two_layer(params: Params, XT: np.ndarray, y: np.ndarray, loss: str, p1, p2):
+    """dS of proposal p2 given that proposal p1 was kept, by the correction above; p1 and p2 are
+    first-layer proposals (layer 0) on different hidden rows. Returns (dS(p2 | p1), dS(p2),
+    number of samples in the correction)."""
+    if p1.layer != 0 or p2.layer != 0 or p1.row == p2.row:
+        raise ValueError("two first-layer proposals on different hidden rows")
+    L1, L2 = params.layers
+    W1, W2 = params.eff64(0), params.eff64(1)
+    z = W2 @ act_fn(L1.act, W1 @ XT, L1.act_param)
+
+    def change(p):
+        zr = W1[p.row] @ XT
+        da = act_fn(L1.act, zr + (p.new - p.old) * XT[p.col], L1.act_param) - \
+            act_fn(L1.act, zr, L1.act_param)
+        return np.outer(W2[:, p.row], da)
+
+    def ell(zz):
+        return loss_per_sample(loss, act_fn(L2.act, zz, L2.act_param), y)
+
+    d1, d2 = change(p1), change(p2)
+    dS2 = float((ell(z + d2) - ell(z)).sum())
+    both = (XT[p1.col] != 0) & (XT[p2.col] != 0)
+    zb, d1b, d2b, yb = z[:, both], d1[:, both], d2[:, both], y[both]
+
+    def ellb(zz):
+        return loss_per_sample(loss, act_fn(L2.act, zz, L2.act_param), yb)
+    corr = float((ellb(zb + d1b + d2b) - ellb(zb + d1b) - ellb(zb + d2b) + ellb(zb)).sum())
+    return dS2 + corr, dS2, int(both.sum())
