@@ -79,3 +79,43 @@ def test_emulated_commit_writes_what_evaluation_computed(setup):
         np.testing.assert_array_equal(refreshed, a.wimg)
         ell = OT.tfm_seq_losses(spec, a.params.astype(np.float64), a.tokens)
         assert np.all(np.abs(a.ell - ell) <= 2e-6 * ell), name
+
+
+def test_emulated_kernel_at_the_largest_shape_it_takes():
+    """Vocabulary 128, d_ff 1024 and three blocks (the largest vocabulary and hidden width the
+    tensor-core kernels accept): forward losses, and candidates at the last row / column of every
+    weight matrix, the last hidden chunk, the last position and the last vocabulary entry, against
+    the oracle; a commit writes what the evaluation computed."""
+    spec = W.TfmSpec(vocab=128, d_ff=1024, n_layer=3)
+    wl = W.char_transformer(batch=2, spec=spec, text_len=20000)
+    a = E.Args(spec, wl.init, wl.tokens)
+    a.split()
+    for pair in range(a.B // 2):
+        E.CTA(a, E.FORWARD, None, pair).run()
+    ell = OT.tfm_seq_losses(spec, a.params.astype(np.float64), a.tokens)
+    assert np.all(np.abs(a.ell - ell) <= 2e-6 * ell)
+    d, F, V, T = a.d, a.F, spec.vocab, spec.ctx
+    bl = a.o_blk0 + 2 * a.blk_size                       # the last block
+    last_tok = int(a.tokens[1, T - 1])
+    picks = {
+        "tok_emb": last_tok * d + d - 1, "pos_emb": a.o_pos + (T - 1) * d + d - 1,
+        "wq": bl + a.r_wq + (d - 1) * d + d - 1, "wv": bl + a.r_wv + (d - 1) * d,
+        "wo": bl + a.r_wo + d - 1, "w1": bl + a.r_w1 + (F - 1) * d + d - 1,
+        "b1": bl + a.r_b1 + F - 1, "w2": bl + a.r_w2 + (d - 1) * F + F - 1,
+        "b2": bl + a.r_b2 + d - 1, "lnf.b": a.o_lnf_b + d - 1,
+        "w_head": a.o_wh + (V - 1) * d + d - 1, "b_head": a.o_bh + V - 1,
+    }
+    for name, idx in picks.items():
+        c = _cand(a, idx, -0.29)
+        q = a.params.copy()
+        q[idx] = c[1]
+        want = OT.tfm_seq_losses(spec, q.astype(np.float64), a.tokens) - ell
+        got = np.concatenate([E.CTA(a, E.EVAL, c, p).run() for p in range(a.B // 2)])
+        assert np.all(np.abs(got - want) <= 2e-6 * ell), (name, got, want)
+    c = _cand(a, picks["w1"], 0.61)
+    ell0 = a.ell.copy()
+    dS = np.concatenate([E.CTA(a, E.EVAL, c, p).run() for p in range(a.B // 2)])
+    a.params[c[0]] = c[1]
+    for p in range(a.B // 2):
+        E.CTA(a, E.COMMIT, c, p).run()
+    np.testing.assert_array_equal(a.ell, (ell0 + dS).astype(np.float32))
