@@ -147,6 +147,16 @@ def is_tfm(wl) -> bool:
     return hasattr(wl, "spec")
 
 
+def acceptance(wl) -> str:
+    return ("greedy (Eq. 6)" if wl.domain.beta == float("inf")
+            else f"Metropolis (Eq. 7), beta = {wl.domain.beta:g}")
+
+
+def proposals(wl) -> str:
+    return ("uniform over all parameters" if not wl.domain.layer_stretch
+            else f"current-layer schedule, {wl.domain.layer_stretch} trials per layer")
+
+
 def host_arrays(wl):
     """The arrays a job uploads: (X, y, init) for an MLP, (tokens, init) for the Transformer."""
     return (wl.tokens, wl.init) if is_tfm(wl) else (wl.X, wl.y, wl.init)
@@ -247,7 +257,8 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
-            "config": {"workload": wl.name, "K": wl.K, "trials_per_step": per_step},
+            "config": {"workload": wl.name, "K": wl.K, "trials_per_step": per_step,
+                       "acceptance": acceptance(wl), "proposals": proposals(wl)},
             "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -419,11 +430,7 @@ def run_ours(args):
                               if not deep else "no flush: a step's candidates recompute from "
                               "cached fields / residual streams that exceed L2 or are rewritten"),
                        "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
-                       "acceptance": ("greedy (Eq. 6)" if wl.domain.beta == float("inf")
-                                      else f"Metropolis (Eq. 7), beta = {wl.domain.beta:g}"),
-                       "proposals": ("uniform over all parameters" if not wl.domain.layer_stretch
-                                     else f"current-layer schedule, {wl.domain.layer_stretch} "
-                                          "trials per layer"),
+                       "acceptance": acceptance(wl), "proposals": proposals(wl),
                        "accepts_timed": st1["accepts"] - st0["accepts"],
                        "batches_timed": st1["batches"] - st0["batches"],
                        "phase_ms": {nm: (st1["phase_ns"][q] - st0["phase_ns"][q]) / 1e6
