@@ -1322,38 +1322,23 @@ mca_status mca_run_channels(mca_handle* h, uint64_t n_trials, uint64_t seed, int
   std::vector<int> node(L + 1);
   std::vector<float> oldw(L), neww(L);
   std::vector<float*> at(L);
-  std::vector<uint32_t> v(2 * L + 4);
   DevState ds;
   mca_status rc = read_state(h, &ds);
   if (rc != MCA_OK) return rc;
   double S = ds.S;
   for (uint64_t t = 0; t < n_trials; ++t) {
     const uint64_t tau = h->tau;
-    for (int q = 0; 4 * q < 2 * L + 1; ++q) {          // channel words: counters (tau, 2, q)
-      const uint4 w = mca::philox4x32_10(
-          make_uint4((uint32_t)tau, (uint32_t)(tau >> 32), 2u, (uint32_t)q),
-          make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
-      v[4 * q] = w.x;
-      v[4 * q + 1] = w.y;
-      v[4 * q + 2] = w.z;
-      v[4 * q + 3] = w.w;
-    }
     for (int m = 0; m <= L; ++m) {
       const unsigned long long n_m =
           m == 0 ? (unsigned long long)h->layers[0].n_in : (unsigned long long)h->layers[m - 1].n_out;
-      node[m] = (int)(((unsigned long long)v[m] * n_m) >> 32);
+      node[m] = mca::channel_node(mca::channel_word(seed, tau, m), n_m);
     }
     for (int m = 0; m < L; ++m) {
       const mca_layer& ly = h->layers[m];
       at[m] = h->w_eff[m] + (size_t)node[m + 1] * ly.n_in + node[m];
-      if (scheme == MCA_CHANNEL_HE) {
-        const float a = (float)std::sqrt(6.0 / (double)ly.n_in);
-        const float u = (float)(v[L + 1 + m] >> 8) * 0x1p-24f;
-        const float r = 2.0f * u;                       // exact
-        neww[m] = a * (r - 1.0f);
-      } else {
-        neww[m] = 0.0f;
-      }
+      neww[m] = scheme == MCA_CHANNEL_HE
+                    ? mca::channel_he_value(mca::channel_word(seed, tau, L + 1 + m), ly.n_in)
+                    : 0.0f;
       CUDA_TRY(h, cudaMemcpyAsync(&oldw[m], at[m], sizeof(float), cudaMemcpyDeviceToHost,
                                   h->stream));
     }

@@ -86,6 +86,29 @@ __host__ __device__ __forceinline__ unsigned int mlp2_trial_index(unsigned long 
   return (unsigned int)(lo + (((unsigned long long)r0 * n) >> 32));
 }
 
+// Channel mutations (Section 2.3): word m of trial tau's channel stream, the m % 4-th word of
+// Philox4x32-10 at counter (tau_lo, tau_hi, 2, m / 4) -- apart from the trial's own counter
+// (tau, 0, 0) and the schedule's (s, 0, 1, 0); a node uniform over n from a word; a redrawn weight
+// a (2u - 1) in fp32 with He's uniform amplitude a = fp32(sqrt(6 / fan_in)), u = (v >> 8) 2^-24.
+__host__ __device__ __forceinline__ uint32_t channel_word(uint64_t seed, uint64_t tau, int m) {
+  const uint4 w = philox4x32_10(make_uint4((uint32_t)tau, (uint32_t)(tau >> 32), 2u,
+                                           (uint32_t)(m >> 2)),
+                                make_uint2((uint32_t)seed, (uint32_t)(seed >> 32)));
+  const int r = m & 3;
+  return r == 0 ? w.x : (r == 1 ? w.y : (r == 2 ? w.z : w.w));
+}
+
+__host__ __device__ __forceinline__ int channel_node(uint32_t v, unsigned long long n) {
+  return (int)(((unsigned long long)v * n) >> 32);
+}
+
+__host__ __device__ __forceinline__ float channel_he_value(uint32_t v, int fan_in) {
+  const float a = (float)sqrt(6.0 / (double)fan_in);
+  const float u = (float)(v >> 8) * 0x1p-24f;
+  const float r = 2.0f * u;                        // exact
+  return a * (r - 1.0f);
+}
+
 // u = (r >> 8) * 2^-24: exact, in [0, 1)
 __device__ __forceinline__ float unit24(uint32_t r) { return __uint2float_rn(r >> 8) * 0x1p-24f; }
 

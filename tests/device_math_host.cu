@@ -7,11 +7,13 @@
 //   stretch SEED S NL                     -> the layer of stretch S
 //   idx2 P P1 SEED TAU R0 M               -> two-layer trial index
 //   idxd SEED TAU R0 M L off0 .. offL     -> deep trial index (L layers, L + 1 offsets)
+//   chan SEED TAU L n0 .. nL fin0 .. finL-1 -> channel nodes c_0 .. c_L, then the L He values
 #include <cstdio>
 #include <cstring>
 #include <iostream>
 #include <sstream>
 #include <string>
+#include <vector>
 
 #include "mca_deep.cuh"
 
@@ -57,6 +59,20 @@ int main() {
       in >> a.seed >> tau >> r0 >> a.stretch >> a.L;
       for (int l = 0; l <= a.L; ++l) in >> a.off[l];
       std::printf("%u\n", mca::deep_trial_index(a, tau, r0));
+    } else if (cmd == "chan") {
+      unsigned long long seed, tau;
+      int L;
+      in >> seed >> tau >> L;
+      std::vector<unsigned long long> nodes(L + 1);
+      std::vector<int> fin(L);
+      for (int m = 0; m <= L; ++m) in >> nodes[m];
+      for (int m = 0; m < L; ++m) in >> fin[m];
+      for (int m = 0; m <= L; ++m)
+        std::printf("%d ", mca::channel_node(mca::channel_word(seed, tau, m), nodes[m]));
+      for (int m = 0; m < L; ++m)
+        std::printf("%.9g ", (double)mca::channel_he_value(mca::channel_word(seed, tau, L + 1 + m),
+                                                           fin[m]));
+      std::printf("\n");
     } else if (!cmd.empty()) {
       std::printf("?\n");
     }

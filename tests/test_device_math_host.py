@@ -2,7 +2,8 @@
 
 csrc/mca_device.cuh and csrc/mca_deep.cuh mark the helpers that turn a trial counter into a
 proposal or a decision (Philox4x32-10, the Metropolis threshold of Eq. 7, the acceptance rule, the
-current-layer schedule's layer choice and the flat index of a trial) as host-and-device functions.
+current-layer schedule's layer choice, the flat index of a trial, and the channel draws of
+Section 2.3's multi-parameter mutations) as host-and-device functions.
 tests/device_math_host.cu is a host program around them; this test builds it with nvcc (no GPU
 needed) and compares its answers with the oracle's independent implementation: Philox words and
 indices bit for bit, thresholds to fp32 rounding. The GPU tests then cover the same functions
@@ -94,3 +95,23 @@ def test_stretch_layer_and_trial_indices(harness):
             wantd = [O.proposal_index(seed, t, int(words[t]), deep, M) for t in range(400)]
             assert [int(v) for v in harness(c2)] == want2
             assert [int(v) for v in harness(cd)] == wantd
+
+
+def test_channel_draws(harness):
+    """The channel of mca_run_channels (nodes of every layer, He redraws) equals the oracle's
+    propose_channel bit for bit."""
+    from paper_2607_08406_gb300 import workloads as W
+    dims = [784, 256, 256, 40, 10]
+    layers = [W.Layer(dims[m], dims[m + 1]) for m in range(len(dims) - 1)]
+    params = O.Params(layers, np.zeros(sum(a * b for a, b in zip(dims[:-1], dims[1:])),
+                                       np.float32))
+    L = len(layers)
+    for seed in (0, 0xFEED_F00D_1234):
+        cmds = [f"chan {seed} {t} {L} " + " ".join(map(str, dims)) + " " +
+                " ".join(str(d) for d in dims[:-1]) for t in range(200)]
+        for t, line in enumerate(harness(cmds)):
+            vals = line.split()
+            ch = O.propose_channel(seed, t, params, "he")
+            nodes = [c[2] for c in ch] + [ch[-1][1]]
+            assert [int(v) for v in vals[:L + 1]] == nodes
+            assert [np.float32(float(v)) for v in vals[L + 1:]] == [np.float32(c[4]) for c in ch]
