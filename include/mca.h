@@ -4,10 +4,13 @@
  * The method (paper "Beyond Backpropagation: Monte Carlo Method Can Train Deep Neural Networks"):
  * pick one parameter at random, give it a new random value (Section 2, Eq. 1), re-evaluate the
  * full-batch training loss (Eq. 2 with R = 0) and keep the change iff the loss does not rise
- * (greedy rule, Section 3.1 Eq. 6); otherwise restore the old value and try again. The loss is
- * re-evaluated from cached per-layer local fields (Section 2.4): a mutation of weight (j, i) of
+ * (greedy rule, Section 3.1 Eq. 6; or Eq. 7's Metropolis rule, mca_domain.temperature);
+ * otherwise restore the old value and try again. The loss is re-evaluated from cached per-layer
+ * local fields (Section 2.4): a mutation of weight (j, i) of
  * layer l changes only row j of that layer's fields (a rank-1 update over all samples) and, through
- * neuron j's activation change, the next layer's fields by one weight column.
+ * neuron j's activation change, the next layer's fields by one weight column. Also: the
+ * current-layer proposal schedule (Section 2.1, mca_domain.layer_stretch) and multi-parameter
+ * channel mutations (Section 2.3, mca_run_channels).
  *
  * Conventions shared by every call:
  *  - Every call returns an mca_status; no C++ exception crosses this boundary. A failed call
