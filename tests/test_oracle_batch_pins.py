@@ -89,3 +89,15 @@ def test_planted_previous_batch_is_caught(monkeypatch):
     monkeypatch.setattr(O, "run_batches", shifted)
     with pytest.raises(AssertionError):
         test_each_stretch_follows_the_definition_on_its_batch()
+
+
+def test_minibatch_generator_draws_without_replacement():
+    """Each batch holds distinct sample indices in ascending order, every sample is equally likely
+    to be drawn (chi-square over 4000 batches), and the same seed gives the same batches."""
+    from scipy import stats
+    bs = W.minibatches(100, 30, 4000, seed=8)
+    for b in bs[:50]:
+        assert len(b) == 30 and np.all(np.diff(b) > 0) and b[0] >= 0 and b[-1] < 100
+    counts = np.bincount(np.concatenate(bs), minlength=100)
+    assert stats.chisquare(counts).pvalue > 1e-4
+    assert all(np.array_equal(a, b) for a, b in zip(bs[:5], W.minibatches(100, 30, 5, seed=8)))
