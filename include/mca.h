@@ -284,19 +284,49 @@ mca_status mca_get_stats(mca_handle* h, mca_run_stats* stats);
 mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
                                size_t n, double* dS);
 
+/* The proposals of trials tau .. tau+n-1 (n <= 128) as mca_run would draw them with Philox key
+ * `seed` (Eq. 1: index rule, current-layer schedule, mutation of the layer's storage kind, domain
+ * check), each evaluated against the current state with no commit (the kernels of
+ * mca_eval_candidates). out[k] (host): tau, idx, old_w, new_w (effective weights), valid, dS (NaN
+ * for a proposal outside the weight domain), S (the handle's current loss sum), accept = forced =
+ * 0. The handle's trial counter and state do not change. This is one shard's step of a chain whose
+ * samples are split over several handles (the loss is a sum over samples, Eq. 2): every shard
+ * evaluates the same trials on its own samples, the shards' dS are added, one decision
+ * (mca_decide_batch) is taken for all, and every shard commits it (mca_force_decisions for the
+ * batch's consumed trials, then mca_run over them). */
+mca_status mca_eval_trials(mca_handle* h, uint64_t seed, uint64_t tau, size_t n,
+                           mca_trace_rec* out);
+
+/* The decision of a batch of trials tau .. tau+n-1 with loss changes dS[k] (host arrays; valid[k]
+ * = 0 skips trial k, as for a proposal outside the weight domain): *kstar = the lowest k with
+ * dS[k] <= theta_{tau+k} (< when the domain is strict), theta = 0 under the greedy rule (Eq. 6)
+ * and -(N / beta) ln u_{tau+k} under Eq. 7's Metropolis rule (mca_domain.temperature), evaluated
+ * exactly as the kernels do (dS rounded to fp32); -1 if none. N = n_samples, the chain's whole
+ * sample count (a sharded chain's sum over all shards), or the handle's own when n_samples = 0.
+ * Host only, no device work. Errors: INVALID, NUMERIC (a non-finite dS of a valid trial before
+ * the accepted one). */
+mca_status mca_decide_batch(mca_handle* h, uint64_t seed, uint64_t tau, size_t n,
+                            const uint8_t* valid, const double* dS, int64_t n_samples,
+                            int32_t* kstar);
+
 /* The same evaluation as mca_eval_candidates, for callers that cannot allocate device memory:
  * a caller whose device memory is entirely reserved by another allocator (a framework's caching
  * allocator, a fixed arena), or a latency-critical loop that cannot afford the device-wide
  * synchronisation a cudaMalloc or cudaFree may cause. The paper has no counterpart; this is an
- * interface convenience. flat_idx [n] (uint32), new_w [n] (fp32) and dS [n] (fp64) are DEVICE
- * arrays owned by the caller. The evaluation's scratch (one partial per candidate and sample
+ * interface convenience. Single-hidden-layer handles only: a deep or Transformer handle gives
+ * MCA_ERR_UNSUPPORTED before any device work and stays usable. The handle's device must be the
+ * current device (else MCA_ERR_INVALID, handle unchanged). flat_idx [n] (uint32), new_w [n]
+ * (fp32) and dS [n] (fp64) are DEVICE arrays owned by the caller; the call copies flat_idx and
+ * new_w back to the host (on the stack) to check them against P and for finiteness, and
+ * synchronises the handle's stream twice (after that read and after the evaluation), so it
+ * returns with the results in dS. The evaluation's scratch (one partial per candidate and sample
  * range, plus a grid barrier) lives in a fixed 128 KB + 256 B device array inside the library,
  * which every GPU that loads the library holds until the process exits; nothing is allocated per
  * call. Limits: n <= 128 candidates and a handle of at most 256 sample ranges, else
  * MCA_ERR_INVALID with a message. The first call on a device looks up the array's device address
  * (once per device), so make that first call before any stream capture. All calls share the
  * array: calls whose work overlaps on the GPU (two handles on different streams, or two threads)
- * race and must be serialised by the caller. Blocks until the results are in dS. */
+ * race and must be serialised by the caller. */
 mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t* flat_idx,
                                        const float* new_w, size_t n, double* dS);
 

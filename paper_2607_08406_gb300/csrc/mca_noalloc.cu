@@ -64,7 +64,8 @@ extern "C" mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t*
   if (!flat_idx || !new_w || !dS) return set_err(h, MCA_ERR_INVALID, "NULL argument");
   if (h->broken)
     return set_err(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
-  if (h->deep)
+  // single-hidden-layer handles only; refused before any CUDA call, the handle stays usable
+  if (h->deep || h->tfm)
     return set_err(h, MCA_ERR_UNSUPPORTED,
                    "the no-allocation evaluation runs single-hidden-layer handles only");
   if (n > (size_t)kNoAllocMaxCandidates)
@@ -76,6 +77,17 @@ extern "C" mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t*
                    "handle uses " + std::to_string(h->NR) +
                        " sample ranges; the no-allocation scratch holds at most " +
                        std::to_string(kNoAllocMaxRanges));
+  // the scratch address and the handle's stream both belong to the current device, so the
+  // caller must have made the handle's device current (a mistake, not a device error)
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    return set_err(h, MCA_ERR_INVALID, "no usable current device");
+  }
+  if (dev != h->device)
+    return set_err(h, MCA_ERR_INVALID,
+                   "current device " + std::to_string(dev) + " is not the handle's device " +
+                       std::to_string(h->device) + "; make the handle's device current first");
   if (!on_device(flat_idx) || !on_device(new_w) || !on_device(dS))
     return set_err(h, MCA_ERR_INVALID, "flat_idx, new_w and dS must be device pointers");
   // the kernel trusts its indices: check them (and the values) on the host, on the stack
@@ -96,10 +108,6 @@ extern "C" mca_status mca_eval_candidates_noalloc(mca_handle* h, const uint32_t*
     if (!std::isfinite(hnew[m]))
       return set_err(h, MCA_ERR_INVALID, "new_w[" + std::to_string(m) + "] not finite");
   }
-  int dev = 0;
-  e = cudaGetDevice(&dev);
-  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-    return set_err(h, MCA_ERR_CUDA, "no usable current device");
   void* base = nullptr;
   e = scratch_address(dev, &base);
   if (e != cudaSuccess)
