@@ -116,31 +116,3 @@ def test_deep_resync_keeps_loss(gpu_lib):
     L_inc = gpu_lib.mca_loss(h)
     gpu_lib.mca_resync(h)
     assert gpu_lib.mca_loss(h) == pytest.approx(L_inc, rel=1e-6)
-
-
-def test_deep_full_size_24x256(gpu_lib):
-    """784-(256 x 24)-10 tanh CE on N = 10000, K = 128: candidates of every layer against the oracle
-    at the initial state, then 256 trials whose proposals and committed weights replay through the
-    oracle's proposal rule, and the final loss."""
-    wl = W.mlp_deep()
-    h = gpu_lib.create_from_workload(wl, trace_cap=256)
-    p0 = O.Params(wl.layers, wl.init)
-    rng = np.random.default_rng(11)
-    idx = _idx_per_layer(wl, rng, 1)[[0, 1, 12, 22, 23, 24]]
-    new = rng.uniform(-1, 1, len(idx)).astype(np.float32)
-    d = gpu_lib.mca_eval_candidates(h, idx, new)
-    want, S0 = _oracle_candidates(wl, p0, idx, new)
-    assert gpu_lib.mca_loss(h) * wl.N == pytest.approx(S0, rel=1e-5)
-    assert np.all(np.abs(d - want) <= TIE_REL * S0), (d, want)
-    st = gpu_lib.mca_run(h, 256, wl.seed)
-    g = gpu_lib.mca_get_trace(h, 256)
-    assert st["trials"] == 256 and len(g) == 256 and st["tensor_cores"] == 1
-    params = O.Params(wl.layers, wl.init)
-    for t in range(256):
-        p = O.propose(wl.seed, t, params, wl.domain)
-        assert p.idx == int(g["idx"][t]) and np.float32(p.new) == g["new_w"][t]
-        if g["accept"][t]:
-            O.apply_proposal(params, p)
-    assert np.array_equal(gpu_lib.mca_get_params(h, wl.n_params), params.flat_eff32())
-    S = O.total_loss(params, wl.X.T.astype(np.float64), wl.y, wl.loss)
-    assert gpu_lib.mca_loss(h) * wl.N == pytest.approx(S, rel=1e-5)

@@ -290,47 +290,3 @@ def test_set_params_resume(gpu_lib):
     assert np.array_equal(gpu_lib.mca_get_params(h3, wl.n_params), p)
     gpu_lib.mca_run(h3, 1000, 9)
     assert np.array_equal(gpu_lib.mca_get_trace(h3, 1000), full[1000:])
-
-
-def test_full_size_wide_bench_config(gpu_lib):
-    """784-16384-10 CE on N = 60000 with K = 64 and the automatic grid (the bench's launch shape):
-    the candidates before the first accept are checked against the oracle's dS at the initial
-    state; the proposals and committed weights of 3000 trials are replayed through the oracle's
-    proposal rule bit for bit; the final loss and 48 sampled candidates are checked against the
-    oracle at the final state."""
-    wl = W.mlp_wide()
-    n = 3000
-    h = gpu_lib.create_from_workload(wl, trace_cap=n)
-    XT = wl.X.T.astype(np.float64)
-    p0 = O.Params(wl.layers, wl.init)
-    Z2 = O.output_fields_blocked(p0, XT)
-    S0 = float(O.loss_per_sample(wl.loss, Z2, wl.y).sum())
-    assert gpu_lib.mca_loss(h) * wl.N == pytest.approx(S0, rel=1e-6)
-    st = gpu_lib.mca_run(h, n, wl.seed)
-    g = gpu_lib.mca_get_trace(h, n)
-    assert len(g) == n and st["trials"] == n
-    first = int(np.argmax(g["accept"] == 1))
-    for t in range(first + 1):
-        want = O.candidate_dS_two_layer(p0, XT, wl.y, wl.loss, Z2, int(g["idx"][t]),
-                                        float(g["new_w"][t]))
-        assert abs(g["dS"][t] - want) <= TIE_REL * S0
-        assert (g["dS"][t] <= 0) == (want <= 0) or abs(want) < TIE_REL * S0
-    params = O.Params(wl.layers, wl.init)
-    for t in range(n):
-        p = O.propose(wl.seed, t, params, wl.domain)
-        assert p.idx == int(g["idx"][t]) and np.float32(p.new) == g["new_w"][t]
-        if g["accept"][t]:
-            O.apply_proposal(params, p)
-    got = gpu_lib.mca_get_params(h, wl.n_params)
-    assert np.array_equal(got, params.flat_eff32())
-    Z2f = O.output_fields_blocked(params, XT)
-    Sf = float(O.loss_per_sample(wl.loss, Z2f, wl.y).sum())
-    assert gpu_lib.mca_loss(h) * wl.N == pytest.approx(Sf, rel=1e-5)
-    rng = np.random.default_rng(1)
-    P1 = 784 * 16384
-    idx = np.concatenate([rng.integers(0, P1, 40), rng.integers(P1, wl.n_params, 8)])
-    new = rng.uniform(-1, 1, len(idx)).astype(np.float32)
-    d = gpu_lib.mca_eval_candidates(h, idx, new)
-    for m in range(len(idx)):
-        want = O.candidate_dS_two_layer(params, XT, wl.y, wl.loss, Z2f, int(idx[m]), float(new[m]))
-        assert abs(d[m] - want) <= TIE_REL * Sf, (m, d[m], want)
