@@ -76,7 +76,7 @@ bool is_device_ptr(const void* p) {
 
 struct Layout {
   size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, accum, bar, st, trace,
-      ex_idx, ex_new, ex_out, scratch, ell, ctl, total;
+      ex_idx, ex_new, ex_out, prop, scratch, ell, ctl, gimg, total;
   std::vector<size_t> w_eff, code, wfix, Z, whi;
 };
 
@@ -94,6 +94,31 @@ bool deep_tc_ok(const std::vector<mca_layer>& layers) {
 int deep_tc_tiles(long long N) { return (int)((N + mca::kTcTS - 1) / mca::kTcTS); }
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
+
+// The forward pass (creation, resync) computes the fields of a layer on the tensor cores
+// (mca_gemm_tc.cu) when its shape allows, unless the process sets MCA_FORWARD_TENSOR_CORES=0 (then
+// with the SIMT SGEMM). Read by mca_workspace_size and mca_create (the operand images are part of
+// the workspace), so it must not change between the two.
+bool forward_tc_enabled() {
+  const char* e = std::getenv("MCA_FORWARD_TENSOR_CORES");
+  return !(e && std::strcmp(e, "0") == 0);
+}
+
+// Layers whose fields the forward pass computes with a GEMM: the first layer of a two-layer net
+// (its output fields have their own kernel), every layer of a deep net.
+bool forward_tc_layer(const std::vector<mca_layer>& layers, size_t l, int Np) {
+  if (!forward_tc_enabled()) return false;
+  if (!is_deep(layers) && l != 0) return false;
+  return mca::gemm_tc_ok(layers[l].n_out, layers[l].n_in, Np);
+}
+
+size_t forward_tc_image_bytes(const std::vector<mca_layer>& layers, int Np) {
+  size_t b = 0;
+  for (size_t l = 0; l < layers.size(); ++l)
+    if (forward_tc_layer(layers, l, Np))
+      b = std::max(b, mca::gemm_tc_image_bytes(layers[l].n_out, layers[l].n_in, Np));
+  return b;
+}
 
 // Device memory of a handle. Single hidden layer: feature CSR of X, z1, sample records, per-range
 // partials. Deep: the fields of every layer, per-sample losses, per-tile partials.
@@ -146,7 +171,10 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   L.ex_idx = take(sizeof(unsigned int) * mca::kKmax);
   L.ex_new = take(sizeof(float) * mca::kKmax);
   L.ex_out = take(sizeof(double) * mca::kKmax);
+  L.prop = take(sizeof(mca_trace_rec) * mca::kKmax);
   L.scratch = take(sizeof(int) * (size_t)(D + 8));
+  const size_t gb = forward_tc_image_bytes(layers, Np);
+  L.gimg = gb ? take(gb) : SIZE_MAX;
   L.total = o;
   return L;
 }
@@ -437,15 +465,30 @@ mca_status resync(mca_handle* h) {
       CUDA_TRY(h, mca::launch_deep_split(a, h->stream));
       h->launches += 1;
     }
-    for (int l = 0; l < a.L; ++l) CUDA_TRY(h, mca::launch_deep_forward_layer(a, l, h->stream));
+    for (int l = 0; l < a.L; ++l) {
+      if (h->gimg && forward_tc_layer(h->layers, (size_t)l, h->Np)) {
+        CUDA_TRY(h, mca::launch_gemm_tc(a.w[l], a.n_out[l], a.n_in[l], l == 0 ? a.XT : a.Z[l - 1],
+                                        l == 0 ? -1 : a.act[l - 1], l == 0 ? 0.0f : a.g[l - 1],
+                                        a.Z[l], h->Np, h->gimg, &h->st->err, h->stream));
+        h->launches += 2;                      // its two operand-image kernels
+      } else {
+        CUDA_TRY(h, mca::launch_deep_forward_layer(a, l, h->stream));
+      }
+    }
     CUDA_TRY(h, mca::launch_deep_losses(a, h->stream));
     CUDA_TRY(h, mca::launch_sum_loss(h->ell, (int)h->N, h->st, h->stream));
     h->launches += a.L + 2;
     return MCA_OK;
   }
   mca::Mlp2Args a = mlp2_args(h);
-  CUDA_TRY(h, mca::launch_sgemm_nn(a.H, h->Np, h->D, h->w_eff[0], h->D, h->XT, h->Np, h->z1,
-                                   h->Np, h->stream));
+  if (h->gimg && forward_tc_layer(h->layers, 0, h->Np)) {
+    CUDA_TRY(h, mca::launch_gemm_tc(h->w_eff[0], a.H, h->D, h->XT, -1, 0.0f, h->z1, h->Np, h->gimg,
+                                    &h->st->err, h->stream));
+    h->launches += 2;                          // the two operand-image kernels
+  } else {
+    CUDA_TRY(h, mca::launch_sgemm_nn(a.H, h->Np, h->D, h->w_eff[0], h->D, h->XT, h->Np, h->z1,
+                                     h->Np, h->stream));
+  }
   CUDA_TRY(h, mca::launch_mlp2_outputs(a, h->y, h->stream));
   CUDA_TRY(h, mca::launch_sum_loss(h->srec + (size_t)mca::kRecLoss * h->Np, (int)h->N, h->st,
                                     h->stream));
@@ -572,8 +615,8 @@ mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
 }
 
 struct TfmMem {
-  size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, scratch, wimg,
-      total;
+  size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, prop, scratch,
+      wimg, total;
 };
 
 // The tensor-core Transformer kernels (mca_tfm_tc.cu) run a handle's sequences when the shape is
@@ -605,6 +648,7 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc) {
   M.ex_idx = take(sizeof(unsigned int) * mca::kKmax);
   M.ex_new = take(sizeof(float) * mca::kKmax);
   M.ex_out = take(sizeof(double) * mca::kKmax);
+  M.prop = take(sizeof(mca_trace_rec) * mca::kKmax);
   M.scratch = take(sizeof(int) * 8);
   M.wimg = tc ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
   M.total = o;
@@ -836,6 +880,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   h->ex_idx = reinterpret_cast<unsigned int*>(base + L.ex_idx);
   h->ex_new = reinterpret_cast<float*>(base + L.ex_new);
   h->ex_out = reinterpret_cast<double*>(base + L.ex_out);
+  h->prop = reinterpret_cast<mca_trace_rec*>(base + L.prop);
+  h->gimg = L.gimg != SIZE_MAX ? reinterpret_cast<float*>(base + L.gimg) : nullptr;
   int* scratch = reinterpret_cast<int*>(base + L.scratch);
   CTRY(cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream));
   CTRY(cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), h->stream));
@@ -897,6 +943,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
   TRY(resync(h));
   DevState ds;
   TRY(read_state(h, &ds));
+  if (ds.err == MCA_ERR_TIMEOUT)
+    return bail(fail(h, MCA_ERR_TIMEOUT, "device-side wait timed out in the forward pass"));
   if (!std::isfinite(ds.S)) return bail(fail(h, MCA_ERR_NUMERIC, "initial loss is not finite"));
 #undef TRY
 #undef CTRY
@@ -1075,7 +1123,13 @@ mca_status mca_resync(mca_handle* h) {
   if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
   mca_status rc = resync(h);
   if (rc != MCA_OK) return rc;
-  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  DevState ds;
+  rc = read_state(h, &ds);
+  if (rc != MCA_OK) return rc;
+  if (ds.err == MCA_ERR_TIMEOUT) {
+    h->broken = true;
+    return fail(h, MCA_ERR_TIMEOUT, "device-side wait timed out in the forward pass");
+  }
   return MCA_OK;
 }
 
@@ -1120,20 +1174,11 @@ mca_status mca_force_decisions(mca_handle* h, const uint64_t* tau, const uint8_t
   return MCA_OK;
 }
 
-mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
-                               size_t n, double* dS) {
-  if (!h || (n && (!flat_idx || !new_w || !dS))) return fail(h, MCA_ERR_INVALID, "NULL argument");
-  if (n > (size_t)mca::kKmax) return fail(h, MCA_ERR_INVALID, "n = %zu > %d", n, mca::kKmax);
-  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
-  if (n == 0) return MCA_OK;
-  for (size_t m = 0; m < n; ++m) {
-    if (flat_idx[m] >= h->P) return fail(h, MCA_ERR_INVALID, "flat_idx[%zu] >= P", m);
-    if (!std::isfinite(new_w[m])) return fail(h, MCA_ERR_INVALID, "new_w[%zu] not finite", m);
-  }
-  CUDA_TRY(h, cudaMemcpyAsync(h->ex_idx, flat_idx, sizeof(unsigned int) * n, cudaMemcpyHostToDevice,
-                              h->stream));
-  CUDA_TRY(h, cudaMemcpyAsync(h->ex_new, new_w, sizeof(float) * n, cudaMemcpyHostToDevice,
-                              h->stream));
+namespace {
+
+// Loss changes of the n candidates in h->ex_idx / h->ex_new against the current state, no commit,
+// into dS (host). The evaluation kernels of mca_run's evaluation step.
+mca_status eval_explicit(mca_handle* h, size_t n, double* dS) {
   if (h->tfm) {
     mca::TfmArgs a = tfm_args(h);
     a.n_explicit = (int)n;
@@ -1171,6 +1216,96 @@ mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const fl
   if (ds.err == MCA_ERR_TIMEOUT) {
     h->broken = true;
     return fail(h, MCA_ERR_TIMEOUT, "device-side wait timed out");
+  }
+  return MCA_OK;
+}
+
+}  // namespace
+
+mca_status mca_eval_candidates(mca_handle* h, const uint32_t* flat_idx, const float* new_w,
+                               size_t n, double* dS) {
+  if (!h || (n && (!flat_idx || !new_w || !dS))) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (n > (size_t)mca::kKmax) return fail(h, MCA_ERR_INVALID, "n = %zu > %d", n, mca::kKmax);
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (n == 0) return MCA_OK;
+  for (size_t m = 0; m < n; ++m) {
+    if (flat_idx[m] >= h->P) return fail(h, MCA_ERR_INVALID, "flat_idx[%zu] >= P", m);
+    if (!std::isfinite(new_w[m])) return fail(h, MCA_ERR_INVALID, "new_w[%zu] not finite", m);
+  }
+  CUDA_TRY(h, cudaMemcpyAsync(h->ex_idx, flat_idx, sizeof(unsigned int) * n, cudaMemcpyHostToDevice,
+                              h->stream));
+  CUDA_TRY(h, cudaMemcpyAsync(h->ex_new, new_w, sizeof(float) * n, cudaMemcpyHostToDevice,
+                              h->stream));
+  return eval_explicit(h, n, dS);
+}
+
+mca_status mca_eval_trials(mca_handle* h, uint64_t seed, uint64_t tau, size_t n,
+                           mca_trace_rec* out) {
+  if (!h) return fail(nullptr, MCA_ERR_INVALID, "NULL handle");
+  if (n && !out) return fail(h, MCA_ERR_INVALID, "NULL out");
+  if (n > (size_t)mca::kKmax) return fail(h, MCA_ERR_INVALID, "n = %zu > %d", n, mca::kKmax);
+  if (h->broken) return fail(h, MCA_ERR_CUDA, "handle unusable after an earlier device error");
+  if (n == 0) return MCA_OK;
+  mca::ProposeArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.L = (int)h->layers.size();
+  a.n = (int)n;
+  for (int l = 0; l < a.L; ++l) {
+    a.off[l] = h->off[l];
+    a.wk[l] = h->layers[l].wkind;
+    a.sc[l] = h->layers[l].scale;
+    a.w[l] = h->w_eff[l];
+    a.code[l] = h->code[l];
+    a.wfix[l] = h->wfix[l];
+  }
+  a.off[a.L] = h->P;
+  a.op = h->dom.op;
+  a.lo = h->dom.lo;
+  a.hi = h->dom.hi;
+  a.delta = h->dom.delta;
+  a.bound = h->dom.bound;
+  a.stretch = h->dom.layer_stretch;
+  a.seed = seed;
+  a.tau0 = tau;
+  a.rec = h->prop;
+  a.ex_idx = h->ex_idx;
+  a.ex_new = h->ex_new;
+  CUDA_TRY(h, mca::launch_propose(a, h->stream));
+  h->launches++;
+  CUDA_TRY(h, cudaMemcpyAsync(out, h->prop, sizeof(mca_trace_rec) * n, cudaMemcpyDeviceToHost,
+                              h->stream));
+  double dS[mca::kKmax];
+  mca_status rc = eval_explicit(h, n, dS);
+  if (rc != MCA_OK) return rc;
+  double S = 0.0;
+  rc = mca_loss(h, &S);
+  if (rc != MCA_OK) return rc;
+  S *= (double)h->N;
+  for (size_t k = 0; k < n; ++k) {
+    out[k].dS = out[k].valid ? dS[k] : std::nan("");
+    out[k].S = S;
+  }
+  return MCA_OK;
+}
+
+mca_status mca_decide_batch(mca_handle* h, uint64_t seed, uint64_t tau, size_t n,
+                            const uint8_t* valid, const double* dS, int64_t n_samples,
+                            int32_t* kstar) {
+  if (!h || !kstar || (n && (!valid || !dS))) return fail(h, MCA_ERR_INVALID, "NULL argument");
+  if (n_samples < 0) return fail(h, MCA_ERR_INVALID, "n_samples < 0");
+  const double N = n_samples > 0 ? (double)n_samples : (double)h->N;
+  const int metro = h->dom.temperature > 0.0f ? 1 : 0;
+  const double msc = N * (double)h->dom.temperature;
+  *kstar = -1;
+  for (size_t k = 0; k < n; ++k) {
+    if (!valid[k]) continue;
+    if (!std::isfinite(dS[k]))
+      return fail(h, MCA_ERR_NUMERIC, "non-finite loss change of trial %llu",
+                  (unsigned long long)(tau + k));
+    if (mca::accept_change((float)dS[k], h->dom.strict, metro, seed, tau + k, msc)) {
+      *kstar = (int32_t)k;
+      break;
+    }
   }
   return MCA_OK;
 }
@@ -1268,6 +1403,7 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->ex_idx = reinterpret_cast<unsigned int*>(base + M.ex_idx);
   h->ex_new = reinterpret_cast<float*>(base + M.ex_new);
   h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
+  h->prop = reinterpret_cast<mca_trace_rec*>(base + M.prop);
   h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
   e = cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream);

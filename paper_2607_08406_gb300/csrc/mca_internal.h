@@ -269,6 +269,35 @@ size_t mlp2_window_smem_bytes(int RS);
 int mlp2_loop_max_grid(const Mlp2Args& a, int num_sms);
 size_t mlp2_loop_smem_bytes(const Mlp2Args& a);
 
+// Proposals of trials tau0 .. tau0 + n - 1 as explicit candidates (mca_propose.cu): the trial's
+// record (index, effective weights before and after, validity) and the candidate arrays of the
+// explicit evaluation (a rejected proposal is evaluated as the no-op).
+struct ProposeArgs {
+  int L, n;
+  unsigned long long off[kMaxLayers + 1];   // flat offset of each layer; off[L] = P
+  int wk[kMaxLayers];
+  float sc[kMaxLayers];
+  const float* w[kMaxLayers];
+  const signed char* code[kMaxLayers];
+  const float* wfix[kMaxLayers];
+  int op;
+  float lo, hi, delta, bound;
+  int stretch;
+  unsigned long long seed, tau0;
+  mca_trace_rec* rec;        // [n]
+  unsigned int* ex_idx;      // [n]
+  float* ex_new;             // [n]
+};
+cudaError_t launch_propose(const ProposeArgs& a, cudaStream_t s);
+
+// Fields of a layer on the tensor cores (mca_gemm_tc.cu): Z[M x Np] = W[M x K] act(B)[K x Np]
+// (act < 0: B as it is), 3xTF32. img: scratch of gemm_tc_image_bytes(M, K, Np) bytes, 256-byte
+// aligned; err: device status word (MCA_ERR_TIMEOUT when a bounded wait ran out).
+bool gemm_tc_ok(int M, int K, int Np);
+size_t gemm_tc_image_bytes(int M, int K, int Np);
+cudaError_t launch_gemm_tc(const float* W, int M, int K, const float* B, int act, float g,
+                           float* Z, int Np, float* img, int* err, cudaStream_t s);
+
 }  // namespace mca
 
 struct mca_handle;
@@ -328,6 +357,8 @@ struct mca_handle {
   unsigned int* ex_idx = nullptr;
   float* ex_new = nullptr;
   double* ex_out = nullptr;
+  mca_trace_rec* prop = nullptr;         // [kKmax] proposals of mca_eval_trials
+  float* gimg = nullptr;                 // operand images of the tensor-core forward pass
   // test hook
   unsigned long long* ftau = nullptr;
   unsigned char* facc = nullptr;

@@ -140,3 +140,34 @@ def test_config_size_transformer(gpu_lib, monkeypatch, tfm_case, tensor_cores):
     assert np.array_equal(gpu_lib.mca_get_params(h, wl.n_params), flat)
     assert gpu_lib.mca_loss(h) * BT == pytest.approx(S, rel=1e-5)
     h.close()
+
+
+def test_config_size_drift_bound(gpu_lib):
+    """784-16384-10 CE, N = 60000: 2 x 10^5 trials of incremental fp32 commits without a resync
+    (the bench's setting) keep the cached loss within 1e-5 of a fresh full forward pass."""
+    wl = W.mlp_wide()
+    h = gpu_lib.create_from_workload(wl)
+    st = gpu_lib.mca_run(h, 200_000, wl.seed)
+    assert st["resyncs"] == 0 and st["accepts"] > 10_000
+    L_inc = gpu_lib.mca_loss(h)
+    gpu_lib.mca_resync(h)
+    assert gpu_lib.mca_loss(h) == pytest.approx(L_inc, rel=1e-5)
+    h.close()
+
+
+@pytest.mark.parametrize("case", ["wide", "deep", "ternary"])
+def test_forward_pass_tensor_cores_against_simt(gpu_lib, monkeypatch, case):
+    """The forward pass on the tensor cores (3xTF32) and the SIMT SGEMM give the same loss to
+    fp32 rounding at the full sizes, and the dyadic workload's exactly representable first layer
+    gives the same loss bit for bit."""
+    make = MLP_CASES[case][0]
+    wl = make()
+    S = {}
+    for flag in ("1", "0"):
+        monkeypatch.setenv("MCA_FORWARD_TENSOR_CORES", flag)
+        h = gpu_lib.create_from_workload(wl)
+        S[flag] = gpu_lib.mca_loss(h)
+        h.close()
+    assert S["1"] == pytest.approx(S["0"], rel=5e-6)
+    if case == "ternary":
+        assert S["1"] == S["0"]
