@@ -99,6 +99,9 @@ SIGNATURES = {
     "mca_get_stats": (c_int32, [c_void_p, POINTER(mca_run_stats)]),
     "mca_eval_candidates": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "mca_eval_candidates_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "mca_eval_trials": (c_int32, [c_void_p, c_uint64, c_uint64, c_size_t, c_void_p]),
+    "mca_decide_batch": (c_int32, [c_void_p, c_uint64, c_uint64, c_size_t, c_void_p, c_void_p,
+                                   c_int64, POINTER(c_int32)]),
     "mca_run_channels": (c_int32, [c_void_p, c_uint64, c_uint64, c_int32, c_void_p, c_void_p]),
     "mca_selftest_wait_timeout": (c_int32, [POINTER(c_int32), POINTER(c_double)]),
     "mca_destroy": (None, [c_void_p]),
@@ -338,6 +341,24 @@ def mca_eval_candidates_noalloc(h: Handle, flat_idx, new_w, dS):
     _check(load_library().mca_eval_candidates_noalloc(h.ptr, flat_idx.data_ptr(), new_w.data_ptr(),
                                                       n, dS.data_ptr()), h.ptr)
     return dS
+
+
+def mca_eval_trials(h: Handle, seed: int, tau: int, n: int) -> np.ndarray:
+    """Proposals of trials tau .. tau+n-1 and their loss changes on this handle's samples (no
+    commit): a structured array of TRACE_DTYPE records."""
+    buf = np.zeros(n, TRACE_DTYPE)
+    _check(load_library().mca_eval_trials(h.ptr, seed, tau, n, buf.ctypes.data), h.ptr)
+    return buf
+
+
+def mca_decide_batch(h: Handle, seed: int, tau: int, valid, dS, n_samples: int = 0) -> int:
+    """Index of the accepted trial of a batch under the handle's rule (Eq. 6 / Eq. 7), -1 if none."""
+    v = np.ascontiguousarray(np.asarray(valid, dtype=np.uint8))
+    d = np.ascontiguousarray(np.asarray(dS, dtype=np.float64))
+    k = c_int32(-1)
+    _check(load_library().mca_decide_batch(h.ptr, seed, tau, len(v), v.ctypes.data, d.ctypes.data,
+                                           n_samples, ctypes.byref(k)), h.ptr)
+    return k.value
 
 
 CHANNEL = {"he": 0, "zero": 1}

@@ -130,3 +130,94 @@ def test_sample_sharded_decisions_match_single_process_oracle():
         assert abs(dS - odS) <= 1e-9 * max(1.0, abs(odS)), (t, dS, odS)
     else:
         assert np.array_equal(out[0][1], params.flat_eff32())
+
+
+class OracleShard:
+    """A shard of ShardedChain evaluated by the oracle's cached-field mode on the rank's samples
+    (the CPU stand-in for a handle on one GPU); records every consumed trial."""
+
+    def __init__(self, wl, shard_rows):
+        from oracle import mca_oracle as O
+        self.O = O
+        self.wl = wl
+        self.XT = wl.X.T.astype(np.float64)[:, shard_rows]
+        self.y = wl.y[shard_rows]
+        self.params = O.Params(wl.layers, wl.init)
+        self.cache = O._Cache(self.params, self.XT, self.y, wl.loss)
+        self.props, self.updates, self.ell, self.last_dS = [], [], [], None
+        self.record = []
+
+    def eval_trials(self, seed, tau, n):
+        O = self.O
+        self.props = [O.propose(seed, tau + k, self.params, self.wl.domain) for k in range(n)]
+        valid = np.array([p.valid for p in self.props])
+        res = [O._candidate(self.params, self.cache, self.XT, self.y, self.wl.loss, p)
+               if p.valid else (0.0, None, None) for p in self.props]
+        self.updates = [r[1] for r in res]
+        self.ell = [r[2] for r in res]
+        part = np.array([r[0] for r in res], np.float64)
+        return valid, part, np.array([p.idx for p in self.props])
+
+    def decide(self, seed, tau, valid, dS, n_samples):
+        O = self.O
+        self.last_dS = dS
+        for k in range(len(valid)):
+            if valid[k] and O._decide(float(dS[k]), self.wl.domain.strict,
+                                      O._threshold(seed, tau + k, self.wl.domain, n_samples)):
+                return k
+        return -1
+
+    def commit(self, seed, tau, m, kstar):
+        for k in range(m):
+            self.record.append((tau + k, self.props[k].idx, k == kstar))
+        if kstar >= 0:
+            self.O.apply_proposal(self.params, self.props[kstar])
+            for lay, upd in self.updates[kstar]:
+                if upd[0] == "row":
+                    self.cache.Z[lay][upd[1]] = upd[2]
+                else:
+                    self.cache.Z[lay] = upd[1]
+            self.cache.ell = self.ell[kstar]
+
+
+def _chain_ranks(rank, world, n_trials, K, beta):
+    import dataclasses
+    from paper_2607_08406_gb300 import workloads as W
+    from paper_2607_08406_gb300.sharded import ShardedChain
+    wl = W.mlp_small(N=300)
+    wl.domain = dataclasses.replace(wl.domain, beta=beta)
+    shard = OracleShard(wl, np.array_split(np.arange(wl.N), world)[rank])
+    chain = ShardedChain(shard, n_samples=wl.N, K=K)
+    st = chain.run(n_trials, wl.seed)
+    return shard.record, shard.params.flat_eff32(), st
+
+
+@pytest.mark.parametrize("beta", [float("inf"), 400.0])
+def test_sharded_chain_module_over_gloo_ranks(beta):
+    """paper_2607_08406_gb300.sharded.ShardedChain over two gloo ranks (each an oracle shard on half
+    of the samples) follows the single-process oracle's trajectory: greedy (Eq. 6) and Eq. 7 with
+    the chain's whole sample count in the threshold."""
+    import dataclasses
+    from oracle import mca_oracle as O
+    from paper_2607_08406_gb300 import workloads as W
+    from parity import TIE_REL
+    n = 150
+    out = _run(_chain_ranks, 2, n, 16, beta)
+    assert out[0][0] == out[1][0] and np.array_equal(out[0][1], out[1][1])
+    assert out[0][2]["exchanges"] == out[0][2]["batches"] < n
+    wl = W.mlp_small(N=300)
+    dom = dataclasses.replace(wl.domain, beta=beta)
+    tr, params, S = O.run_incremental(wl.layers, wl.loss, wl.X, wl.y, wl.init, n, wl.seed, dom)
+    theta = O.metropolis_threshold(wl.seed, np.arange(n, dtype=np.uint64), beta, wl.N)
+    band = np.abs(tr["dS"] - theta) < TIE_REL * np.abs(tr["S"])
+    rec = out[0][0]
+    assert [r[0] for r in rec] == list(range(n))
+    assert [r[1] for r in rec] == [int(i) for i in tr["idx"]]
+    if beta != float("inf"):
+        assert 0 < int(tr["accept"].sum()) and np.any(tr["accept"] & (tr["dS"] > 0))
+    for (t, idx, acc), oacc, tie in zip(rec, tr["accept"], band):
+        if tie:
+            break                                 # after a tie-band decision the runs may part
+        assert acc == bool(oacc), t
+    else:
+        assert np.array_equal(out[0][1], params.flat_eff32())

@@ -1,68 +1,105 @@
-"""The sample-sharded chain through the C ABI on one GPU (needs a GPU).
+"""The sample-sharded chain (paper_2607_08406_gb300.sharded) through the C ABI (needs a GPU).
 
-The loss is a sum over samples (Eq. 2), so one chain can be split over shards that each hold part
-of the samples: every shard evaluates each candidate of a batch on its own samples, the K partial
-loss changes are exchanged and added in shard order, every shard takes the same decision (Eq. 6)
-and commits the same accepted candidate. Here two handles hold the two halves of a workload's
-samples on one GPU and the host does the exchange (a multi-GPU run would all-gather the K floats);
-nothing on the device waits for another handle. The chain must follow the oracle's single-process
-trajectory, and the two shards must end with the same weights.
+The loss is a sum over samples (Eq. 2), so one chain can be split over ranks that each hold part
+of the samples: every rank evaluates each trial of a batch on its own samples (mca_eval_trials),
+the partial loss changes are all-gathered and added in rank order, every rank takes the same
+decision (mca_decide_batch) and commits it on its shard. Here two ranks are two processes (gloo
+for the exchange) whose handles hold the two halves of a workload's samples on the one GPU;
+nothing on the device waits for another rank. The chain must follow the oracle's single-process
+trajectory, and both shards must end with the same weights.
 """
+import os
+import sys
+
 import numpy as np
 import pytest
 
-from oracle import mca_oracle as O
-from paper_2607_08406_gb300 import workloads as W
-
-from parity import TIE_REL, tie_band
-
 pytestmark = pytest.mark.gpu
 
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+from test_multirank_cpu import _run  # noqa: E402
 
-def test_two_shard_chain_follows_the_single_process_trajectory(gpu_lib):
-    wl = W.make("mlp_wide", N=4000, H=96)
-    n, K, seed = 400, 8, 6
+
+def _workload():
+    from paper_2607_08406_gb300 import workloads as W
+    return W.make("mlp_wide", N=4000, H=96)
+
+
+def _rank(rank, world, n, K, seed, forced):
+    import torch
+    from paper_2607_08406_gb300 import mca
+    from paper_2607_08406_gb300 import workloads as W
+    from paper_2607_08406_gb300.sharded import LibraryShard, ShardedChain
+    torch.cuda.set_device(0)
+    wl = _workload()
+    rows = np.array_split(np.arange(wl.N), world)[rank]
+    sub = W.MLPWorkload(wl.name, wl.layers, wl.loss, np.ascontiguousarray(wl.X[rows]),
+                        np.ascontiguousarray(wl.y[rows]), wl.init, n, K, seed, wl.domain)
+    h = mca.create_from_workload(sub, K=K, trace_cap=n)
+    chain = ShardedChain(LibraryShard(h), n_samples=wl.N, K=K)
+    st = chain.run(n, seed, forced=forced)
+    tr = mca.mca_get_trace(h, n)
+    out = (st, mca.mca_get_params(h, wl.n_params), tr["idx"].astype(np.int64),
+           tr["accept"].astype(bool), mca.mca_loss(h) * len(rows))
+    h.close()
+    return out
+
+
+def test_two_rank_sharded_chain_follows_the_single_process_trajectory(gpu_lib):
+    from oracle import mca_oracle as O
+    from parity import TIE_REL, tie_band
+    wl = _workload()
+    n, K, seed = 400, 16, 6
     tr, params, S = O.run_incremental(wl.layers, wl.loss, wl.X, wl.y, wl.init, n, seed, wl.domain)
     band = tie_band(tr)
-    halves = (slice(0, 2000), slice(2000, 4000))
-    shards = []
-    for hs in halves:
-        sub = W.MLPWorkload(wl.name, wl.layers, wl.loss, np.ascontiguousarray(wl.X[hs]),
-                            np.ascontiguousarray(wl.y[hs]), wl.init, n, K, seed, wl.domain)
-        shards.append(gpu_lib.create_from_workload(sub, K=K))
-    words = O.draw_words(seed, np.arange(n, dtype=np.uint64))
-    P = wl.n_params
-    idx = ((words[:, 0] * np.uint64(P)) >> np.uint64(32)).astype(np.uint32)
-    u = (words[:, 1] >> np.uint64(8)).astype(np.float32) * np.float32(2.0 ** -24)
-    new = (np.float32(-1.0) + np.float32(2.0) * u).astype(np.float32)   # replacement values
-    tau, exchanges = 0, 0
-    while tau < n:
-        kb = min(K, n - tau)
-        part = [gpu_lib.mca_eval_candidates(h, idx[tau:tau + kb], new[tau:tau + kb])
-                for h in shards]
-        exchanges += 1
-        dS = part[0] + part[1]                               # added in shard order
-        kstar, dec = -1, []
-        for k in range(kb):
-            t = tau + k
-            assert abs(dS[k] - tr["dS"][t]) <= TIE_REL * abs(tr["S"][t]), t
-            d = bool(tr["accept"][t]) if band[t] else bool(dS[k] <= 0.0)
-            if not band[t]:
-                assert d == bool(tr["accept"][t]), t
-            dec.append(d)
-            if d:
-                kstar = k
-                break
-        m = kstar + 1 if kstar >= 0 else kb
-        for h in shards:                                     # every shard commits the same way
+    forced = {int(t): bool(a) for t, a in zip(tr["tau"][band], tr["accept"][band])}
+    out = _run(_rank, 2, n, K, seed, forced)
+    (st0, p0, idx0, acc0, S0), (st1, p1, idx1, acc1, S1) = out[0], out[1]
+    assert st0 == st1 and st0["trials"] == n
+    assert st0["exchanges"] == st0["batches"] < n           # batches consumed several trials
+    assert np.array_equal(idx0, tr["idx"]) and np.array_equal(idx1, tr["idx"])
+    assert np.array_equal(acc0, tr["accept"]) and np.array_equal(acc1, tr["accept"])
+    assert np.array_equal(p0, p1) and np.array_equal(p0, params.flat_eff32())
+    assert S0 + S1 == pytest.approx(S, rel=TIE_REL)
+
+
+def test_eval_trials_and_decide_batch_match_the_handles_own_run(gpu_lib):
+    """One handle: mca_eval_trials proposes and evaluates exactly what mca_run would (index, old and
+    new weights, dS of every trial before the first accept), and mca_decide_batch takes mca_run's
+    decision."""
+    from paper_2607_08406_gb300 import workloads as W
+    from parity import TIE_REL
+    for wl in (W.make("mlp_wide", N=3000, H=64), W.make("mlp_ternary", N=3000, H=64),
+               W.make("mlp_deep", N=600, width=40, depth=3)):
+        h = gpu_lib.create_from_workload(wl, K=16, trace_cap=64)
+        h2 = gpu_lib.create_from_workload(wl, K=16, trace_cap=64)
+        tau = 0
+        for _ in range(6):
+            rec = gpu_lib.mca_eval_trials(h, 3, tau, 16)
+            k = gpu_lib.mca_decide_batch(h, 3, tau, rec["valid"], np.nan_to_num(rec["dS"]))
+            m = k + 1 if k >= 0 else 16
+            v = rec["valid"][:m].astype(bool)
+            S = float(rec["S"][0])
+            tie = bool(np.any(np.abs(rec["dS"][:m][v]) < TIE_REL * S))
+            if tie:                                  # either decision is correct: take this one
+                gpu_lib.mca_force_decisions(h2, np.arange(tau, tau + m, dtype=np.uint64),
+                                            (np.arange(m) == k).astype(np.uint8))
+            gpu_lib.mca_run(h2, m, 3)
+            gpu_lib.mca_force_decisions(h2, [], [])
+            g = gpu_lib.mca_get_trace(h2, m)[-m:]
+            assert np.array_equal(g["idx"], rec["idx"][:m])
+            assert np.array_equal(g["old_w"], rec["old_w"][:m])
+            assert np.array_equal(g["new_w"], rec["new_w"][:m])
+            assert np.array_equal(g["valid"], rec["valid"][:m])
+            # the explicit evaluation may add a range's shares in another order than the loop
+            assert np.all(np.abs(g["dS"][v] - rec["dS"][:m][v]) <= TIE_REL * S)
+            assert np.array_equal(g["accept"].astype(bool), np.arange(m) == k)
             gpu_lib.mca_force_decisions(h, np.arange(tau, tau + m, dtype=np.uint64),
-                                        np.array(dec[:m] if kstar >= 0 else [False] * m))
-            st = gpu_lib.mca_run(h, m, seed)
-            assert st["tau"] == tau + m
-        tau += m
-    p0 = gpu_lib.mca_get_params(shards[0], P)
-    assert np.array_equal(p0, gpu_lib.mca_get_params(shards[1], P))
-    assert np.array_equal(p0, params.flat_eff32())
-    assert exchanges < n                                     # batches consumed several trials
-    L = sum(gpu_lib.mca_loss(h) * 2000 for h in shards)
-    assert L == pytest.approx(S, rel=TIE_REL)
+                                        (np.arange(m) == k).astype(np.uint8))
+            gpu_lib.mca_run(h, m, 3)
+            gpu_lib.mca_force_decisions(h, [], [])
+            tau += m
+        assert np.array_equal(gpu_lib.mca_get_params(h, wl.n_params),
+                              gpu_lib.mca_get_params(h2, wl.n_params))
+        h.close()
+        h2.close()
