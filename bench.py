@@ -31,11 +31,11 @@ sys.path.insert(0, ROOT)
 METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roofline"
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the trial-loop kernel per trial,
-# from the ncu launch list of `python bench.py --steps 3 --warmup 3 --no-e2e --no-cpu` summarised in
-# profiles/. It is only valid for the kernel source it was measured on; any other source hash
-# reports null.
-LOOP_TRAFFIC = {"source_sha1": "4e88068a1e68ea52e4b82a19ac9993baaf728611",
-                "bytes_per_trial": 359559.0}
+# from one ncu capture (one pass, one launch: the first timed step, trials 200k..240k) of
+# `python bench.py --steps 20 --warmup 5 --no-e2e --no-cpu`, summarised in profiles/. It is only
+# valid for the kernel source it was measured on; any other source hash reports null.
+LOOP_TRAFFIC = {"source_sha1": "d226e40a5b6369a5b1cfa03226a2bb7319f8dc8f",
+                "bytes_per_trial": 374000.0}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
 
