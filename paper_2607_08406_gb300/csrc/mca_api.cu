@@ -76,8 +76,8 @@ bool is_device_ptr(const void* p) {
 
 struct Layout {
   size_t XT, y, xs_off, xs_n, xs_v, xs_sect, xs_roff, z1, srec, partial, accum, bar, st, trace,
-      ex_idx, ex_new, ex_out, prop, scratch, ell, ctl, gimg, total;
-  std::vector<size_t> w_eff, code, wfix, Z, whi;
+      ex_idx, ex_new, ex_out, prop, scratch, ell, ctl, gimg, scr_tab, total;
+  std::vector<size_t> w_eff, code, wfix, Z, whi, scr;
 };
 
 bool is_deep(const std::vector<mca_layer>& layers) { return layers.size() > 2; }
@@ -92,6 +92,11 @@ bool deep_tc_ok(const std::vector<mca_layer>& layers) {
   return true;
 }
 int deep_tc_tiles(long long N) { return (int)((N + mca::kTcTS - 1) / mca::kTcTS); }
+
+// Candidate scratch slots of the deep tensor-core path (min(K, kDeepScrSlots)); none elsewhere.
+int deep_scratch_slots(const std::vector<mca_layer>& layers, int K) {
+  return deep_tc_ok(layers) ? std::min(K, mca::kDeepScrSlots) : 0;
+}
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
 
@@ -123,7 +128,7 @@ size_t forward_tc_image_bytes(const std::vector<mca_layer>& layers, int Np) {
 // Device memory of a handle. Single hidden layer: feature CSR of X, z1, sample records, per-range
 // partials. Deep: the fields of every layer, per-sample losses, per-tile partials.
 Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long nnz, int trace_cap,
-            int NR) {
+            int NR, int nscr) {
   const bool deep = is_deep(layers);
   Layout L;
   size_t o = 0;
@@ -175,6 +180,14 @@ Layout plan(const std::vector<mca_layer>& layers, long long N, int D, long long 
   L.scratch = take(sizeof(int) * (size_t)(D + 8));
   const size_t gb = forward_tc_image_bytes(layers, Np);
   L.gimg = gb ? take(gb) : SIZE_MAX;
+  L.scr_tab = SIZE_MAX;
+  if (deep && nscr > 0) {
+    L.scr_tab = take(sizeof(float*) * (size_t)nscr * (layers.size() + 1));
+    for (int k = 0; k < nscr; ++k) {
+      for (const auto& ly : layers) L.scr.push_back(take(sizeof(float) * (size_t)ly.n_out * Np));
+      L.scr.push_back(take(sizeof(float) * (size_t)Np));
+    }
+  }
   L.total = o;
   return L;
 }
@@ -731,7 +744,7 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
   if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
   const mca_options o = opt ? *opt : default_options();
   if (is_deep(ls)) {
-    *bytes = plan(ls, data->n, data->d, 0, o.trace_cap, 0).total;
+    *bytes = plan(ls, data->n, data->d, 0, o.trace_cap, 0, deep_scratch_slots(ls, o.K)).total;
     return MCA_OK;
   }
   long long nnz = 0;
@@ -740,7 +753,7 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
   Ranges R;
   rc = choose_ranges(ls, loss, data->n, o.grid, &R);
   if (rc != MCA_OK) return rc;
-  *bytes = plan(ls, data->n, data->d, nnz, o.trace_cap, R.NR).total;
+  *bytes = plan(ls, data->n, data->d, nnz, o.trace_cap, R.NR, deep_scratch_slots(ls, o.K)).total;
   return MCA_OK;
 }
 
@@ -833,7 +846,8 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     h->smem_records = R.smem_records;
     h->window = R.window;
   }
-  const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap, h->NR);
+  h->nscr = h->deep ? deep_scratch_slots(ls, o.K) : 0;
+  const Layout L = plan(ls, h->N, h->D, h->nnz, o.trace_cap, h->NR, h->nscr);
   if (o.workspace) {
     if (o.workspace_bytes < L.total)
       return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
@@ -868,6 +882,13 @@ mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
     h->ell = reinterpret_cast<float*>(base + L.ell);
     h->ctl = reinterpret_cast<mca::DeepCtl*>(base + L.ctl);
     CTRY(cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream));
+    if (h->nscr > 0) {
+      for (size_t q = 0; q < L.scr.size(); ++q)
+        h->scr.push_back(reinterpret_cast<float*>(base + L.scr[q]));
+      h->scr_dev = reinterpret_cast<float**>(base + L.scr_tab);
+      CTRY(cudaMemcpyAsync(h->scr_dev, h->scr.data(), sizeof(float*) * h->scr.size(),
+                           cudaMemcpyHostToDevice, h->stream));
+    }
   } else {
     h->z1 = reinterpret_cast<float*>(base + L.z1);
     h->srec = reinterpret_cast<float*>(base + L.srec);
@@ -989,10 +1010,14 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
       } else {
         a.tau = h->tau;
         a.Kb = (int)kb;
+        a.scr = h->scr_dev;
+        a.nscr = h->nscr;
         CUDA_TRY(h, mca::launch_deep_eval(a, h->stream));
         CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_deep_decide(a, h->stream));
-        CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+        // with scratch slots the commit follows the decision on the host (below)
+        if (h->nscr == 0) CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+        else h->launches -= 1;
       }
       CUDA_TRY(h, cudaEventRecord(h->ev[2], h->stream));
       h->launches += 3;
@@ -1000,15 +1025,57 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
       CUDA_TRY(h, cudaMemcpyAsync(&ctl, h->ctl, sizeof(ctl), cudaMemcpyDeviceToHost, h->stream));
       CUDA_TRY(h, cudaStreamSynchronize(h->stream));
       {
-        float ms_eval = 0.0f, ms_rest = 0.0f;
+        float ms_eval = 0.0f, ms_rest = 0.0f, ms_c = 0.0f;
         CUDA_TRY(h, cudaEventElapsedTime(&ms_eval, h->ev[0], h->ev[1]));
         CUDA_TRY(h, cudaEventElapsedTime(&ms_rest, h->ev[1], h->ev[2]));
+        if (h->ev_c_pending) {             // the previous batch's adoption or commit
+          CUDA_TRY(h, cudaEventElapsedTime(&ms_c, h->ev_c[0], h->ev_c[1]));
+          h->ev_c_pending = false;
+        }
         h->eval_ns += (uint64_t)(ms_eval * 1e6f);
-        h->rest_ns += (uint64_t)(ms_rest * 1e6f);
+        h->rest_ns += (uint64_t)((ms_rest + ms_c) * 1e6f);
       }
       if (ctl.kstar == -2 || ctl.consumed <= 0) {
         h->broken = true;
         return fail(h, MCA_ERR_NUMERIC, "non-finite loss change");
+      }
+      if (!h->tfm && h->nscr > 0 && ctl.kstar >= 0) {
+        // The accepted candidate's fields: adopted from its scratch slot (row j of its layer
+        // copied, the later layers' arrays and the losses swapped with the slot's), or, for a
+        // candidate without a dense chain or beyond the slots, recomputed by the commit kernel.
+        if (!h->ev_c[0]) {
+          for (auto& e : h->ev_c) CUDA_TRY(h, cudaEventCreate(&e));
+        }
+        CUDA_TRY(h, cudaEventRecord(h->ev_c[0], h->stream));
+        const mca::DeepCand& c = ctl.acc;
+        const int L = (int)h->layers.size();
+        if (ctl.kstar < h->nscr && c.valid && c.delta != 0.0f && c.layer <= L - 3) {
+          float** sk = h->scr.data() + (size_t)ctl.kstar * (L + 1);
+          const size_t row = (size_t)c.row * h->Np;
+          CUDA_TRY(h, cudaMemcpyAsync(h->Z[c.layer] + row, sk[c.layer] + row,
+                                      sizeof(float) * (size_t)h->N, cudaMemcpyDeviceToDevice,
+                                      h->stream));
+          for (int m = c.layer + 1; m < L; ++m) std::swap(h->Z[m], sk[m]);
+          std::swap(h->ell, sk[L]);
+          CUDA_TRY(h, cudaMemcpyAsync(h->scr_dev + (size_t)ctl.kstar * (L + 1), sk,
+                                      sizeof(float*) * (size_t)(L + 1), cudaMemcpyHostToDevice,
+                                      h->stream));
+          const uint64_t sd = a.seed;
+          a = deep_args(h);
+          a.seed = sd;
+        } else {
+          CUDA_TRY(h, mca::launch_deep_commit(a, h->stream));
+          h->launches += 1;
+        }
+        CUDA_TRY(h, cudaEventRecord(h->ev_c[1], h->stream));
+        h->ev_c_pending = true;
+        if (remaining == (uint64_t)ctl.consumed) {   // the run's last batch: its time now
+          float ms_c = 0.0f;
+          CUDA_TRY(h, cudaEventSynchronize(h->ev_c[1]));
+          CUDA_TRY(h, cudaEventElapsedTime(&ms_c, h->ev_c[0], h->ev_c[1]));
+          h->rest_ns += (uint64_t)(ms_c * 1e6f);
+          h->ev_c_pending = false;
+        }
       }
       h->tau += (uint64_t)ctl.consumed;
       remaining -= (uint64_t)ctl.consumed;
@@ -1547,6 +1614,8 @@ void mca_destroy(mca_handle* h) {
   if (!h) return;
   cudaStreamSynchronize(h->stream);
   for (auto& e : h->ev)
+    if (e) cudaEventDestroy(e);
+  for (auto& e : h->ev_c)
     if (e) cudaEventDestroy(e);
   if (h->ws_owned && h->ws) cudaFree(h->ws);
   if (h->ftau) cudaFree(h->ftau);

@@ -2,23 +2,29 @@
 //   Z'_m = Z_m + W_m (f(Z'_{m-1}) - f(Z_{m-1})),   m = l+2 .. L-2   (Section 2.4),
 // as error-compensated 3xTF32 tcgen05 MMAs with the accumulator in tensor memory.
 //
-// One CTA per (candidate, tile of kTcTS = 128 samples), 512 threads. Per dense layer the CTA computes
-// the transposed change D^T[samples x 256] = A[samples x 256] W_m^T, where A holds the previous
-// layer's activation changes split as A = A_hi + A_lo (each rounded to tf32) and W_m = W_hi + W_lo
-// (kept split in global memory, updated with every commit):
+// One CTA per (candidate, tile of kTcTS = 128 samples): 16 worker warps and one control warp. Per
+// dense layer the CTA computes the transposed change D^T[samples x 256] = A[samples x 256] W_m^T,
+// where A holds the previous layer's activation changes split as A = A_hi + A_lo (each rounded to
+// tf32) and W_m = W_hi + W_lo (kept split in global memory, updated with every commit):
 //   D = A_lo W_hi^T + A_hi W_lo^T + A_hi W_hi^T      (the A_lo W_lo^T term, ~2^-22 relative, dropped)
-// Tensor memory (512 columns): D in columns [0, 256) (lane = sample, column = output feature),
-// A_hi in columns [256, 512) (the A operand of two of the three MMAs). A_lo lives in shared memory
-// (128 KB); W streams through three 32 KB stages of 16-wide K chunks (hi + lo), each filled by one
-// bulk copy, in a ring run by one thread (full / empty mbarriers) that reaches across layer
-// boundaries. All operands are K-major without swizzle: 8-row x 16-byte core matrices.
 //
-// The epilogue (all 16 warps; warp w reads tensor-memory lanes 32 (w mod 4) .. + 31 and a quarter of
-// the features) adds D to the cached fields, forms the next activation change f(z') - f(z) (exactly 0
-// where a field did not change), and writes its hi part to tensor memory and its lo part to shared
-// memory for the next layer; after the last dense layer it accumulates the output layer instead.
-// Every per-(candidate, tile) loss change depends only on that pair: the trajectory does not depend
-// on the batch width. COMMIT writes the fields exactly as the evaluation computed them.
+// The layers are pipelined chunk by chunk. The workers produce A in K chunks of 16 features (hi and
+// lo, 16 KB) into a ring of four shared-memory slots; the control thread issues each chunk's six
+// MMAs as soon as the chunk and its weight stage are there, so layer m+1's MMAs run while the
+// workers are still forming layer m's later chunks. Two accumulators in tensor memory (columns
+// [0, 256) and [256, 512)) alternate by layer: the workers read layer m's finished D while the
+// MMAs of layer m+1 fill the other one. W streams through four 32 KB stages of 16-wide K chunks
+// (hi + lo), each one bulk copy, reaching across layer boundaries. All operands are K-major without
+// swizzle: 8-row x 16-byte core matrices.
+//
+// Worker warp w reads tensor-memory lanes 32 (w mod 4) .. + 31 (its samples) and, in every chunk,
+// the four features 4 (w / 4) .. + 3: the cached field + D gives the new field, the next activation
+// change f(z') - f(z) (exactly 0 where a field did not change) goes into the ring, and after the
+// last dense layer the changes accumulate into the output layer instead. Every per-(candidate,
+// tile) loss change depends only on that pair: the trajectory does not depend on the batch width.
+// COMMIT writes the fields exactly as the evaluation computed them. Every wait is bounded (2 s); on a
+// time-out the CTA records MCA_ERR_TIMEOUT, lets its issued copies and MMAs complete (bounded) and
+// frees its tensor memory.
 #include <cstdio>
 
 #include "mca_deep.cuh"
@@ -29,66 +35,106 @@
 namespace mca {
 namespace {
 
-constexpr int kTcThreads = 512;
-constexpr int kParts = kTcThreads / 128;     // feature parts per sample (warps sharing a lane quarter)
-constexpr int kTcW = 256;                  // width of the dense layers
-constexpr int kPartW = kTcW / kParts;
-constexpr int kTcKC = 16;                  // K chunk of a W stage
+constexpr int kWorkWarps = 16;
+constexpr int kTcThreads = (kWorkWarps + 1) * 32;   // + one control warp
+constexpr int kCtl = kWorkWarps * 32;                // the control thread
+constexpr int kParts = 4;                            // feature parts per lane quarter
+constexpr int kTcW = 256;                            // width of the dense layers
+constexpr int kTcKC = 16;                            // K chunk
 constexpr int kTcChunks = kTcW / kTcKC;
-constexpr int kAloBytes = kTcTS * kTcW * 4;          // 128 KB
-constexpr int kWHalfBytes = kTcW * kTcKC * 4;        // 16 KB: one of hi / lo of one chunk
+constexpr int kAHalf = kTcTS * kTcKC * 4;            // 8 KB: hi or lo of one A chunk
+constexpr int kASlot = 2 * kAHalf;
+constexpr int kASlots = 4;
+constexpr int kWHalfBytes = kTcW * kTcKC * 4;        // 16 KB: hi or lo of one W chunk
 constexpr int kWStageBytes = 2 * kWHalfBytes;        // 32 KB
-constexpr int kStages = 3;
-constexpr int kTcSmem = kAloBytes + kStages * kWStageBytes;
-// core-matrix strides (bytes): A_lo: K groups 2 KB apart, sample groups 128 B apart;
+constexpr int kStages = 4;
+constexpr int kTcSmem = kASlots * kASlot + kStages * kWStageBytes;
+// core-matrix strides (bytes): A chunk: K groups 2 KB apart, sample groups 128 B apart;
 // W stage: K groups 4 KB apart, row groups 128 B apart. The split weights of a layer are kept in
 // global memory as kTcChunks consecutive 32 KB stage images (hi then lo), so that one bulk copy
 // fills a stage.
-constexpr uint32_t kAloLBO = (kTcTS / 8) * 128, kAloSBO = 128;
+constexpr uint32_t kALBO = (kTcTS / 8) * 128, kASBO = 128;
 constexpr uint32_t kWLBO = (kTcW / 8) * 128, kWSBO = 128;
 // kind::tf32, D fp32, A and B tf32 K-major, M = 128, N = 256
 constexpr uint32_t kIdesc = tc_idesc_tf32(kTcTS, kTcW);
 
 static_assert(kTcSmem + 2048 <= 227 * 1024, "shared memory of the chain kernel");
+static_assert((kParts - 1) * kMaxC * kTcTS * 4 <= kStages * kWStageBytes, "output scratch");
 
 // One thread: stage st <- the 32 KB image of one chunk, completion counted on mbarrier full.
 __device__ __forceinline__ void load_stage(uint32_t dst, const void* src, uint64_t* full) {
   bulk_load(dst, src, (uint32_t)kWStageBytes, full);
 }
 
-// A_lo element (sample s, feature k) in shared memory: 16 consecutive features of one sample as
-// four 16-byte stores.
-__device__ __forceinline__ void store_alo16(unsigned char* alo, int s, int f0, const float (&v)[16]) {
-#pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const int k = f0 + 4 * g;
-    *reinterpret_cast<float4*>(alo + (size_t)(k >> 2) * kAloLBO + (size_t)s * 16) =
-        make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
-  }
-}
-
 __device__ __forceinline__ void prefetch_l2(const void* p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
 
-// Field rows of one layer for this tile into L2 (thread t: row t, four 128-byte lines).
-__device__ __forceinline__ void prefetch_tile(const float* Zm, int Np, int n0, int tid) {
+// Field rows of one layer for this tile into L2: worker thread t, row t / 2, two 128-byte lines.
+__device__ __forceinline__ void prefetch_tile(const float* Zm, int Np, int n0, int t) {
+  const float* r = Zm + (size_t)(t >> 1) * Np + n0 + 64 * (t & 1);
+  prefetch_l2(r);
+  prefetch_l2(r + 32);
+}
+
+// Four accumulator columns of this thread's lane into r, left in flight: the values may be read only
+// after tmem_wait4(r).
+__device__ __forceinline__ void tmem_issue4(uint32_t taddr, uint32_t (&r)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(taddr) : "memory");
+}
+
+// Wait for this thread's tensor-memory loads; r is tied to the wait so that no read of it moves
+// above it.
+__device__ __forceinline__ void tmem_wait4(uint32_t (&r)[4]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]) :: "memory");
+}
+
+// Every lane waits for the phase; true in every lane iff no lane timed out.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity) ? 1 : 0) != 0;
+}
+
+// Worker: put four activation changes of sample s (features 4 fp .. + 3 of the chunk) into ring
+// slot ga % kASlots as hi and lo tf32 parts, once the MMAs of the chunk kASlots earlier are done
+// with the slot; then the warp's arrival on the slot's full barrier.
+__device__ __forceinline__ bool produce_chunk(unsigned char* aring, uint64_t* afull,
+                                              uint64_t* aempty, int ga, int fp, int s,
+                                              const float (&d)[4]) {
+  const int as = ga % kASlots;
+  if (ga >= kASlots && !warp_wait(&aempty[as], (uint32_t)((ga / kASlots) - 1) & 1u)) return false;
+  float hi[4], lo[4];
 #pragma unroll
-  for (int p = 0; p < kTcTS / 32; ++p) prefetch_l2(Zm + (size_t)tid * Np + n0 + 32 * p);
+  for (int q = 0; q < 4; ++q) {
+    hi[q] = tf32_rna(d[q]);
+    lo[q] = tf32_rna(d[q] - hi[q]);
+  }
+  unsigned char* slot = aring + (size_t)as * kASlot + (size_t)fp * kALBO + (size_t)s * 16;
+  *reinterpret_cast<float4*>(slot) = make_float4(hi[0], hi[1], hi[2], hi[3]);
+  *reinterpret_cast<float4*>(slot + kAHalf) = make_float4(lo[0], lo[1], lo[2], lo[3]);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  tc_fence_before();
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0)
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&afull[as])) : "memory");
+  return true;
 }
 
 // ACTH: transfer function of the hidden layers (-1: read per layer at run time).
 template <bool COMMIT, int ACTH>
 __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a) {
   extern __shared__ __align__(1024) unsigned char tsm[];
-  unsigned char* alo = tsm;                                   // A_lo
-  unsigned char* wst = tsm + kAloBytes;                       // W stages
+  unsigned char* aring = tsm;                                 // A chunks
+  unsigned char* wst = tsm + kASlots * kASlot;                // W stages
   __shared__ DeepCand s_cand;
   __shared__ float s_da[kTcTS];
   __shared__ float s_red[32];
-  __shared__ __align__(8) uint64_t s_full[kStages], s_empty[kStages];
+  __shared__ __align__(8) uint64_t s_wfull[kStages], s_wempty[kStages];
+  __shared__ __align__(8) uint64_t s_afull[kASlots], s_aempty[kASlots];
+  __shared__ __align__(8) uint64_t s_dfull[2], s_drain;
   __shared__ uint32_t s_tmem;
-  __shared__ int s_fail;
+  __shared__ volatile int s_fail;
   __shared__ int s_k;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int k = 0, tile = COMMIT ? blockIdx.x : 0;
@@ -128,8 +174,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
   const int L = a.L, l = c.layer, j = c.row, i = c.col;
   const int Np = a.Np, N = a.N;
   float dl = 0.0f;
-  if (l + 1 < L - 1 && a.n_out[l + 1] == kTcW && tid < kTcW)
-    prefetch_tile(a.Z[l + 1], Np, n0, tid);
+  // this candidate's scratch slot, when it has one and a dense chain (layer <= L-3)
+  float* const* sk = (!COMMIT && k < a.nscr && l <= L - 3) ? a.scr + (size_t)k * (L + 1) : nullptr;
+  if (l + 1 < L - 1 && a.n_out[l + 1] == kTcW && tid < kCtl) prefetch_tile(a.Z[l + 1], Np, n0, tid);
 
   // ---- row j of layer l (thread s = sample)
   if (tid < kTcTS) {
@@ -153,6 +200,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
       } else {
         da = act_rt(a.act[l], zn, a.g[l]) - act_rt(a.act[l], z, a.g[l]);
         if (COMMIT) *zp = zn;
+        if (sk) sk[l][(size_t)j * Np + n] = zn;
       }
     }
     s_da[tid] = da;
@@ -183,9 +231,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
     }
   } else if (l < L - 2) {
     const bool dense = l + 2 <= L - 2;
-    const int qd = warp & 3, hf = warp >> 2;         // lane quarter, feature part
+    const int nd = dense ? (L - 2) - (l + 2) + 1 : 0;      // dense layers of the chain
+    const int nchunks = nd * kTcChunks;
+    const bool worker = warp < kWorkWarps;
+    const int qd = warp & 3, fp = (warp >> 2) & 3;        // lane quarter, feature part
     const int s = qd * 32 + lane, n = n0 + s;
-    const bool live = n < N;
+    const bool live = worker && n < N;
     const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
     uint32_t tmem = 0;
     if (dense) {
@@ -194,181 +245,244 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
                      ::"r"(smem_u32(&s_tmem)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
       }
-      if (tid == 0) {
+      if (tid == kCtl) {
         for (int q = 0; q < kStages; ++q) {
-          asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_full[q])));
-          asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&s_empty[q])));
+          mbar_init(&s_wfull[q], 1);
+          mbar_init(&s_wempty[q], 1);
         }
+        for (int q = 0; q < kASlots; ++q) {
+          mbar_init(&s_afull[q], kWorkWarps);
+          mbar_init(&s_aempty[q], 1);
+        }
+        mbar_init(&s_dfull[0], 1);
+        mbar_init(&s_dfull[1], 1);
+        mbar_init(&s_drain, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        // the first two chunks of the first dense layer load during the rank-1 step
+        // the first weight chunks of the first dense layer load during the rank-1 step
         const unsigned char* w0 = reinterpret_cast<const unsigned char*>(a.whi[l + 2]);
         const uint32_t sw0 = smem_u32(wst);
-        for (int q = 0; q < kStages - 1 && q < (L - 2 - (l + 2) + 1) * kTcChunks; ++q)
-          load_stage(sw0 + (uint32_t)(q * kWStageBytes), w0 + (size_t)q * kWStageBytes, &s_full[q]);
+        for (int q = 0; q < kStages - 1 && q < nchunks; ++q)
+          load_stage(sw0 + (uint32_t)(q * kWStageBytes), w0 + (size_t)q * kWStageBytes, &s_wfull[q]);
       }
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      tc_fence_before();
       __syncthreads();
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      tc_fence_after();
       tmem = s_tmem;
     }
-    // output-layer accumulation of this thread's feature half (after the last change matrix)
     float outp[kMaxC];
 #pragma unroll
     for (int q = 0; q < kMaxC; ++q) outp[q] = 0.0f;
     const float* Wout = a.w[L - 1];
     const int Kout = a.n_in[L - 1];
 
-    // ---- layer l+1: rank-1 change through column j of W_{l+1}; its activation change is the
-    // first A (dense) or feeds the output layer directly (l = L-3)
-    {
-      const int m1 = l + 1;
-      const float* W1 = a.w[m1];
-      const int K1 = a.n_in[m1];
-      const float da = s_da[s];
-      float* Zm = a.Z[m1];
-      const bool moves = live && da != 0.0f;
-      for (int f0 = hf * kPartW; f0 < (hf + 1) * kPartW; f0 += 16) {
-        float hi[16], lo[16], zo[16], wv[16];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {          // loads first (n < Np: always in the array)
-          wv[q] = W1[(size_t)(f0 + q) * K1 + j];
-          zo[q] = Zm[(size_t)(f0 + q) * Np + n];
-        }
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const int f = f0 + q;
-          const float zn = fmaf(wv[q], da, zo[q]);
-          const bool ch = moves && zn != zo[q];
-          const float an = act<ACTH>(zn, a.g[m1], a.act[m1]);
-          const float ao = act<ACTH>(zo[q], a.g[m1], a.act[m1]);
-          const float d = ch ? an - ao : 0.0f;
-          if (COMMIT && ch) Zm[(size_t)f * Np + n] = zn;
-          if (dense) {
-            hi[q] = tf32_rna(d);
-            lo[q] = tf32_rna(d - hi[q]);
-          } else {
-#pragma unroll
-            for (int o = 0; o < kMaxC; ++o)
-              if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f], d, outp[o]);
+    if (!worker) {
+      // ---- control thread: every dense layer's MMAs, chunk by chunk as the workers produce A
+      if (dense && lane == 0) {
+        const uint32_t sw = smem_u32(wst), sa = smem_u32(aring);
+        int issued_w = kStages - 1 < nchunks ? kStages - 1 : nchunks;   // weight chunks requested
+        int landed_w = 0;                                               // ... and waited for
+        bool ok = true;
+        for (int gc = 0; gc < nchunks && ok; ++gc) {
+          const int li = gc / kTcChunks, cc = gc % kTcChunks;
+          const int as = gc % kASlots, st = gc % kStages;
+          if (!mbar_wait(&s_wfull[st], (uint32_t)(gc / kStages) & 1u)) {
+            ok = false;
+            break;
           }
-        }
-        if (dense) {
-          tmem_st16(tmem + lane_base + 256u + (uint32_t)f0, hi);
-          store_alo16(alo, s, f0, lo);
-        }
-      }
-    }
-
-    // ---- dense layers m = l+2 .. L-2 on the tensor cores
-    if (dense) {
-      const uint32_t sw = smem_u32(wst), salo = smem_u32(alo);
-      const int nchunks = (L - 2 - (l + 2) + 1) * kTcChunks;   // chunks of all dense layers
-      for (int m = l + 2; m <= L - 2; ++m) {
-        const int li = m - (l + 2);
-        if (tid < kTcW) prefetch_tile(a.Z[m], Np, n0, tid);
-        // the previous step's A (tensor memory, shared memory) complete before the MMAs read it
-        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();
-        if (tid == 0) {
-          // one thread: wait for a chunk, issue its MMAs, release its stage, refill two ahead
-          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-          for (int cidx = 0; cidx < kTcChunks; ++cidx) {
-            const int gc = li * kTcChunks + cidx, st = gc % kStages;
-            if (!mbar_wait(&s_full[st], (uint32_t)(gc / kStages) & 1u)) {
-              s_fail = 1;
+          landed_w = gc + 1;
+          if (!mbar_wait(&s_afull[as], (uint32_t)(gc / kASlots) & 1u)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dt = tmem + (uint32_t)(li & 1) * 256u;
+#pragma unroll
+          for (int ks = 0; ks < kTcKC / 8; ++ks) {
+            const uint32_t ab = sa + (uint32_t)(as * kASlot) + (uint32_t)ks * 2u * kALBO;
+            const uint32_t wb = sw + (uint32_t)(st * kWStageBytes) + (uint32_t)ks * 2u * kWLBO;
+            const uint64_t dahi = umma_desc(ab, kALBO, kASBO);
+            const uint64_t dalo = umma_desc(ab + kAHalf, kALBO, kASBO);
+            const uint64_t dwhi = umma_desc(wb, kWLBO, kWSBO);
+            const uint64_t dwlo = umma_desc(wb + kWHalfBytes, kWLBO, kWSBO);
+            mma_ss(dt, dalo, dwhi, kIdesc, (cc > 0 || ks > 0) ? 1u : 0u);
+            mma_ss(dt, dahi, dwlo, kIdesc, 1u);
+            mma_ss(dt, dahi, dwhi, kIdesc, 1u);
+          }
+          umma_commit(&s_aempty[as]);
+          umma_commit(&s_wempty[st]);
+          if (cc == kTcChunks - 1) umma_commit(&s_dfull[li & 1]);
+          // chunk gc + kStages - 1 goes to the stage chunk gc - 1 used, once its MMAs are done
+          const int nc = gc + kStages - 1;
+          if (nc < nchunks) {
+            const int ns = nc % kStages;
+            if (gc >= 1 && !mbar_wait(&s_wempty[ns], (uint32_t)((gc - 1) / kStages) & 1u)) {
+              ok = false;
               break;
             }
-#pragma unroll
-            for (int ks = 0; ks < kTcKC / 8; ++ks) {
-              const int g = cidx * (kTcKC / 8) + ks;       // K step of 8 over the layer
-              const uint64_t dalo = umma_desc(salo + (uint32_t)g * 2u * kAloLBO, kAloLBO, kAloSBO);
-              const uint32_t wb = sw + (uint32_t)(st * kWStageBytes) + (uint32_t)ks * 2u * kWLBO;
-              const uint64_t dwhi = umma_desc(wb, kWLBO, kWSBO);
-              const uint64_t dwlo = umma_desc(wb + kWHalfBytes, kWLBO, kWSBO);
-              const uint32_t tahi = tmem + 256u + (uint32_t)(g * 8);
-              mma_ss(tmem, dalo, dwhi, kIdesc, g > 0 ? 1u : 0u);
-              mma_ts(tmem, tahi, dwlo, kIdesc, 1u);
-              mma_ts(tmem, tahi, dwhi, kIdesc, 1u);
-            }
-            umma_commit(&s_empty[st]);
-            // chunk gc + 2 goes to the stage chunk gc - 1 used, once its MMAs are done
-            const int nc = gc + kStages - 1;
-            if (nc < nchunks) {
-              const int ns = nc % kStages;
-              if (gc >= 1 && !mbar_wait(&s_empty[ns], (uint32_t)((gc - 1) / kStages) & 1u)) {
-                s_fail = 1;
-                break;
-              }
-              const int nl = l + 2 + nc / kTcChunks, nci = nc % kTcChunks;
-              load_stage(sw + (uint32_t)(ns * kWStageBytes),
-                         reinterpret_cast<const unsigned char*>(a.whi[nl]) +
-                             (size_t)nci * kWStageBytes,
-                         &s_full[ns]);
-            }
+            const int nl = l + 2 + nc / kTcChunks, nci = nc % kTcChunks;
+            load_stage(sw + (uint32_t)(ns * kWStageBytes),
+                       reinterpret_cast<const unsigned char*>(a.whi[nl]) +
+                           (size_t)nci * kWStageBytes,
+                       &s_wfull[ns]);
+            issued_w = nc + 1;
           }
         }
-        // every MMA of the layer done: the last chunk's commit (commits complete in order)
-        {
-          const int gl = li * kTcChunks + kTcChunks - 1;
-          if (!mbar_wait(&s_empty[gl % kStages], (uint32_t)(gl / kStages) & 1u)) s_fail = 1;
+        if (!ok) s_fail = 1;
+        // drain: every MMA issued above complete, every requested weight chunk landed
+        umma_commit(&s_drain);
+        if (!mbar_wait(&s_drain, 0u)) s_fail = 1;
+        for (int q = landed_w; q < issued_w; ++q)
+          if (!mbar_wait(&s_wfull[q % kStages], (uint32_t)(q / kStages) & 1u)) s_fail = 1;
+      }
+    } else {
+      // ---- workers
+      bool ok = true;
+      int ga = 0;                                         // A chunks produced
+      float zo_n[4];                                      // cached fields one chunk ahead
+      if (dense) prefetch_tile(a.Z[l + 2], Np, n0, tid);
+      // layer l+1: rank-1 change through column j of W_{l+1}; its activation change is the first
+      // A (dense) or feeds the output layer directly (l = L-3)
+      {
+        const int m1 = l + 1;
+        const float* W1 = a.w[m1];
+        const int K1 = a.n_in[m1];
+        const float da = s_da[s];
+        float* Zm = a.Z[m1];
+        const bool moves = live && da != 0.0f;
+        // loads one chunk ahead of their use (n < Np: always in the array)
+        float wv[4], zo[4], wv_n[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          wv_n[q] = W1[(size_t)(fp * 4 + q) * K1 + j];
+          zo_n[q] = Zm[(size_t)(fp * 4 + q) * Np + n];
         }
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        __syncthreads();
-        if (s_fail) break;                            // the same value in every thread here
-
-        // epilogue: new fields, the next A (or the output layer after the last dense layer)
+        for (int cc = 0; cc < kTcChunks; ++cc) {
+          const int f0 = cc * kTcKC + fp * 4;
+          float d[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            wv[q] = wv_n[q];
+            zo[q] = zo_n[q];
+          }
+          if (cc + 1 < kTcChunks) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              wv_n[q] = W1[(size_t)(f0 + kTcKC + q) * K1 + j];
+              zo_n[q] = Zm[(size_t)(f0 + kTcKC + q) * Np + n];
+            }
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float zn = fmaf(wv[q], da, zo[q]);
+            const bool ch = moves && zn != zo[q];
+            const float an = act<ACTH>(zn, a.g[m1], a.act[m1]);
+            const float ao = act<ACTH>(zo[q], a.g[m1], a.act[m1]);
+            d[q] = ch ? an - ao : 0.0f;
+            if (COMMIT && ch) Zm[(size_t)(f0 + q) * Np + n] = zn;
+            if (sk) sk[m1][(size_t)(f0 + q) * Np + n] = ch ? zn : zo[q];
+          }
+          if (dense) {
+            if (!produce_chunk(aring, s_afull, s_aempty, ga, fp, s, d)) {
+              ok = false;
+              break;
+            }
+            ++ga;
+          } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+#pragma unroll
+              for (int o = 0; o < kMaxC; ++o)
+                if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f0 + q], d[q], outp[o]);
+          }
+        }
+      }
+      // dense layers m = l+2 .. L-2: read D of layer m as its MMAs finish, form the next A
+      if (dense) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) zo_n[q] = a.Z[l + 2][(size_t)(fp * 4 + q) * Np + n];
+      }
+      for (int li = 0; li < nd && ok; ++li) {
+        const int m = l + 2 + li;
         const bool last = m == L - 2;
+        if (!last) prefetch_tile(a.Z[m + 1], Np, n0, tid);
+        if (!warp_wait(&s_dfull[li & 1], (uint32_t)(li >> 1) & 1u)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
         float* Zm = a.Z[m];
-        for (int f0 = hf * kPartW; f0 < (hf + 1) * kPartW; f0 += 16) {
-          float zo[16];
+        const uint32_t dt = tmem + lane_base + (uint32_t)(li & 1) * 256u;
+        // accumulator columns one chunk ahead: chunk cc + 1's load is in flight while chunk cc is
+        // processed
+        uint32_t dr[4], dr_n[4];
+        tmem_issue4(dt + (uint32_t)(fp * 4), dr_n);
+        tmem_wait4(dr_n);
+        for (int cc = 0; cc < kTcChunks; ++cc) {
+          const int f0 = cc * kTcKC + fp * 4;
+          float zo[4], dv[4], d[4];
 #pragma unroll
-          for (int q = 0; q < 16; ++q) zo[q] = Zm[(size_t)(f0 + q) * Np + n];
-          float dv[16];
-          tmem_ld16(tmem + lane_base + (uint32_t)f0, dv);
-          float hi[16], lo[16];
+          for (int q = 0; q < 4; ++q) {
+            dr[q] = dr_n[q];
+            dv[q] = __uint_as_float(dr[q]);
+          }
+          if (cc + 1 < kTcChunks) tmem_issue4(dt + (uint32_t)(f0 + kTcKC), dr_n);
 #pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            const int f = f0 + q;
+          for (int q = 0; q < 4; ++q) zo[q] = zo_n[q];
+          if (cc + 1 < kTcChunks) {            // the next chunk's cached fields, one chunk ahead
+#pragma unroll
+            for (int q = 0; q < 4; ++q) zo_n[q] = Zm[(size_t)(f0 + kTcKC + q) * Np + n];
+          } else if (!last) {                  // the next layer's first chunk
+#pragma unroll
+            for (int q = 0; q < 4; ++q) zo_n[q] = a.Z[m + 1][(size_t)(fp * 4 + q) * Np + n];
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
             const float zn = zo[q] + dv[q];
             const bool ch = live && zn != zo[q];
             const float an = act<ACTH>(zn, a.g[m], a.act[m]);
             const float ao = act<ACTH>(zo[q], a.g[m], a.act[m]);
-            const float d = ch ? an - ao : 0.0f;
-            if (COMMIT && ch) Zm[(size_t)f * Np + n] = zn;
-            if (!last) {
-              hi[q] = tf32_rna(d);
-              lo[q] = tf32_rna(d - hi[q]);
-            } else {
+            d[q] = ch ? an - ao : 0.0f;
+            if (COMMIT && ch) Zm[(size_t)(f0 + q) * Np + n] = zn;
+            if (sk) sk[m][(size_t)(f0 + q) * Np + n] = ch ? zn : zo[q];
+          }
+          bool okc = true;
+          if (!last) {
+            okc = produce_chunk(aring, s_afull, s_aempty, ga, fp, s, d);
+            ++ga;
+          } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
 #pragma unroll
               for (int o = 0; o < kMaxC; ++o)
-                if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f], d, outp[o]);
-            }
+                if (o < a.C) outp[o] = fmaf(Wout[(size_t)o * Kout + f0 + q], d[q], outp[o]);
           }
-          if (!last) {
-            tmem_st16(tmem + lane_base + 256u + (uint32_t)f0, hi);
-            store_alo16(alo, s, f0, lo);
+          tmem_wait4(dr_n);                    // chunk cc + 1's columns (none in flight at the end)
+          if (!okc) {
+            ok = false;
+            break;
           }
         }
       }
+      if (!ok) s_fail = 1;
     }
 
     // ---- output layer: the feature parts of each sample, in a fixed order
+    tc_fence_before();
+    __syncthreads();                                  // the control thread has drained
     float* xo = reinterpret_cast<float*>(wst);        // W stages are free now
-    __syncthreads();
-    if (hf >= 1) {
+    if (worker && fp >= 1) {
 #pragma unroll
-      for (int o = 0; o < kMaxC; ++o) xo[((hf - 1) * kMaxC + o) * kTcTS + s] = outp[o];
+      for (int o = 0; o < kMaxC; ++o) xo[((fp - 1) * kMaxC + o) * kTcTS + s] = outp[o];
     }
     __syncthreads();
-    if (hf == 0) {
+    if (worker && fp == 0) {
 #pragma unroll
       for (int p = 1; p < kParts; ++p)
 #pragma unroll
         for (int o = 0; o < kMaxC; ++o) outp[o] += xo[((p - 1) * kMaxC + o) * kTcTS + s];
     }
-    if (hf == 0 && live) {
+    const bool failed = s_fail != 0;                  // the same value in every thread here
+    if (worker && fp == 0 && live && !failed) {
       float zz[kMaxC];
       bool changed = false;
 #pragma unroll
@@ -382,12 +496,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) deep_chain_tc_kernel(DeepArgs a
         }
       }
       dl = out_delta<COMMIT>(a, n, zz, changed);
+      if (sk) {                                       // the same output fields and loss as a commit
+#pragma unroll
+        for (int o = 0; o < kMaxC; ++o)
+          if (o < a.C) sk[L - 1][(size_t)o * Np + n] = zz[o];
+        const int Lo = L - 1;
+        sk[L][n] = changed ? sample_loss<-1, -1, kMaxC>(zz, a.C, a.y[n], a.g[Lo], a.act[Lo], a.loss)
+                           : a.ell[n];
+      }
+    } else if (sk && worker && fp == 0 && !failed) {  // padding samples keep their values
+#pragma unroll
+      for (int o = 0; o < kMaxC; ++o)
+        if (o < a.C) sk[L - 1][(size_t)o * Np + n] = a.Z[L - 1][(size_t)o * Np + n];
+      sk[L][n] = a.ell[n];
     }
     if (dense) {
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      __syncthreads();
+      tc_fence_after();
       if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
-      if (tid == 0 && s_fail) atomicCAS(&a.st->err, 0, (int)MCA_ERR_TIMEOUT);
+      if (tid == 0 && failed) atomicCAS(&a.st->err, 0, (int)MCA_ERR_TIMEOUT);
     }
   }
   if (!COMMIT) {

@@ -115,6 +115,7 @@ constexpr int kTcTS = 128;         // samples per tile of the tensor-core chain 
 constexpr int kDeepThreads = 256;
 constexpr int kDeepMaxWidth = 256; // widths of the layers inside the dense chain
 constexpr int kDeepKC = 16;        // weight-tile depth of the chain GEMM
+constexpr int kDeepScrSlots = 16;  // candidates whose fields the tensor-core evaluation keeps
 
 struct DeepCand {
   unsigned int idx;
@@ -166,6 +167,12 @@ struct DeepArgs {
   const unsigned int* ex_idx;
   const float* ex_new;
   double* ex_out;
+  // tensor-core evaluation of candidate k < nscr with a dense chain (layer <= L-3): every field it
+  // computes goes to scr[k * (L + 1) + m] (layer m: row j of the mutated layer, the full layers
+  // after it; m = L: the per-sample losses), so that an accepted candidate's fields are adopted
+  // by swapping pointers instead of recomputing them
+  float* const* scr;
+  int nscr;
 };
 
 cudaError_t launch_deep_eval(const DeepArgs& a, cudaStream_t s);    // grid (Kb, ntiles)
@@ -359,6 +366,11 @@ struct mca_handle {
   double* ex_out = nullptr;
   mca_trace_rec* prop = nullptr;         // [kKmax] proposals of mca_eval_trials
   float* gimg = nullptr;                 // operand images of the tensor-core forward pass
+  int nscr = 0;                          // deep tensor-core path: candidate scratch slots
+  std::vector<float*> scr;               // [nscr x (L + 1)] layer m of slot k (m = L: losses)
+  float** scr_dev = nullptr;             // the same table in device memory
+  cudaEvent_t ev_c[2] = {nullptr, nullptr};   // around the adoption / commit after a decision
+  bool ev_c_pending = false;
   // test hook
   unsigned long long* ftau = nullptr;
   unsigned char* facc = nullptr;

@@ -20,46 +20,67 @@ sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
 from test_multirank_cpu import _run  # noqa: E402
 
 
-def _workload():
+def _workload(kind):
     from paper_2607_08406_gb300 import workloads as W
-    return W.make("mlp_wide", N=4000, H=96)
+    if kind == "wide":
+        return W.make("mlp_wide", N=4000, H=96)
+    if kind == "deep":
+        return W.make("mlp_deep", N=1200, width=40, depth=3)
+    spec = W.TfmSpec(vocab=17, ctx=8, d_model=16, n_layer=2, n_head=2, d_ff=32)
+    return W.char_transformer(batch=8, text_len=20000, spec=spec, n_trials=300, K=8)
 
 
-def _rank(rank, world, n, K, seed, forced):
+def _rank(rank, world, kind, n, K, seed, forced):
     import torch
     from paper_2607_08406_gb300 import mca
     from paper_2607_08406_gb300 import workloads as W
     from paper_2607_08406_gb300.sharded import LibraryShard, ShardedChain
     torch.cuda.set_device(0)
-    wl = _workload()
-    rows = np.array_split(np.arange(wl.N), world)[rank]
-    sub = W.MLPWorkload(wl.name, wl.layers, wl.loss, np.ascontiguousarray(wl.X[rows]),
-                        np.ascontiguousarray(wl.y[rows]), wl.init, n, K, seed, wl.domain)
-    h = mca.create_from_workload(sub, K=K, trace_cap=n)
-    chain = ShardedChain(LibraryShard(h), n_samples=wl.N, K=K)
+    wl = _workload(kind)
+    if kind == "tfm":                        # the loss is a sum over sequences: shard those
+        rows = np.array_split(np.arange(wl.tokens.shape[0]), world)[rank]
+        sub = W.TfmWorkload(wl.name, wl.spec, np.ascontiguousarray(wl.tokens[rows]), wl.init, n,
+                            K, seed, wl.domain)
+        h = mca.create_from_tfm_workload(sub, K=K, trace_cap=n)
+        n_total, n_mine = wl.tokens.shape[0] * wl.spec.ctx, len(rows) * wl.spec.ctx
+    else:
+        rows = np.array_split(np.arange(wl.N), world)[rank]
+        sub = W.MLPWorkload(wl.name, wl.layers, wl.loss, np.ascontiguousarray(wl.X[rows]),
+                            np.ascontiguousarray(wl.y[rows]), wl.init, n, K, seed, wl.domain)
+        h = mca.create_from_workload(sub, K=K, trace_cap=n)
+        n_total, n_mine = wl.N, len(rows)
+    chain = ShardedChain(LibraryShard(h), n_samples=n_total, K=K)
     st = chain.run(n, seed, forced=forced)
     tr = mca.mca_get_trace(h, n)
     out = (st, mca.mca_get_params(h, wl.n_params), tr["idx"].astype(np.int64),
-           tr["accept"].astype(bool), mca.mca_loss(h) * len(rows))
+           tr["accept"].astype(bool), mca.mca_loss(h) * n_mine)
     h.close()
     return out
 
 
-def test_two_rank_sharded_chain_follows_the_single_process_trajectory(gpu_lib):
+@pytest.mark.parametrize("kind,n,K", [("wide", 400, 16), ("deep", 300, 8), ("tfm", 200, 8)])
+def test_two_rank_sharded_chain_follows_the_single_process_trajectory(gpu_lib, kind, n, K):
+    """Single hidden layer, a deep net (samples split) and a Transformer (sequences split)."""
     from oracle import mca_oracle as O
+    from oracle import mca_tfm as T
     from parity import TIE_REL, tie_band
-    wl = _workload()
-    n, K, seed = 400, 16, 6
-    tr, params, S = O.run_incremental(wl.layers, wl.loss, wl.X, wl.y, wl.init, n, seed, wl.domain)
+    wl = _workload(kind)
+    seed = 6
+    if kind == "tfm":
+        tr, flat, S = T.run_full_tfm(wl.spec, wl.tokens, wl.init, n, seed, wl.domain)
+    else:
+        tr, params, S = O.run_incremental(wl.layers, wl.loss, wl.X, wl.y, wl.init, n, seed,
+                                          wl.domain)
+        flat = params.flat_eff32()
     band = tie_band(tr)
     forced = {int(t): bool(a) for t, a in zip(tr["tau"][band], tr["accept"][band])}
-    out = _run(_rank, 2, n, K, seed, forced)
+    out = _run(_rank, 2, kind, n, K, seed, forced)
     (st0, p0, idx0, acc0, S0), (st1, p1, idx1, acc1, S1) = out[0], out[1]
     assert st0 == st1 and st0["trials"] == n
     assert st0["exchanges"] == st0["batches"] < n           # batches consumed several trials
     assert np.array_equal(idx0, tr["idx"]) and np.array_equal(idx1, tr["idx"])
     assert np.array_equal(acc0, tr["accept"]) and np.array_equal(acc1, tr["accept"])
-    assert np.array_equal(p0, p1) and np.array_equal(p0, params.flat_eff32())
+    assert np.array_equal(p0, p1) and np.array_equal(p0, flat)
     assert S0 + S1 == pytest.approx(S, rel=TIE_REL)
 
 
