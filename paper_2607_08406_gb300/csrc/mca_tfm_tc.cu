@@ -14,13 +14,15 @@
 //   A Wv^T (tensor-memory columns 0, 128, 256; A at 384) -> K and V to shared memory -> causal
 //   attention of (row, head g) on the CUDA cores with a running softmax -> its output as the next
 //   A -> A Wo^T -> X += . + bo -> LN2 -> A -> per 64-wide hidden chunk c: U = A W1_c^T,
-//   act(U + b1) as A2 (hi in tensor memory, lo in shared memory), F += A2 W2_c^T -> X += F + b2.
+//   act(U + b1) as A2 (hi and lo parts both in tensor memory), F += A2 W2_c^T -> X += F + b2.
 // After the last block: LNf -> A -> logits = A Whead^T (vocabulary padded to 128) -> next-token
 // cross-entropy per row -> each sequence's loss summed over its rows in a fixed order.
 //
 // The weights come from split images (mca_tc_layout.h), 16 columns per chunk and one bulk copy per
-// chunk, through three shared-memory stages run by one thread with full / empty mbarriers; loads
-// run ahead of the MMAs except across an attention step, whose K and V reuse the stage memory. The
+// chunk, through five shared-memory stages run by one thread with full / empty mbarriers (a stage
+// is refilled once the MMAs of its chunk completed, so the ring's depth sets how much of the
+// copies' latency the MMAs hide); loads run ahead of the MMAs except across an attention step,
+// whose K and V reuse the lo part of A and the first four stages. The
 // images hold the current parameters: a candidate's changed weight W[i][j] enters as the rank-1 term
 // delta * A[:, j] on output column i in that projection's epilogue, and a changed bias, LN or
 // embedding parameter through a patched read. The commit kernel computes exactly what the
@@ -43,25 +45,25 @@ constexpr int kD = kTcTfmD;
 constexpr int kT = kTcTfmT;
 constexpr int kHc = kTcTfmHc;
 constexpr int kXLd = kD + 4;                     // residual row stride: conflict-free row access
-constexpr int kStages = 3;
+constexpr int kStages = 5;
 constexpr int kStageBytes = 16384;               // one chunk of 128 rows (64-row chunks use half)
 constexpr int kXsBytes = kRows * kXLd * 4;       // 67,584
 constexpr int kAloBytes = kRows * kD * 4;        // 65,536: lo part of A (K = 128)
-constexpr int kA2Bytes = kRows * kHc * 4;        // 32,768: lo part of A2 (K = 64)
-constexpr int kSmem = kXsBytes + kAloBytes + kA2Bytes + kStages * kStageBytes;
+constexpr int kSmem = kXsBytes + kAloBytes + kStages * kStageBytes;
 constexpr uint32_t kALBO = (kRows / 8) * 128;    // A operands: K groups 2 KB apart, rows 16 B
 constexpr uint32_t kIdN128 = tc_idesc_tf32(kRows, 128);
 constexpr uint32_t kIdN64 = tc_idesc_tf32(kRows, 64);
 // tensor-memory columns
 constexpr uint32_t kColQ = 0, kColK = 128, kColV = 256, kColA = 384;
 constexpr uint32_t kColU = 0, kColF = 128, kColA2 = 256;   // Wo and the head also use kColU
+constexpr uint32_t kColA2lo = 320;                         // lo part of A2 (K = 64)
 // weight chunks of one block: Wq Wk Wv (24), Wo (8), then per hidden chunk W1_c (8) and W2_c (4)
 constexpr int kQkvChunks = 24, kWoChunk0 = 24, kFfnChunk0 = 32, kFfnPerChunk = 12;
 constexpr int kHeadChunks = 8;
 
 static_assert(kSmem + 8 * 1024 <= 227 * 1024, "shared memory of the Transformer tensor-core kernel");
-// K and V (2 x 64 KB) overlay the lo parts of A and A2 and the first two stages
-static_assert(2 * kRows * kD * 4 <= kAloBytes + kA2Bytes + 2 * kStageBytes, "K and V overlay");
+// K and V (2 x 64 KB) overlay the lo part of A and the first four stages
+static_assert(2 * kRows * kD * 4 <= kAloBytes + 4 * kStageBytes, "K and V overlay");
 
 __device__ __forceinline__ float prm(const TfmArgs& a, unsigned long long i,
                                      unsigned long long midx, float mval) {
@@ -122,7 +124,6 @@ __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
 struct Ctx {
   float* xs;                 // residual stream [128][kXLd]
   unsigned char* alo;        // lo part of A, core-matrix order (element (r, k) at (k/4) kALBO + 16 r)
-  unsigned char* a2lo;       // lo part of A2, same order
   unsigned char* wst;        // weight stages
   float* ks;                 // K [128][128], 16-byte slots of a row swizzled by (row mod 8)
   float* vs;                 // V, same
@@ -136,7 +137,8 @@ struct Ctx {
   Target tg;
 };
 
-// Loads of the weight ring, run by one thread.
+// State of the weight ring, in shared memory: nload belongs to the loading thread, nwait and
+// ncommit to the MMA thread, limit is set before the CTA barrier that starts an MMA phase.
 struct Issuer {
   int nload;                 // next chunk to load
   int limit;                 // chunks at or past this one may not be loaded yet
@@ -186,16 +188,18 @@ __device__ bool topup(const TfmArgs& a, const Ctx& c, Issuer& is, int upto, uint
   return true;
 }
 
-// One thread: the MMAs of chunks x0 .. x0 + n - 1, each released to its stage's empty barrier.
+// One thread: the MMAs of chunks x0 .. x0 + n - 1, each released to its stage's empty barrier. It
+// waits only for each chunk's data; the stages are refilled by another thread (produce).
 __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n, uint64_t* full,
                       uint64_t* empty) {
   tc_fence_after();
-  const uint32_t salo = smem_u32(c.alo), sa2 = smem_u32(c.a2lo), sw = smem_u32(c.wst);
+  const uint32_t salo = smem_u32(c.alo), sw = smem_u32(c.wst);
   for (int x = x0; x < x0 + n; ++x) {
     const int st = x % kStages;
     if (!mbar_wait(&full[st], (uint32_t)(x / kStages) & 1u)) return false;
     is.nwait = x + 1;
     uint32_t dcol = kColU, idesc = kIdN128, alo = salo, acol = kColA, R = 128;
+    bool lo_tm = false;                          // A's lo part in tensor memory (A2)
     int kc;
     bool first;
     if (x < c.nb * c.cpb) {
@@ -216,7 +220,7 @@ __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
           first = kc == 0;
         } else {                                 // W2 of hidden chunk h, accumulated over h
           dcol = kColF;
-          alo = sa2;
+          lo_tm = true;
           acol = kColA2;
           kc = u - 8;
           first = h == 0 && kc == 0;
@@ -235,15 +239,30 @@ __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
       const uint64_t dwhi = umma_desc(wb, lbo, 128u);
       const uint64_t dwlo = umma_desc(wb + 4u * lbo, lbo, 128u);
       const uint32_t d = c.tmem + dcol, ta = c.tmem + acol + (uint32_t)gk * 8u;
-      mma_ss(d, da, dwhi, idesc, (first && ks == 0) ? 0u : 1u);
+      if (lo_tm)
+        mma_ts(d, c.tmem + kColA2lo + (uint32_t)gk * 8u, dwhi, idesc, (first && ks == 0) ? 0u : 1u);
+      else
+        mma_ss(d, da, dwhi, idesc, (first && ks == 0) ? 0u : 1u);
       mma_ts(d, ta, dwlo, idesc, 1u);
       mma_ts(d, ta, dwhi, idesc, 1u);
     }
     umma_commit(&empty[st]);
     is.ncommit = x + 1;
-    if (!topup(a, c, is, x + kStages, full, empty)) return false;
   }
   return true;
+}
+
+// An MMA phase of chunks x0 .. x0 + n - 1: thread 0 issues the MMAs while thread 32 refills each
+// stage as soon as the MMAs of its previous chunk complete, up to kStages - 1 chunks past the
+// phase (within the limit), so that the MMA thread never waits for a refill. Both waits end by
+// the time the phase's MMAs complete.
+__device__ __forceinline__ void mma_phase(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
+                                          uint64_t* full, uint64_t* empty, volatile int* fail) {
+  if (threadIdx.x == 0) {
+    if (!issue(a, c, is, x0, n, full, empty)) *fail = 1;
+  } else if (threadIdx.x == 32) {
+    if (!topup(a, c, is, x0 + n - 1 + kStages, full, empty)) *fail = 1;
+  }
 }
 
 // Every thread: wait for the MMAs of chunk `last` (and so of every earlier chunk); false, the same
@@ -295,6 +314,20 @@ __device__ __forceinline__ void store_a(const Ctx& c, const float (&v)[N], uint3
           make_float4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
     }
   }
+}
+
+// The A2 operand of row r, columns k0 .. k0 + 15: tf32 hi and lo parts into tensor-memory columns
+// col .. and lo_col .. .
+__device__ __forceinline__ void store_a2(const Ctx& c, const float (&v)[16], uint32_t col,
+                                         uint32_t lo_col) {
+  float hi[16], lo[16];
+#pragma unroll
+  for (int q = 0; q < 16; ++q) {
+    hi[q] = tf32_rna(v[q]);
+    lo[q] = tf32_rna(v[q] - hi[q]);
+  }
+  tmem_st16(c.tmem + c.trow + col, hi);
+  tmem_st16(c.tmem + c.trow + lo_col, lo);
 }
 
 // Layer norm of row r (its 32 columns here, statistics over all four parts) written as the A
@@ -418,8 +451,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   c.trow = (uint32_t)((warp & 3) * 32) << 16;
   c.xs = reinterpret_cast<float*>(tsm);
   c.alo = tsm + kXsBytes;
-  c.a2lo = c.alo + kAloBytes;
-  c.wst = c.a2lo + kA2Bytes;
+  c.wst = c.alo + kAloBytes;
   c.ks = reinterpret_cast<float*>(c.alo);
   c.vs = c.ks + kRows * kD;
   if (MODE == kTfmCommit && a.ctl->kstar < 0) return;
@@ -508,9 +540,12 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
                  ::"r"(smem_u32(&s_tmem)));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
-  Issuer is;
-  is.nload = is.nwait = is.ncommit = 0;
-  is.limit = c.nb > 0 ? kWoChunk0 : kHeadChunks;
+  __shared__ Issuer s_is;
+  Issuer& is = s_is;
+  if (tid == 0) {
+    is.nload = is.nwait = is.ncommit = 0;
+    is.limit = c.nb > 0 ? kWoChunk0 : kHeadChunks;
+  }
   if (tid == 0) {
     for (int q = 0; q < kStages; ++q) {
       mbar_init(&s_full[q], 1);
@@ -560,7 +595,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
             (here && c.tg.mat >= kTcQ && c.tg.mat <= kTcV) ? c.tg.col : -1, s_part, s_acol);
     tc_publish_operands();
     __syncthreads();
-    if (tid == 0 && !issue(a, c, is, gc, kQkvChunks, s_full, s_empty)) *fail = 1;
+    mma_phase(a, c, is, gc, kQkvChunks, s_full, s_empty, fail);
     gc += kQkvChunks;
     if (!(ok = group_done(s_empty, gc - 1, fail))) break;
     float q[32];
@@ -597,15 +632,13 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
       }
       store_a<32>(c, o, kColA + 32u * (uint32_t)c.g, c.alo, 32 * c.g);
     }
-    tc_publish_operands();
-    __syncthreads();
-    if (tid == 0) {
+    if (tid == 0) {              // loads may now run into the next block's Q, K, V chunks
       const int jb = b - c.b0s;
       is.limit = jb + 1 < c.nb ? (jb + 1) * c.cpb + kWoChunk0 : c.total;
-      if (!topup(a, c, is, gc + kStages, s_full, s_empty) ||
-          !issue(a, c, is, gc, kFfnChunk0 - kWoChunk0, s_full, s_empty))
-        *fail = 1;
     }
+    tc_publish_operands();
+    __syncthreads();
+    mma_phase(a, c, is, gc, kFfnChunk0 - kWoChunk0, s_full, s_empty, fail);
     gc += kFfnChunk0 - kWoChunk0;
     if (!(ok = group_done(s_empty, gc - 1, fail))) break;
     {
@@ -621,7 +654,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
             s_part, s_acol);
     tc_publish_operands();
     __syncthreads();
-    if (tid == 0 && !issue(a, c, is, gc, 8, s_full, s_empty)) *fail = 1;
+    mma_phase(a, c, is, gc, 8, s_full, s_empty, fail);
     gc += 8;
     for (int h = 0; h < nH; ++h) {
       if (!(ok = group_done(s_empty, gc - 1, fail))) break;
@@ -637,11 +670,11 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
         for (int i = 0; i < 16; ++i)
           if (f0 + i == c.tg.col) s_acol[c.r] = u[i];
       }
-      store_a<16>(c, u, kColA2 + 16u * (uint32_t)c.g, c.a2lo, 16 * c.g);
+      store_a2(c, u, kColA2 + 16u * (uint32_t)c.g, kColA2lo + 16u * (uint32_t)c.g);
       tc_publish_operands();
       __syncthreads();
       const int n = h + 1 < nH ? kFfnPerChunk : 4;   // W2 of chunk h, then W1 of chunk h + 1
-      if (tid == 0 && !issue(a, c, is, gc, n, s_full, s_empty)) *fail = 1;
+      mma_phase(a, c, is, gc, n, s_full, s_empty, fail);
       gc += n;
     }
     if (!ok || !(ok = group_done(s_empty, gc - 1, fail))) break;
@@ -668,7 +701,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
             s_acol);
     tc_publish_operands();
     __syncthreads();
-    if (tid == 0 && !issue(a, c, is, gc, kHeadChunks, s_full, s_empty)) *fail = 1;
+    mma_phase(a, c, is, gc, kHeadChunks, s_full, s_empty, fail);
     gc += kHeadChunks;
     ok = group_done(s_empty, gc - 1, fail);
   }

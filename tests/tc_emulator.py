@@ -17,14 +17,13 @@ from oracle.mca_oracle import act_fn
 
 f32 = np.float32
 kThreads, kRows, kD, kT, kHc, kXLd = 512, 128, 128, 64, 64, 132
-kStages, kStageBytes = 3, 16384
+kStages, kStageBytes = 5, 16384
 kXsBytes = kRows * kXLd * 4
 kAloBytes = kRows * kD * 4
-kA2Bytes = kRows * kHc * 4
-kSmem = kXsBytes + kAloBytes + kA2Bytes + kStages * kStageBytes
+kSmem = kXsBytes + kAloBytes + kStages * kStageBytes
 kALBO = (kRows // 8) * 128
 kColQ, kColK, kColV, kColA = 0, 128, 256, 384
-kColU, kColF, kColA2 = 0, 128, 256
+kColU, kColF, kColA2, kColA2lo = 0, 128, 256, 320
 kQkvChunks, kWoChunk0, kFfnChunk0, kFfnPerChunk, kHeadChunks = 24, 24, 32, 12, 8
 kTcQ, kTcK, kTcV, kTcO, kTcW1, kTcW2, kTcHead, kNone = 0, 1, 2, 3, 4, 5, 6, -1
 EVAL, COMMIT, FORWARD = 0, 1, 2
@@ -211,7 +210,7 @@ class CTA:
             if x >= kStages:
                 self.wait(self.empty[st], x - kStages)
             src, nbytes = self.chunk_src(x)
-            dst = (kXsBytes + kAloBytes + kA2Bytes + st * kStageBytes) // 4
+            dst = (kXsBytes + kAloBytes + st * kStageBytes) // 4
             # overwrite hazard: record which bytes a load covers at issue time
             self.sm[dst:dst + nbytes // 4] = self.a.wimg[src:src + nbytes // 4]
             self.loaded_regions.append((x, dst * 4, nbytes))
@@ -246,12 +245,13 @@ class CTA:
             self.tm[:M, dcol:dcol + N] = D
 
     def issue(self, x0, n):
-        salo, sa2, sw = kXsBytes, kXsBytes + kAloBytes, kXsBytes + kAloBytes + kA2Bytes
+        salo, sw = kXsBytes, kXsBytes + kAloBytes
         for x in range(x0, x0 + n):
             st = x % kStages
             self.wait(self.full[st], x)
             self.nwait = x + 1
             dcol, idsc, alo, acol, R = kColU, kIdN128, salo, kColA, 128
+            lo_tm = False                       # A's lo part in tensor memory (A2)
             if x < self.nb * self.cpb:
                 q = x % self.cpb
                 if q < kWoChunk0:
@@ -268,7 +268,7 @@ class CTA:
                         idsc, R, kc = kIdN64, 64, u
                         first = kc == 0
                     else:
-                        dcol, alo, acol, kc = kColF, sa2, kColA2, u - 8
+                        dcol, lo_tm, acol, kc = kColF, True, kColA2, u - 8
                         first = h == 0 and kc == 0
             else:
                 kc = x - self.nb * self.cpb
@@ -281,7 +281,10 @@ class CTA:
                 dwhi = umma_desc(wb, lbo, 128)
                 dwlo = umma_desc(wb + 4 * lbo, lbo, 128)
                 ta = acol + gk * 8
-                self.mma(dcol, da, dwhi, idsc, 0 if (first and ks == 0) else 1, False)
+                if lo_tm:
+                    self.mma(dcol, kColA2lo + gk * 8, dwhi, idsc, 0 if (first and ks == 0) else 1, True)
+                else:
+                    self.mma(dcol, da, dwhi, idsc, 0 if (first and ks == 0) else 1, False)
                 self.mma(dcol, ta, dwlo, idsc, 1, True)
                 self.mma(dcol, ta, dwhi, idsc, 1, True)
             self.empty[st].k += 1
@@ -315,6 +318,13 @@ class CTA:
                 fi = self.smf(addr)
                 for e in range(4):
                     self.sm[fi + e] = lo[:, 4 * q + e]
+
+    def store_a2(self, v, col, lo_col):
+        # v: [128 rows, 16]: hi and lo tf32 parts into tensor-memory columns col.. and lo_col..
+        seg = v.astype(np.float32)
+        hi = tf32_rna(seg)
+        self.tm[:, col:col + 16] = hi
+        self.tm[:, lo_col:lo_col + 16] = tf32_rna(seg - hi)
 
     def ln_to_a(self, og, ob, stash):
         x = np.stack([self.sm[self.xr_addr(g)[:, None] + np.arange(32)[None, :]] for g in range(4)])  # [4,128,32]
@@ -506,7 +516,7 @@ class CTA:
                         u[:, i] = act_fn(a.act, (u[:, i] + self.prm(base + a.r_b1 + f0 + i)).astype(np.float64), a.g).astype(np.float32)
                     if here and tg[0] == kTcW2 and f0 <= tg[2] < f0 + 16:
                         self.s_acol_w2 = u[:, tg[2] - f0].copy()
-                    self.store_a(u, kColA2 + 16 * g, kXsBytes + kAloBytes, 16 * g, g, 16)
+                    self.store_a2(u, kColA2 + 16 * g, kColA2lo + 16 * g)
                 if here and tg[0] == kTcW2 and h * kHc <= tg[2] < h * kHc + kHc:
                     self.s_acol = self.s_acol_w2
                 n = kFfnPerChunk if h + 1 < nH else 4
