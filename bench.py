@@ -33,9 +33,9 @@ METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roo
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of the trial-loop kernel per trial,
 # from one ncu capture (one pass, one launch: the first timed step, trials 200k..240k) of
 # `python bench.py --steps 20 --warmup 5 --no-e2e --no-cpu`, summarised in profiles/. It is only
-# valid for the kernel source it was measured on; any other source hash reports null.
+# valid for the kernel source and the workload it was measured on; anything else reports null.
 LOOP_TRAFFIC = {"source_sha1": "d226e40a5b6369a5b1cfa03226a2bb7319f8dc8f",
-                "bytes_per_trial": 374000.0}
+                "workload": "mlp784-16384-10_ce_n60000", "bytes_per_trial": 374000.0}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
 
@@ -381,7 +381,8 @@ def run_ours(args):
     else:
         bytes_timed = st1["alg_bytes"] - st0["alg_bytes"]
         achieved = bytes_timed / K / (total_ms / K / 1e3) / 1e9
-        if LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and LOOP_TRAFFIC["bytes_per_trial"]:
+        if (LOOP_TRAFFIC["source_sha1"] == loop_source_sha1() and
+                LOOP_TRAFFIC["workload"] == wl.name and LOOP_TRAFFIC["bytes_per_trial"]):
             traffic = LOOP_TRAFFIC["bytes_per_trial"] * (st1["trials"] - st0["trials"]) / K
         roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                     "frac": achieved / peak, "traffic": traffic, "kernel": "mlp2_window_loop",
