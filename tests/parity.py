@@ -15,10 +15,15 @@ def oracle_trace(wl, n_trials, seed=0, mode="incremental", domain=None):
 
 def tie_band(tr, theta=0.0):
     """Trials where the oracle's dS lies within TIE_REL * S of the acceptance threshold theta (0 for
-    the greedy rule, Eq. 6; per trial for the Metropolis rule, Eq. 7) and dS != 0 (exact zeros,
-    the no-op proposals, must match)."""
+    the greedy rule, Eq. 6; per trial for the Metropolis rule, Eq. 7), except exact zeros of
+    proposals that leave the parameter unchanged (new == old): those are no-ops and must match.
+    An exact zero of a changed parameter is a tie like any other: it comes from an invariance of
+    the network (a key bias adds the same q . b_k to every score of an attention row, which the
+    softmax removes), which the fp64 oracle resolves to 0 and an fp32 evaluation to a
+    rounding-size value of either sign."""
     d = np.abs(tr["dS"] - theta)
-    return tr["valid"] & (d < TIE_REL * np.abs(tr["S"])) & (tr["dS"] != 0.0)
+    noop = (tr["dS"] == 0.0) & (tr["new"] == tr["old"])
+    return tr["valid"] & (d < TIE_REL * np.abs(tr["S"])) & ~noop
 
 
 def forced_from_oracle(tr, theta=0.0):
