@@ -173,7 +173,7 @@ typedef struct {
   uint32_t tensor_cores;   /* 1: this handle's dense recomputation runs on the tcgen05 tensor-core
                               kernels (3xTF32): a deep net whose hidden layers are all 256 x 256,
                               or a Transformer with ctx 64, d_model 128, 4 heads, d_ff a multiple
-                              of 64 up to 1024, vocab <= 128 and an even number of sequences
+                              of 128 up to 1024, vocab <= 128 and an even number of sequences
                               (unless the process sets MCA_TFM_TENSOR_CORES=0 before creating
                               the handle); 0: the SIMT fp32 kernels */
   uint32_t reserved;       /* 0 */
@@ -232,7 +232,7 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
  * int32, host or device (inputs tokens[:, :ctx], targets tokens[:, 1:]); init_params: [P] fp32,
  * host or device, in the flat order above. Every parameter is an fp32 weight (Eq. 1 replacement or
  * perturbation). mca_loss reports S / (n_seq * ctx). Errors as for mca_create.
- * Kernels: with ctx 64, d_model 128, 4 heads, d_ff a multiple of 64 up to 1024, vocab <= 128 and an
+ * Kernels: with ctx 64, d_model 128, 4 heads, d_ff a multiple of 128 up to 1024, vocab <= 128 and an
  * even n_seq the sequences run on the tensor-core kernels (3xTF32 tcgen05, two sequences per CTA);
  * for other shapes, or when the process environment has MCA_TFM_TENSOR_CORES=0, on the SIMT fp32
  * kernels. The variable is read by this call and by mca_tfm_workspace_size (the tensor-core kernels'

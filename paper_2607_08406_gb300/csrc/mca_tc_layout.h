@@ -30,22 +30,24 @@ MCA_HD size_t tc_image_index(int r, int k, int R, int cols) {
 // Distance in floats from a high part to its low part.
 MCA_HD size_t tc_image_lo(int R) { return (size_t)R * 16; }
 
-// Transformer (d_model 128, d_ff = F a multiple of 64): per block Wq, Wk, Wv, Wo (128 x 128,
-// R = 128), W1 (F x 128, R = 64), W2 (128 x F, R = 128); after the last block the head (vocab rows,
-// padded with zero rows to 128, R = 128).
+// Transformer (d_model 128, d_ff = F a multiple of 128): per block Wq, Wk, Wv, Wo (128 x 128,
+// R = 128), W1 (F x 128, R = 128: the hidden units of two 64-wide FFN chunks per row block), W2
+// (128 x F, R = 128); after the last block the head (vocab rows, padded with zero rows to 128,
+// R = 128).
 enum TfmTcMat { kTcMatNone = -1, kTcQ = 0, kTcK = 1, kTcV = 2, kTcO = 3, kTcW1 = 4, kTcW2 = 5,
                 kTcHead = 6 };
 
 constexpr int kTcTfmD = 128;        // model width of the tensor-core Transformer kernels
 constexpr int kTcTfmT = 64;         // tokens per sequence
 constexpr int kTcTfmHeads = 4;
-constexpr int kTcTfmHc = 64;        // feed-forward hidden columns per chunk
+constexpr int kTcTfmHc = 64;        // feed-forward hidden columns per chunk (activation, W2)
+constexpr int kTcTfmHp = 128;       // feed-forward hidden columns per W1 product (two chunks)
 
 MCA_HD size_t tfm_tc_block_floats(int F) { return (size_t)4 * 32768 + (size_t)512 * F; }
 MCA_HD size_t tfm_tc_image_floats(int F, int nL) {
   return (size_t)nL * tfm_tc_block_floats(F) + 32768;
 }
-MCA_HD int tfm_tc_rows(int mat) { return mat == kTcW1 ? 64 : 128; }
+MCA_HD int tfm_tc_rows(int) { return 128; }
 
 // Float offset of the high part of element (r, k) of matrix `mat` of block b.
 MCA_HD size_t tfm_tc_image_offset(int mat, int b, int r, int k, int F, int nL) {
@@ -53,14 +55,14 @@ MCA_HD size_t tfm_tc_image_offset(int mat, int b, int r, int k, int F, int nL) {
   if (mat == kTcHead) return (size_t)nL * blk + tc_image_index(r, k, 128, kTcTfmD);
   const size_t base = (size_t)b * blk;
   if (mat <= kTcO) return base + (size_t)mat * 32768 + tc_image_index(r, k, 128, kTcTfmD);
-  if (mat == kTcW1) return base + 131072 + tc_image_index(r, k, 64, kTcTfmD);
+  if (mat == kTcW1) return base + 131072 + tc_image_index(r, k, kTcTfmHp, kTcTfmD);
   return base + 131072 + (size_t)256 * F + tc_image_index(r, k, 128, F);
 }
 
 // Shapes the tensor-core Transformer kernels handle: T = 64, d = 128, 4 heads of 32, d_ff a
-// multiple of 64 up to 1024, vocab <= 128, an even number of sequences (two per CTA).
+// multiple of 128 up to 1024, vocab <= 128, an even number of sequences (two per CTA).
 MCA_HD bool tfm_tc_shape_ok(int T, int d, int H, int F, int V, long long B) {
-  return T == kTcTfmT && d == kTcTfmD && H == kTcTfmHeads && F % kTcTfmHc == 0 && F >= 64 &&
+  return T == kTcTfmT && d == kTcTfmD && H == kTcTfmHeads && F % kTcTfmHp == 0 && F >= kTcTfmHp &&
          F <= 1024 && V >= 2 && V <= 128 && B % 2 == 0;
 }
 

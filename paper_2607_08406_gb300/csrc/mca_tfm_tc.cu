@@ -13,8 +13,10 @@
 //   LN1 -> A (tf32 hi part in tensor memory, lo part in shared memory) -> Q, K, V = A Wq^T, A Wk^T,
 //   A Wv^T (tensor-memory columns 0, 128, 256; A at 384) -> K and V to shared memory -> causal
 //   attention of (row, head g) on the CUDA cores with a running softmax -> its output as the next
-//   A -> A Wo^T -> X += . + bo -> LN2 -> A -> per 64-wide hidden chunk c: U = A W1_c^T,
-//   act(U + b1) as A2 (hi and lo parts both in tensor memory), F += A2 W2_c^T -> X += F + b2.
+//   A -> A Wo^T -> X += . + bo -> LN2 -> A -> per pair of 64-wide hidden chunks: U = A W1_pair^T
+//   (N = 128: a tcgen05 MMA takes about as long at N = 64 as at N = 128, so pairing halves W1's
+//   MMAs), then per chunk c of the pair act(U_c + b1) as A2 (hi and lo parts both in tensor
+//   memory), F += A2 W2_c^T -> X += F + b2.
 // After the last block: LNf -> A -> logits = A Whead^T (vocabulary padded to 128) -> next-token
 // cross-entropy per row -> each sequence's loss summed over its rows in a fixed order.
 //
@@ -52,13 +54,14 @@ constexpr int kAloBytes = kRows * kD * 4;        // 65,536: lo part of A (K = 12
 constexpr int kSmem = kXsBytes + kAloBytes + kStages * kStageBytes;
 constexpr uint32_t kALBO = (kRows / 8) * 128;    // A operands: K groups 2 KB apart, rows 16 B
 constexpr uint32_t kIdN128 = tc_idesc_tf32(kRows, 128);
-constexpr uint32_t kIdN64 = tc_idesc_tf32(kRows, 64);
 // tensor-memory columns
 constexpr uint32_t kColQ = 0, kColK = 128, kColV = 256, kColA = 384;
 constexpr uint32_t kColU = 0, kColF = 128, kColA2 = 256;   // Wo and the head also use kColU
 constexpr uint32_t kColA2lo = 320;                         // lo part of A2 (K = 64)
-// weight chunks of one block: Wq Wk Wv (24), Wo (8), then per hidden chunk W1_c (8) and W2_c (4)
-constexpr int kQkvChunks = 24, kWoChunk0 = 24, kFfnChunk0 = 32, kFfnPerChunk = 12;
+// weight chunks of one block: Wq Wk Wv (24), Wo (8), then per pair p of hidden chunks W1 of the pair
+// (8, N = 128) and W2 of its two chunks (4 + 4)
+constexpr int kQkvChunks = 24, kWoChunk0 = 24, kFfnChunk0 = 32, kFfnPerPair = 16;
+constexpr int kHp = kTcTfmHp;                    // hidden columns per W1 product
 constexpr int kHeadChunks = 8;
 
 static_assert(kSmem + 8 * 1024 <= 227 * 1024, "shared memory of the Transformer tensor-core kernel");
@@ -156,14 +159,13 @@ __device__ __forceinline__ void chunk_src(const TfmArgs& a, const Ctx& c, int x,
       bytes = 16384;
       return;
     }
-    const int f = q - kFfnChunk0, h = f / kFfnPerChunk, u = f - h * kFfnPerChunk;
-    if (u < 8) {
-      src = base + 131072 + (size_t)(h * 8 + u) * 2048;
-      bytes = 8192;
-    } else {
-      src = base + 131072 + (size_t)256 * a.F + (size_t)(h * 4 + u - 8) * 4096;
-      bytes = 16384;
+    const int f = q - kFfnChunk0, p = f / kFfnPerPair, u = f - p * kFfnPerPair;
+    if (u < 8) {                                 // W1 of pair p
+      src = base + 131072 + (size_t)(p * 8 + u) * 4096;
+    } else {                                     // W2 of hidden chunk 2p + (u - 8) / 4
+      src = base + 131072 + (size_t)256 * a.F + (size_t)(p * 8 + u - 8) * 4096;
     }
+    bytes = 16384;
   } else {
     src = a.wimg + (size_t)a.nL * tfm_tc_block_floats(a.F) + (size_t)(x - c.nb * c.cpb) * 4096;
     bytes = 16384;
@@ -212,18 +214,16 @@ __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
         kc = q - kWoChunk0;
         first = kc == 0;
       } else {
-        const int f = q - kFfnChunk0, h = f / kFfnPerChunk, u = f - h * kFfnPerChunk;
-        if (u < 8) {                             // W1 of hidden chunk h
-          idesc = kIdN64;
-          R = 64;
+        const int f = q - kFfnChunk0, p = f / kFfnPerPair, u = f - p * kFfnPerPair;
+        if (u < 8) {                             // W1 of hidden pair p (N = 128)
           kc = u;
           first = kc == 0;
-        } else {                                 // W2 of hidden chunk h, accumulated over h
+        } else {                                 // W2 of hidden chunk 2p + (u-8)/4, accumulated
           dcol = kColF;
           lo_tm = true;
           acol = kColA2;
-          kc = u - 8;
-          first = h == 0 && kc == 0;
+          kc = (u - 8) & 3;
+          first = p == 0 && u == 8;
         }
       }
     } else {                                     // head
@@ -531,7 +531,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   const int b0 = (fwd || cd.layer < 0) ? -1 : cd.layer;
   c.b0s = b0 < 0 ? 0 : b0;
   c.nb = a.nL - c.b0s;
-  c.cpb = kFfnChunk0 + kFfnPerChunk * (a.F / kHc);
+  c.cpb = kFfnChunk0 + kFfnPerPair * (a.F / kHp);
   c.total = c.nb * c.cpb + kHeadChunks;
 
   // tensor memory, the stage ring, the first chunks
@@ -586,7 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   volatile int* fail = &s_fail;
   int gc = 0;                    // next chunk whose MMAs are issued (the same in every thread)
   bool ok = true;
-  const int nH = a.F / kHc;
+  const int nP = a.F / kHp;
   for (int b = c.b0s; ok && b < a.nL; ++b) {
     const bool here = b == c.cstage;
     const unsigned long long base = a.o_blk0 + (unsigned long long)b * a.blk_size;
@@ -649,17 +649,19 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) xr[i] += v[i] + prm(a, bo + i, c.midx, c.mval);
     }
-    // ---- feed-forward network in hidden chunks of 64
+    // ---- feed-forward network: W1 for two 64-wide hidden chunks at a time (N = 128), then per
+    // chunk the activation as A2 and its W2 product
     ln_to_a(a, c, base + a.r_ln2g, base + a.r_ln2b, (here && c.tg.mat == kTcW1) ? c.tg.col : -1,
             s_part, s_acol);
     tc_publish_operands();
     __syncthreads();
     mma_phase(a, c, is, gc, 8, s_full, s_empty, fail);
     gc += 8;
-    for (int h = 0; h < nH; ++h) {
+    for (int h = 0; h < 2 * nP; ++h) {
       if (!(ok = group_done(s_empty, gc - 1, fail))) break;
+      // this thread's 16 hidden units of chunk h, from the pair's U (columns 0-63 or 64-127)
       float u[16];
-      tmem_ld16(c.tmem + c.trow + kColU + 16u * (uint32_t)c.g, u);
+      tmem_ld16(c.tmem + c.trow + kColU + (uint32_t)((h & 1) * kHc) + 16u * (uint32_t)c.g, u);
       const int f0 = h * kHc + 16 * c.g;
       if (here && c.tg.mat == kTcW1) add_at(u, c.tg.row - f0, c.dlt * s_acol[c.r]);
 #pragma unroll
@@ -673,7 +675,8 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
       store_a2(c, u, kColA2 + 16u * (uint32_t)c.g, kColA2lo + 16u * (uint32_t)c.g);
       tc_publish_operands();
       __syncthreads();
-      const int n = h + 1 < nH ? kFfnPerChunk : 4;   // W2 of chunk h, then W1 of chunk h + 1
+      // W2 of chunk h; after a pair's second chunk (its U fully read) also W1 of the next pair
+      const int n = (h & 1) && h + 1 < 2 * nP ? 12 : 4;
       mma_phase(a, c, is, gc, n, s_full, s_empty, fail);
       gc += n;
     }

@@ -24,7 +24,8 @@ kSmem = kXsBytes + kAloBytes + kStages * kStageBytes
 kALBO = (kRows // 8) * 128
 kColQ, kColK, kColV, kColA = 0, 128, 256, 384
 kColU, kColF, kColA2, kColA2lo = 0, 128, 256, 320
-kQkvChunks, kWoChunk0, kFfnChunk0, kFfnPerChunk, kHeadChunks = 24, 24, 32, 12, 8
+kQkvChunks, kWoChunk0, kFfnChunk0, kFfnPerPair, kHeadChunks = 24, 24, 32, 16, 8
+kHp = 128           # hidden columns per W1 product (two 64-wide chunks)
 kTcQ, kTcK, kTcV, kTcO, kTcW1, kTcW2, kTcHead, kNone = 0, 1, 2, 3, 4, 5, 6, -1
 EVAL, COMMIT, FORWARD = 0, 1, 2
 
@@ -33,7 +34,7 @@ def idesc(M, N):
     return (1 << 4) | (2 << 7) | (2 << 10) | ((N >> 3) << 17) | ((M >> 4) << 24)
 
 
-kIdN128, kIdN64 = idesc(128, 128), idesc(128, 64)
+kIdN128 = idesc(128, 128)
 
 
 def tf32_rna(x):
@@ -70,12 +71,12 @@ def image_offset(mat, b, r, k, F, nL):
     if mat <= kTcO:
         return base + mat * 32768 + tc_image_index(r, k, 128, kD)
     if mat == kTcW1:
-        return base + 131072 + tc_image_index(r, k, 64, kD)
+        return base + 131072 + tc_image_index(r, k, 128, kD)
     return base + 131072 + 256 * F + tc_image_index(r, k, 128, F)
 
 
 def lo_off(mat):
-    return (64 if mat == kTcW1 else 128) * 16
+    return 128 * 16
 
 
 class Args:
@@ -196,10 +197,10 @@ class CTA:
             if q < kFfnChunk0:
                 return base + q * 4096, 16384
             f = q - kFfnChunk0
-            h, u = divmod(f, kFfnPerChunk)
+            p, u = divmod(f, kFfnPerPair)
             if u < 8:
-                return base + 131072 + (h * 8 + u) * 2048, 8192
-            return base + 131072 + 256 * A.F + (h * 4 + u - 8) * 4096, 16384
+                return base + 131072 + (p * 8 + u) * 4096, 16384
+            return base + 131072 + 256 * A.F + (p * 8 + u - 8) * 4096, 16384
         return A.nL * blk_floats(A.F) + (x - self.nb * self.cpb) * 4096, 16384
 
     def topup(self, upto):
@@ -263,13 +264,13 @@ class CTA:
                     first = kc == 0
                 else:
                     f = q - kFfnChunk0
-                    h, u = divmod(f, kFfnPerChunk)
+                    p, u = divmod(f, kFfnPerPair)
                     if u < 8:
-                        idsc, R, kc = kIdN64, 64, u
+                        kc = u
                         first = kc == 0
                     else:
-                        dcol, lo_tm, acol, kc = kColF, True, kColA2, u - 8
-                        first = h == 0 and kc == 0
+                        dcol, lo_tm, acol, kc = kColF, True, kColA2, (u - 8) & 3
+                        first = p == 0 and u == 8
             else:
                 kc = x - self.nb * self.cpb
                 first = kc == 0
@@ -419,7 +420,7 @@ class CTA:
         b0 = -1 if (mode == FORWARD or layer < 0) else layer
         self.b0s = 0 if b0 < 0 else b0
         self.nb = a.nL - self.b0s
-        self.cpb = kFfnChunk0 + kFfnPerChunk * (a.F // kHc)
+        self.cpb = kFfnChunk0 + kFfnPerPair * (a.F // kHp)
         self.total = self.nb * self.cpb + kHeadChunks
         self.nload = self.nwait = self.ncommit = 0
         self.limit = kWoChunk0 if self.nb > 0 else kHeadChunks
@@ -441,7 +442,7 @@ class CTA:
         for g in range(4):
             self.sm[self.xr_addr(g)[:, None] + np.arange(32)[None, :]] = xs[:, 32 * g:32 * g + 32]
         gc = 0
-        nH = a.F // kHc
+        nP = a.F // kHp
         for b in range(self.b0s, a.nL):
             here = b == cstage
             base = a.o_blk0 + b * a.blk_size
@@ -503,10 +504,11 @@ class CTA:
             self.ln_to_a(base + a.r_ln2g, base + a.r_ln2b, tg[2] if (here and tg[0] == kTcW1) else -1)
             self.issue(gc, 8)
             gc += 8
-            for h in range(nH):
+            for h in range(2 * nP):
                 self.group_done(gc - 1)
                 for g in range(4):
-                    u = self.tm[:, kColU + 16 * g:kColU + 16 * g + 16].copy()
+                    c0 = kColU + (h & 1) * kHc + 16 * g       # the pair's U, chunk h's columns
+                    u = self.tm[:, c0:c0 + 16].copy()
                     f0 = h * kHc + 16 * g
                     if here and tg[0] == kTcW1:
                         at = tg[1] - f0
@@ -519,7 +521,7 @@ class CTA:
                     self.store_a2(u, kColA2 + 16 * g, kColA2lo + 16 * g)
                 if here and tg[0] == kTcW2 and h * kHc <= tg[2] < h * kHc + kHc:
                     self.s_acol = self.s_acol_w2
-                n = kFfnPerChunk if h + 1 < nH else 4
+                n = 12 if (h & 1) and h + 1 < 2 * nP else 4
                 self.issue(gc, n)
                 gc += n
             self.group_done(gc - 1)

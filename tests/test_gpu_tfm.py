@@ -2,7 +2,7 @@
 
 Small specs check trajectories (proposals bit for bit, decisions with the tie band replayed, final
 parameters) on the SIMT kernels; specs of the tensor-core kernels' shape (context 64, d_model 128,
-4 heads, d_ff a multiple of 64, an even number of sequences) with few sequences and narrow FFNs
+4 heads, d_ff a multiple of 128, an even number of sequences) with few sequences and narrow FFNs
 check trajectories and candidates of every parameter tensor on the tensor-core kernels. The
 config-sized spec is in test_gpu_config_size.py.
 """
@@ -19,7 +19,7 @@ pytestmark = pytest.mark.gpu
 SMALL = W.TfmSpec(vocab=17, ctx=8, d_model=16, n_layer=2, n_head=2, d_ff=32)
 MID = W.TfmSpec(vocab=23, ctx=20, d_model=40, n_layer=1, n_head=4, d_ff=200, act="gaussian")
 # the tensor-core kernels' shape with one or two blocks, narrow FFNs and few sequences
-TC_ONE = W.TfmSpec(vocab=65, ctx=64, d_model=128, n_layer=1, n_head=4, d_ff=64)
+TC_ONE = W.TfmSpec(vocab=65, ctx=64, d_model=128, n_layer=1, n_head=4, d_ff=128)
 TC_TWO = W.TfmSpec(vocab=65, ctx=64, d_model=128, n_layer=2, n_head=4, d_ff=128, act="gaussian",
                    act_param=0.4)
 

@@ -99,8 +99,8 @@ def test_image_matches_descriptor_layout(probe, R, rows, cols):
 
 
 def test_transformer_images_tile_and_follow_the_chunk_order(probe):
-    """Per block: Wq Wk Wv Wo as 8 chunks of 4096 floats each (32 in a row), W1 as (hidden chunk h,
-    K chunk u) 2048-float chunks from 131072, W2 as 4096-float chunks from 131072 + 256 F; the head
+    """Per block: Wq Wk Wv Wo as 8 chunks of 4096 floats each (32 in a row), W1 as (hidden pair p,
+    K chunk u) 4096-float chunks from 131072, W2 as 4096-float chunks from 131072 + 256 F; the head
     after the last block. Hi and lo offsets of all entries tile the image exactly once."""
     F, nL = 128, 2
     lines = probe("tfm", F, nL)
@@ -117,8 +117,8 @@ def test_transformer_images_tile_and_follow_the_chunk_order(probe):
     start[qkvo] = base[qkvo] + (m[qkvo] * 8 + k[qkvo] // 16) * 4096
     size[qkvo] = 4096
     w1 = m == 4
-    start[w1] = base[w1] + 131072 + ((r[w1] // 64) * 8 + k[w1] // 16) * 2048
-    size[w1] = 2048
+    start[w1] = base[w1] + 131072 + ((r[w1] // 128) * 8 + k[w1] // 16) * 4096
+    size[w1] = 4096
     w2 = m == 5
     start[w2] = base[w2] + 131072 + 256 * F + (k[w2] // 16) * 4096
     size[w2] = 4096
@@ -131,8 +131,11 @@ def test_transformer_images_tile_and_follow_the_chunk_order(probe):
 
 def test_shape_gate(probe):
     """The character-level workload (T 64, d 128, 4 heads, FFN 512, vocabulary 65, 256 sequences)
-    qualifies; other widths, odd sequence counts, or a vocabulary above 128 do not."""
+    qualifies; other widths, an FFN that is not a multiple of 128 (W1 is issued 128 hidden units at
+    a time), odd sequence counts, or a vocabulary above 128 do not."""
     assert probe("ok", 64, 128, 4, 512, 65, 256) == ["1"]
+    assert probe("ok", 64, 128, 4, 128, 65, 2) == ["1"]
     for args in [(32, 128, 4, 512, 65, 256), (64, 96, 4, 512, 65, 256), (64, 128, 2, 512, 65, 256),
-                 (64, 128, 4, 500, 65, 256), (64, 128, 4, 512, 200, 256), (64, 128, 4, 512, 65, 255)]:
+                 (64, 128, 4, 500, 65, 256), (64, 128, 4, 192, 65, 256), (64, 128, 4, 64, 65, 256),
+                 (64, 128, 4, 512, 200, 256), (64, 128, 4, 512, 65, 255)]:
         assert probe("ok", *args) == ["0"], args
