@@ -9,6 +9,7 @@
 #include <cstring>
 #include <new>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include <nvtx3/nvToolsExt.h>
@@ -248,9 +249,25 @@ mca_domain default_domain() {
   return d;
 }
 
+// Non-zeros of a host array, counted by up to 16 threads (the counts add up in any order).
 long long host_nnz(const float* x, size_t n) {
+  auto count = [x](size_t b, size_t e) {
+    long long c = 0;
+    for (size_t i = b; i < e; ++i) c += x[i] != 0.0f;
+    return c;
+  };
+  const unsigned hw = std::thread::hardware_concurrency();
+  const unsigned nt = n < (size_t)(1u << 22) ? 1u : std::max(1u, std::min(16u, hw));
+  if (nt == 1) return count(0, n);
+  const size_t per = (n + nt - 1) / nt;
+  std::vector<long long> part(nt, 0);
+  std::vector<std::thread> th;
+  th.reserve(nt);
+  for (unsigned t = 0; t < nt; ++t)
+    th.emplace_back([&, t] { part[t] = count(std::min(n, t * per), std::min(n, (t + 1) * per)); });
+  for (auto& q : th) q.join();
   long long c = 0;
-  for (size_t i = 0; i < n; ++i) c += x[i] != 0.0f;
+  for (long long v : part) c += v;
   return c;
 }
 
