@@ -131,9 +131,12 @@ typedef struct {
                               caller-owned device buffer of >= mca_workspace_size() bytes,
                               256-byte aligned, that must outlive the handle */
   size_t workspace_bytes;
-  int32_t fixed_K;         /* 0: each batch evaluates ceil(c / p) candidates, at most K, where p is
-                              the recently observed acceptance rate per trial (fewer discarded
-                              candidates while many are accepted; the trajectory is the same);
+  int32_t fixed_K;         /* 0: the batch width follows p, the recently observed acceptance rate
+                              per trial, at most K (fewer discarded candidates while many are
+                              accepted; the trajectory is the same): ceil(2 / p) candidates for
+                              single-hidden-layer networks; for deep nets and Transformers the K
+                              that maximises the expected trials consumed, (1 - (1-p)^K) / p, per
+                              batch cost r + K (r about 2 candidate evaluations);
                               1: every batch evaluates K candidates */
 } mca_options;
 

@@ -1005,8 +1005,10 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     while (remaining > 0) {
       NvtxRange nv_batch(h->tfm ? "mca batch (transformer)" : "mca batch (deep)");
       const int Kw = h->opt.fixed_K ? h->opt.K
-                                    : mca::batch_width(h->rate_acc, h->rate_trials,
-                                                       mca::kWidthDeep, h->opt.K);
+                                    : mca::batch_width_cost(h->rate_acc, h->rate_trials,
+                                                            h->tfm ? mca::kBatchCostTfm
+                                                                   : mca::kBatchCostDeep,
+                                                            h->opt.K);
       uint64_t kb = std::min<uint64_t>(remaining, (uint64_t)Kw);
       if (R > 0) kb = std::min<uint64_t>(kb, R - h->tau % R);
       if (!h->ev[0]) {

@@ -21,10 +21,33 @@ constexpr int kLoopThreads = 512; // threads per CTA of the trial-loop kernel
 constexpr int kLoopWarps = kLoopThreads / 32;
 constexpr int kMaxSubs = 8;       // sub-chunks of one candidate inside one sample range
 constexpr int kRangeTarget = 64;
-// Batch width: ceil(c / p) candidates, p = (A + 0.5) / (T + 1) from counts decayed per batch.
+// Batch width of the single-hidden-layer loop: ceil(c / p) candidates, p = (A + 0.5) / (T + 1) from
+// counts decayed per batch.
 constexpr float kRateDecay = 0.95f;
 constexpr float kWidthMlp2 = 2.0f;
-constexpr float kWidthDeep = 1.0f;   // deep nets and the Transformer (host-driven batches)
+// Host-driven batches (deep nets, the Transformer): a batch of K candidates consumes
+// (1 - (1 - p)^K) / p trials on average and costs about r + K candidate evaluations, r being its
+// fixed part (decision, commit, launch gaps, the last partial wave of CTAs). The width maximises
+// trials per cost. r was fitted to fixed-width runs on GB300 (batch time against K): about 1.9
+// candidate-times for the 24 x 256 chain at N = 10000, 1.4 for the d_model 128 Transformer on 256
+// sequences.
+constexpr float kBatchCostDeep = 1.9f;
+constexpr float kBatchCostTfm = 1.4f;
+
+inline int batch_width_cost(float acc, float trials, float r, int K) {
+  const double p = ((double)acc + 0.5) / ((double)trials + 1.0);
+  double qk = 1.0, best = -1.0;
+  int kb = 1;
+  for (int k = 1; k <= K; ++k) {
+    qk *= 1.0 - p;
+    const double v = (1.0 - qk) / ((double)r + (double)k);
+    if (v > best) {
+      best = v;
+      kb = k;
+    }
+  }
+  return kb;
+}
 constexpr int kSmemRecordBytes = 160 * 1024;  // larger ranges keep their records in global memory
 // Window of the trial loop: kWS candidate slots per CTA, each caching up to kCap entries of the
 // candidate's segment (range-local sample, activation change, new hidden field), prepared ahead of

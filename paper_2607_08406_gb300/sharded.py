@@ -16,9 +16,8 @@ trials every rank
      them: the shard's kernels re-evaluate those candidates and take the given decisions).
 
 No device work waits for another rank; the exchange is the only collective. The batch width
-follows the observed acceptance rate as in the library's host-driven paths (ceil(c / p) trials,
-p = (A + 1/2) / (T + 1) from counts decayed by 0.95 per batch, at most K); every rank computes it
-from the same decisions.
+follows the observed acceptance rate (ceil(c / p) trials, p = (A + 1/2) / (T + 1) from counts
+decayed by 0.95 per batch, at most K); every rank computes it from the same decisions.
 
 A shard is any object with eval_trials / decide / commit (LibraryShard wraps a handle), so the
 same chain runs over other evaluators, e.g. in CPU tests.
