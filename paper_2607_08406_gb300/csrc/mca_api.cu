@@ -94,9 +94,17 @@ bool deep_tc_ok(const std::vector<mca_layer>& layers) {
 }
 int deep_tc_tiles(long long N) { return (int)((N + mca::kTcTS - 1) / mca::kTcTS); }
 
+// Accepted candidates are adopted from scratch slots written by their evaluation (deep and
+// Transformer tensor-core paths) unless the process sets MCA_ADOPT=0: then the commit kernels
+// recompute them. Read by the workspace-size calls and creation, so it must not change between them.
+bool adopt_enabled() {
+  const char* e = std::getenv("MCA_ADOPT");
+  return !(e && std::strcmp(e, "0") == 0);
+}
+
 // Candidate scratch slots of the deep tensor-core path (min(K, kDeepScrSlots)); none elsewhere.
 int deep_scratch_slots(const std::vector<mca_layer>& layers, int K) {
-  return deep_tc_ok(layers) ? std::min(K, mca::kDeepScrSlots) : 0;
+  return deep_tc_ok(layers) && adopt_enabled() ? std::min(K, mca::kDeepScrSlots) : 0;
 }
 
 int pad_n(long long N) { return (int)((N + 127) / 128 * 128); }
@@ -646,7 +654,8 @@ mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
 
 struct TfmMem {
   size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, prop, scratch,
-      wimg, total;
+      wimg, scrX, scr_ell, total;
+  int nscr;
 };
 
 // The tensor-core Transformer kernels (mca_tfm_tc.cu) run a handle's sequences when the shape is
@@ -658,7 +667,16 @@ bool tfm_use_tc(const mca_tfm_spec& t, long long B) {
   return mca::tfm_tc_shape_ok(t.ctx, t.d_model, t.n_head, t.d_ff, t.vocab, B);
 }
 
-TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc) {
+// Scratch slots of the tensor-core Transformer kernels: candidate k < nscr of a batch writes its
+// residual streams and sequence losses to slot k, min(K, kTfmScrSlots) slots within 8 GiB.
+int tfm_scratch_slots(const mca_tfm_spec& t, long long B, int K, bool tc) {
+  if (!tc || !adopt_enabled()) return 0;
+  const size_t slot = sizeof(float) * ((size_t)(t.n_layer + 1) * B * t.ctx * t.d_model + B);
+  const size_t cap = (size_t)8 << 30;
+  return (int)std::min<size_t>((size_t)std::min(K, mca::kTfmScrSlots), cap / slot);
+}
+
+TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc, int K) {
   TfmMem M;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -681,6 +699,9 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc) {
   M.prop = take(sizeof(mca_trace_rec) * mca::kKmax);
   M.scratch = take(sizeof(int) * 8);
   M.wimg = tc ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
+  M.nscr = tfm_scratch_slots(t, B, K, tc);
+  M.scrX = take(sizeof(float) * (size_t)M.nscr * (t.n_layer + 1) * B * t.ctx * t.d_model);
+  M.scr_ell = take(sizeof(float) * (size_t)M.nscr * B);
   M.total = o;
   return M;
 }
@@ -1018,9 +1039,18 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
       if (h->tfm) {
         ta.tau = h->tau;
         ta.Kb = (int)kb;
+        ta.nscr = h->nscr;
+        ta.scrX = h->tfm_scrX;
+        ta.scr_ell = h->tfm_scr_ell;
         CUDA_TRY(h, mca::launch_tfm_eval(ta, h->stream));
         CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
+        // an accepted candidate with a scratch slot is adopted from it (the commit kernel then
+        // returns at once); one beyond the slots is recomputed by the commit kernel
+        if (ta.nscr > 0) {
+          CUDA_TRY(h, mca::launch_tfm_tc_adopt(ta, h->stream));
+          h->launches += 1;
+        }
         CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
         if (ta.tc) {
           CUDA_TRY(h, mca::launch_tfm_tc_image_update(ta, h->stream));
@@ -1402,7 +1432,7 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
   if (rc != MCA_OK) return rc;
   if (!bytes) return fail(nullptr, MCA_ERR_INVALID, "bytes is NULL");
   const mca_options o = opt ? *opt : default_options();
-  *bytes = tfm_plan(*spec, n_seq, o.trace_cap, tfm_use_tc(*spec, n_seq)).total;
+  *bytes = tfm_plan(*spec, n_seq, o.trace_cap, tfm_use_tc(*spec, n_seq), o.K).total;
   return MCA_OK;
 }
 
@@ -1459,7 +1489,7 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
     e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
   if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));
   h->tc = tfm_use_tc(*spec, n_seq);
-  const TfmMem M = tfm_plan(*spec, n_seq, o.trace_cap, h->tc);
+  const TfmMem M = tfm_plan(*spec, n_seq, o.trace_cap, h->tc, o.K);
   if (o.workspace) {
     if (o.workspace_bytes < M.total)
       return bail(fail(h, MCA_ERR_OOM, "workspace of %zu bytes < %zu needed", o.workspace_bytes,
@@ -1491,6 +1521,9 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
   h->prop = reinterpret_cast<mca_trace_rec*>(base + M.prop);
   h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
+  h->nscr = M.nscr;
+  h->tfm_scrX = reinterpret_cast<float*>(base + M.scrX);
+  h->tfm_scr_ell = reinterpret_cast<float*>(base + M.scr_ell);
   e = cudaMemsetAsync(h->st, 0, sizeof(DevState), h->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ctl, 0, sizeof(mca::DeepCtl), h->stream);
   if (e != cudaSuccess) return bail(fail(h, MCA_ERR_CUDA, "%s", cudaGetErrorString(e)));

@@ -139,6 +139,7 @@ constexpr int kDeepThreads = 256;
 constexpr int kDeepMaxWidth = 256; // widths of the layers inside the dense chain
 constexpr int kDeepKC = 16;        // weight-tile depth of the chain GEMM
 constexpr int kDeepScrSlots = 16;  // candidates whose fields the tensor-core evaluation keeps
+constexpr int kTfmScrSlots = 16;   // candidates whose residual streams the evaluation keeps
 
 struct DeepCand {
   unsigned int idx;
@@ -261,6 +262,12 @@ struct TfmArgs {
   double* ex_out;
   int tc;                    // 1: the tensor-core kernels (mca_tfm_tc.cu) run the sequences
   float* wimg;               // their split-weight images (mca_tc_layout.h), tc = 1 only
+  // scratch slots (tc = 1, trial loop only): candidate k < nscr of a batch writes the residual
+  // streams it recomputes to slot k of scrX ([nscr][(nL + 1) x B x T x d]) and its sequence losses
+  // to scr_ell ([nscr][B]); an accepted candidate with a slot is adopted from it
+  float* scrX;
+  float* scr_ell;
+  int nscr;
 };
 
 size_t tfm_smem_bytes(int T, int d, int dh, int V);
@@ -275,6 +282,7 @@ cudaError_t launch_tfm_tc_eval(const TfmArgs& a, cudaStream_t s);      // grid (
 cudaError_t launch_tfm_tc_commit(const TfmArgs& a, cudaStream_t s);    // grid B / 2
 cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s);   // grid B / 2
 cudaError_t launch_tfm_tc_image_update(const TfmArgs& a, cudaStream_t s);
+cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s);     // grid (B, nL + 1)
 
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
 cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
@@ -389,7 +397,7 @@ struct mca_handle {
   double* ex_out = nullptr;
   mca_trace_rec* prop = nullptr;         // [kKmax] proposals of mca_eval_trials
   float* gimg = nullptr;                 // operand images of the tensor-core forward pass
-  int nscr = 0;                          // deep tensor-core path: candidate scratch slots
+  int nscr = 0;                          // tensor-core paths: candidate scratch slots
   std::vector<float*> scr;               // [nscr x (L + 1)] layer m of slot k (m = L: losses)
   float** scr_dev = nullptr;             // the same table in device memory
   cudaEvent_t ev_c[2] = {nullptr, nullptr};   // around the adoption / commit after a decision
@@ -411,5 +419,7 @@ struct mca_handle {
   float* params = nullptr;               // [P] flat parameters
   int* tokens = nullptr;                 // [B x (ctx + 1)]
   float* X = nullptr;                    // cached residual stream at every stage
-  float* tfm_img = nullptr;              // split-weight images of the tensor-core kernels (tc)
+  float* tfm_img = nullptr;
+  float* tfm_scrX = nullptr;             // Transformer tensor-core path: candidate scratch slots
+  float* tfm_scr_ell = nullptr;          // (h->nscr of them)              // split-weight images of the tensor-core kernels (tc)
 };

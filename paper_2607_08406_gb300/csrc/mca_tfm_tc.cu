@@ -29,7 +29,9 @@
 // delta * A[:, j] on output column i in that projection's epilogue, and a changed bias, LN or
 // embedding parameter through a patched read. The commit kernel computes exactly what the
 // evaluation computed (same images, same terms) and writes the cached residual streams and
-// sequence losses; the image entry of the accepted weight is refreshed after it.
+// sequence losses; the image entry of the accepted weight is refreshed after it. In the trial loop
+// the evaluation of candidate k < nscr also writes what the commit would write into scratch slot
+// k, and an accepted candidate with a slot is adopted by copying it (the commit kernel returns).
 #include <cstdio>
 
 #include "mca_device.cuh"
@@ -454,7 +456,9 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   c.wst = c.alo + kAloBytes;
   c.ks = reinterpret_cast<float*>(c.alo);
   c.vs = c.ks + kRows * kD;
-  if (MODE == kTfmCommit && a.ctl->kstar < 0) return;
+  // the commit recomputes an accepted candidate that has no scratch slot (kstar >= nscr); one with
+  // a slot is adopted from it by tfm_tc_adopt_kernel
+  if (MODE == kTfmCommit && a.ctl->kstar < a.nscr) return;
   int k = 0, pair = blockIdx.x;
   if (MODE == kTfmEval) {
     // Longest recomputations first: CTAs start in linear block order, so the linear index is
@@ -500,6 +504,14 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   __syncthreads();
   const DeepCand cd = s_c;
   float* part = a.partial + (size_t)k * a.B + s0;
+  // where the recomputed residual streams and sequence losses go: the handle's (commit, forward)
+  // or, in an evaluation, the candidate's scratch slot when it has one
+  const size_t seq_floats = (size_t)kT * kD;
+  const bool slot = MODE == kTfmEval && k < a.nscr;
+  float* const xout = MODE != kTfmEval ? a.X
+                      : slot ? a.scrX + (size_t)k * (size_t)(a.nL + 1) * a.B * seq_floats
+                             : nullptr;
+  float* const lout = MODE != kTfmEval ? a.ell : slot ? a.scr_ell + (size_t)k * a.B : nullptr;
   if (!cd.valid || cd.delta == 0.0f) {
     if (MODE == kTfmEval && tid < 2) part[tid] = 0.0f;
     return;
@@ -561,7 +573,6 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
 
   // residual stream entering the first stage run
   float* xr = c.xs + c.r * kXLd + 32 * c.g;
-  const size_t seq_floats = (size_t)kT * kD;
   if (b0 < 0) {
     const int tok = s_tok[c.sl][c.t];
 #pragma unroll
@@ -570,8 +581,8 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
       xr[i] = prm(a, a.o_tok + (unsigned long long)tok * kD + col, c.midx, c.mval) +
               prm(a, a.o_pos + (unsigned long long)c.t * kD + col, c.midx, c.mval);
     }
-    if (MODE != kTfmEval && !s_skip[c.sl]) {
-      float* dst = a.X + (size_t)(s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+    if (xout && !s_skip[c.sl]) {
+      float* dst = xout + (size_t)(s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
         reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
@@ -689,8 +700,8 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) xr[i] += v[i] + prm(a, b2 + i, c.midx, c.mval);
     }
-    if (MODE != kTfmEval && !s_skip[c.sl]) {
-      float* dst = a.X + ((size_t)(b + 1) * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+    if (xout && !s_skip[c.sl]) {
+      float* dst = xout + ((size_t)(b + 1) * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
         reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
@@ -742,10 +753,8 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
     if (tid < 2) {
       float l = 0.0f;
       for (int t = 0; t < kT; ++t) l += s_rowv[tid * kT + t];
-      if (MODE == kTfmEval)
-        part[tid] = s_skip[tid] ? 0.0f : l - a.ell[s0 + tid];
-      else if (!s_skip[tid])
-        a.ell[s0 + tid] = l;
+      if (MODE == kTfmEval) part[tid] = s_skip[tid] ? 0.0f : l - a.ell[s0 + tid];
+      if (lout && !s_skip[tid]) lout[s0 + tid] = l;
     }
   }
 
@@ -807,6 +816,37 @@ __global__ void tfm_tc_image_update_kernel(TfmArgs a) {
   a.wimg[o + tc_image_lo(tfm_tc_rows(tg.mat))] = tf32_rna(w - hi);
 }
 
+// After the decision: the accepted candidate's residual streams (the stages its evaluation
+// recomputed: X[0 ..] for an embedding, X[b + 1 ..] for block b, none for the final LN and head)
+// and sequence losses, copied from its scratch slot. CTA (s, x) copies sequence s of stream x;
+// sequences the evaluation skipped (a token embedding whose token they do not contain) keep theirs.
+__global__ void tfm_tc_adopt_kernel(TfmArgs a) {
+  const int ks = a.ctl->kstar;
+  if (ks < 0 || ks >= a.nscr) return;
+  const DeepCand cd = a.ctl->acc;
+  if (!cd.valid || cd.delta == 0.0f) return;
+  const int s = blockIdx.x, x = blockIdx.y;
+  __shared__ int s_skip;
+  if (threadIdx.x == 0) {
+    int skip = 0;
+    if (cd.row >= 0) {
+      skip = 1;
+      for (int t = 0; t < kT; ++t) skip &= a.tokens[(size_t)s * (kT + 1) + t] != cd.row;
+    }
+    s_skip = skip;
+  }
+  __syncthreads();
+  if (s_skip) return;
+  if (x == 0 && threadIdx.x == 0) a.ell[s] = a.scr_ell[(size_t)ks * a.B + s];
+  if (x < (cd.layer < 0 ? 0 : cd.layer + 1)) return;
+  const size_t seq_floats = (size_t)kT * kD;
+  const size_t at = ((size_t)x * a.B + s) * seq_floats;
+  const float4* src = reinterpret_cast<const float4*>(
+      a.scrX + (size_t)ks * (size_t)(a.nL + 1) * a.B * seq_floats + at);
+  float4* dst = reinterpret_cast<float4*>(a.X + at);
+  for (int q = threadIdx.x; q < (int)(seq_floats / 4); q += blockDim.x) dst[q] = src[q];
+}
+
 template <int MODE>
 cudaError_t launch_tc(const TfmArgs& a, dim3 grid, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute((const void*)tfm_tc_kernel<MODE>,
@@ -834,6 +874,11 @@ cudaError_t launch_tfm_tc_commit(const TfmArgs& a, cudaStream_t s) {
 
 cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s) {
   return launch_tc<kTfmForward>(a, dim3(a.B / 2), s);
+}
+
+cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s) {
+  tfm_tc_adopt_kernel<<<dim3(a.B, a.nL + 1), 256, 0, s>>>(a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_tfm_tc_image_update(const TfmArgs& a, cudaStream_t s) {

@@ -170,9 +170,33 @@ class Bar:
         self.k = 0          # completed phases
 
 
+class Slot:
+    """A candidate's scratch slot: the residual streams and sequence losses its evaluation writes."""
+    def __init__(self, a):
+        self.X = np.full_like(a.X, np.nan)
+        self.ell = np.full_like(a.ell, np.nan)
+
+
+def adopt(a, slot, cand):
+    """The adopt kernel: the accepted candidate's recomputed streams (X[0..] for an embedding,
+    X[b+1..] for block b, none for the head stage) and losses from its slot, sequences it skipped
+    (a token embedding whose token they lack) left as they are."""
+    idx, neww, delta, layer, row = cand
+    if delta == 0.0:
+        return
+    first = 0 if layer < 0 else layer + 1
+    for s in range(a.B):
+        if row >= 0 and np.all(a.tokens[s, :kT] != row):
+            continue
+        a.ell[s] = slot.ell[s]
+        for x in range(first, a.nL + 1):
+            a.X[x, s] = slot.X[x, s]
+
+
 class CTA:
-    def __init__(self, a, mode, cand, pair):
+    def __init__(self, a, mode, cand, pair, slot=None):
         self.a, self.mode, self.pair = a, mode, pair
+        self.slot = slot    # EVAL: the candidate's scratch slot, if it has one
         self.sm = np.zeros(kSmem // 4, np.float32)
         self.tm = np.zeros((128, 512), np.float32)
         self.full = [Bar() for _ in range(kStages)]
@@ -428,15 +452,17 @@ class CTA:
         self.topup(kStages)
         self.s_acol = np.zeros(128, np.float32)
         # residual
+        xout = a.X if mode != EVAL else (self.slot.X if self.slot is not None else None)
+        lout = a.ell if mode != EVAL else (self.slot.ell if self.slot is not None else None)
         xs = np.zeros((128, kD), np.float32)
         if b0 < 0:
             tok = toks[sl, t]
             for col in range(kD):
                 xs[:, col] = self.prm(a.o_tok + tok * kD + col) + self.prm(a.o_pos + t * kD + col)
-            if mode != EVAL:
+            if xout is not None:
                 for q in range(2):
                     if not skip[q]:
-                        a.X[0, s0 + q] = xs[q * kT:(q + 1) * kT]
+                        xout[0, s0 + q] = xs[q * kT:(q + 1) * kT]
         else:
             xs[:] = a.X[b0, s0 + sl, t]
         for g in range(4):
@@ -534,11 +560,11 @@ class CTA:
                 xa = self.xr_addr(g)
                 for i in range(32):
                     self.sm[xa + i] = self.sm[xa + i] + (v[:, i] + self.prm(base + a.r_b2 + 32 * g + i))
-            if mode != EVAL:
+            if xout is not None:
                 for q in range(2):
                     if not skip[q]:
                         for g in range(4):
-                            a.X[b + 1, s0 + q, :, 32 * g:32 * g + 32] = self.sm[self.xr_addr(g)[q * kT:(q + 1) * kT, None] + np.arange(32)[None, :]]
+                            xout[b + 1, s0 + q, :, 32 * g:32 * g + 32] = self.sm[self.xr_addr(g)[q * kT:(q + 1) * kT, None] + np.arange(32)[None, :]]
         # head
         here = cstage == a.nL
         self.ln_to_a(a.o_lnf_g, a.o_lnf_b, tg[2] if (here and tg[0] == kTcHead) else -1)
@@ -573,8 +599,8 @@ class CTA:
                 lsum = f32(lsum + rowv[q * kT + tt])
             if mode == EVAL:
                 out[q] = 0.0 if skip[q] else lsum - a.ell[s0 + q]
-            elif not skip[q]:
-                a.ell[s0 + q] = lsum
+            if lout is not None and not skip[q]:
+                lout[s0 + q] = lsum
         return out
 
 

@@ -6,6 +6,8 @@ biases, LN parameters and embeddings), and the commit writing exactly what the e
 This checks the kernel's offsets, descriptors, chunk schedule, swizzles and epilogue terms, not the
 hardware: the kernel itself is compared with the oracle by the GPU tests.
 """
+import copy
+
 import numpy as np
 import pytest
 
@@ -79,6 +81,35 @@ def test_emulated_commit_writes_what_evaluation_computed(setup):
         np.testing.assert_array_equal(refreshed, a.wimg)
         ell = OT.tfm_seq_losses(spec, a.params.astype(np.float64), a.tokens)
         assert np.all(np.abs(a.ell - ell) <= 2e-6 * ell), name
+
+
+def test_emulated_adoption_writes_what_the_commit_writes(setup):
+    """An evaluation with a scratch slot followed by the adopt kernel leaves the residual streams and
+    sequence losses exactly as the commit kernel would, for a candidate of every stage kind: token
+    embeddings (one whose token some sequences lack: they keep theirs), a position embedding, a
+    block-0 projection, the last block's FFN and the head."""
+    spec, a0 = setup
+    picks = _picks(a0)
+    # a token that some sequences contain and others do not
+    present = np.array([[np.any(a0.tokens[s, :E.kT] == v) for s in range(a0.B)]
+                        for v in range(a0.V)])
+    partial = np.nonzero(present.any(axis=1) & ~present.all(axis=1))[0]
+    assert len(partial) > 0
+    picks["tok_emb_partial"] = int(partial[0]) * a0.d + 11
+    for name in ("tok_emb", "tok_emb_partial", "pos_emb", "wq", "w2", "w_head"):
+        a = copy.deepcopy(a0)
+        c = _cand(a, picks[name], 0.37)
+        slot = E.Slot(a)
+        for p in range(a.B // 2):
+            E.CTA(a, E.EVAL, c, p, slot).run()
+        b = copy.deepcopy(a)
+        a.params[c[0]] = c[1]                       # the decide kernel's write
+        b.params[c[0]] = c[1]
+        for p in range(a.B // 2):
+            E.CTA(a, E.COMMIT, c, p).run()
+        E.adopt(b, slot, c)
+        np.testing.assert_array_equal(b.X, a.X, err_msg=name)
+        np.testing.assert_array_equal(b.ell, a.ell, err_msg=name)
 
 
 def test_emulated_kernel_at_the_largest_shape_it_takes():
