@@ -27,12 +27,12 @@ constexpr float kRateDecay = 0.95f;
 constexpr float kWidthMlp2 = 2.0f;
 // Host-driven batches (deep nets, the Transformer): a batch of K candidates consumes
 // (1 - (1 - p)^K) / p trials on average and costs about r + K candidate evaluations, r being its
-// fixed part (decision, commit, launch gaps, the last partial wave of CTAs). The width maximises
-// trials per cost. r was fitted to fixed-width runs on GB300 (batch time against K): about 1.9
-// candidate-times for the 24 x 256 chain at N = 10000, 1.4 for the d_model 128 Transformer on 256
-// sequences.
+// fixed part (decision, adoption or commit, launch gaps, the last partial wave of CTAs). The width
+// maximises trials per cost. r was fitted to fixed-width runs on GB300 (batch time against K):
+// about 1.9 candidate-times for the 24 x 256 chain at N = 10000, 0.5 for the d_model 128
+// Transformer on 256 sequences.
 constexpr float kBatchCostDeep = 1.9f;
-constexpr float kBatchCostTfm = 1.4f;
+constexpr float kBatchCostTfm = 0.5f;
 
 inline int batch_width_cost(float acc, float trials, float r, int K) {
   const double p = ((double)acc + 0.5) / ((double)trials + 1.0);
