@@ -1045,15 +1045,12 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
         CUDA_TRY(h, mca::launch_tfm_eval(ta, h->stream));
         CUDA_TRY(h, cudaEventRecord(h->ev[1], h->stream));
         CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
-        // an accepted candidate with a scratch slot is adopted from it (the commit kernel then
-        // returns at once); one beyond the slots is recomputed by the commit kernel
-        if (ta.nscr > 0) {
-          CUDA_TRY(h, mca::launch_tfm_tc_adopt(ta, h->stream));
-          h->launches += 1;
-        }
+        // the commit kernel recomputes an accepted candidate beyond the scratch slots (and
+        // returns at once otherwise); then the accepted weight's image entry and, for a
+        // candidate with a slot, its adoption
         CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
         if (ta.tc) {
-          CUDA_TRY(h, mca::launch_tfm_tc_image_update(ta, h->stream));
+          CUDA_TRY(h, mca::launch_tfm_tc_adopt(ta, h->stream));
           h->launches += 1;
         }
       } else {

@@ -244,10 +244,9 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
   if (k < Kb) {
     const DeepCand c = deep_candidate(a, k);
     s_c[k] = c;
-    float hi = 0.0f, lo = 0.0f;
-    if (c.valid && c.delta != 0.0f)
-      for (int t = 0; t < a.ntiles; ++t) two_sum_add(hi, lo, a.partial[(size_t)k * a.ntiles + t]);
-    const float d = c.valid ? hi + lo : __int_as_float(0x7fc00000);
+    const float sum = c.valid && c.delta != 0.0f
+                          ? ordered_sum(a.partial + (size_t)k * a.ntiles, a.ntiles) : 0.0f;
+    const float d = c.valid ? sum : __int_as_float(0x7fc00000);
     s_dS[k] = d;
     if (a.n_explicit > 0) {
       a.ex_out[k] = (double)d;

@@ -436,6 +436,21 @@ __device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
   lo += err;
 }
 
+// Compensated sum of x[0 .. n) in index order: the same additions, in the same order, as one
+// two_sum_add per term, with the loads of 32 terms in flight at a time.
+__device__ __forceinline__ float ordered_sum(const float* x, int n) {
+  float hi = 0.0f, lo = 0.0f;
+  for (int q0 = 0; q0 < n; q0 += 32) {
+    float v[32];
+#pragma unroll
+    for (int u = 0; u < 32; ++u) v[u] = q0 + u < n ? x[q0 + u] : 0.0f;
+#pragma unroll
+    for (int u = 0; u < 32; ++u)
+      if (q0 + u < n) two_sum_add(hi, lo, v[u]);
+  }
+  return hi + lo;
+}
+
 // Lane 0 receives the compensated sum of the warp's (hi, lo) pairs (fixed xor tree).
 __device__ __forceinline__ float warp_sum_comp(float hi, float lo) {
 #pragma unroll

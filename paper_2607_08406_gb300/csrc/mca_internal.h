@@ -281,7 +281,7 @@ cudaError_t launch_tfm_tc_split(const TfmArgs& a, cudaStream_t s);
 cudaError_t launch_tfm_tc_eval(const TfmArgs& a, cudaStream_t s);      // grid (Kb, B / 2)
 cudaError_t launch_tfm_tc_commit(const TfmArgs& a, cudaStream_t s);    // grid B / 2
 cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s);   // grid B / 2
-cudaError_t launch_tfm_tc_image_update(const TfmArgs& a, cudaStream_t s);
+// After the commit kernel: the accepted weight's image entry and, with a scratch slot, adoption.
 cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s);     // grid (B, nL + 1)
 
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.

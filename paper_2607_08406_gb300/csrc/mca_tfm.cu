@@ -429,10 +429,9 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
   if (k < Kb) {
     const DeepCand c = tfm_candidate(a, k);
     s_c[k] = c;
-    float hi = 0.0f, lo = 0.0f;
-    if (c.valid && c.delta != 0.0f)
-      for (int q = 0; q < a.B; ++q) two_sum_add(hi, lo, a.partial[(size_t)k * a.B + q]);
-    const float d = c.valid ? hi + lo : __int_as_float(0x7fc00000);
+    const float sum = c.valid && c.delta != 0.0f ? ordered_sum(a.partial + (size_t)k * a.B, a.B)
+                                                  : 0.0f;
+    const float d = c.valid ? sum : __int_as_float(0x7fc00000);
     s_dS[k] = d;
     if (a.n_explicit > 0) {
       a.ex_out[k] = (double)d;

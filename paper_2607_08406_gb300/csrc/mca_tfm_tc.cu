@@ -31,7 +31,8 @@
 // evaluation computed (same images, same terms) and writes the cached residual streams and
 // sequence losses; the image entry of the accepted weight is refreshed after it. In the trial loop
 // the evaluation of candidate k < nscr also writes what the commit would write into scratch slot
-// k, and an accepted candidate with a slot is adopted by copying it (the commit kernel returns).
+// k, and an accepted candidate with a slot is adopted by copying it (the commit kernel returns;
+// the copy kernel also refreshes the image entry).
 #include <cstdio>
 
 #include "mca_device.cuh"
@@ -802,11 +803,9 @@ __global__ void tfm_tc_split_kernel(TfmArgs a) {
   }
 }
 
-// After a commit: the image entry of the accepted weight-matrix parameter.
-__global__ void tfm_tc_image_update_kernel(TfmArgs a) {
-  const DeepCtl* ctl = a.ctl;
-  if (ctl->kstar < 0) return;
-  const DeepCand c = ctl->acc;
+// The image entry of the accepted weight-matrix parameter (after the commit kernel, which reads the
+// old one).
+__device__ void image_update(const TfmArgs& a, const DeepCand& c) {
   const Target tg = tc_target(a, c.idx, c.layer);
   if (tg.mat == kTcMatNone) return;
   const float w = a.params[c.idx];
@@ -816,15 +815,17 @@ __global__ void tfm_tc_image_update_kernel(TfmArgs a) {
   a.wimg[o + tc_image_lo(tfm_tc_rows(tg.mat))] = tf32_rna(w - hi);
 }
 
-// After the decision: the accepted candidate's residual streams (the stages its evaluation
-// recomputed: X[0 ..] for an embedding, X[b + 1 ..] for block b, none for the final LN and head)
-// and sequence losses, copied from its scratch slot. CTA (s, x) copies sequence s of stream x;
+// After the decision and the commit kernel: the image entry of the accepted weight (CTA (0, 0)),
+// and, for an accepted candidate with a scratch slot, its residual streams (the stages its
+// evaluation recomputed: X[0 ..] for an embedding, X[b + 1 ..] for block b, none for the final LN
+// and head) and sequence losses, copied from the slot. CTA (s, x) copies sequence s of stream x;
 // sequences the evaluation skipped (a token embedding whose token they do not contain) keep theirs.
 __global__ void tfm_tc_adopt_kernel(TfmArgs a) {
   const int ks = a.ctl->kstar;
-  if (ks < 0 || ks >= a.nscr) return;
+  if (ks < 0) return;
   const DeepCand cd = a.ctl->acc;
-  if (!cd.valid || cd.delta == 0.0f) return;
+  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) image_update(a, cd);
+  if (ks >= a.nscr || !cd.valid || cd.delta == 0.0f) return;
   const int s = blockIdx.x, x = blockIdx.y;
   __shared__ int s_skip;
   if (threadIdx.x == 0) {
@@ -881,9 +882,5 @@ cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_tfm_tc_image_update(const TfmArgs& a, cudaStream_t s) {
-  tfm_tc_image_update_kernel<<<1, 1, 0, s>>>(a);
-  return cudaGetLastError();
-}
 
 }  // namespace mca
