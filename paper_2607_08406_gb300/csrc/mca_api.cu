@@ -654,7 +654,7 @@ mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
 
 struct TfmMem {
   size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, prop, scratch,
-      wimg, scrX, scr_ell, total;
+      wimg, Xmid, scrX, scr_ell, total;
   int nscr;
 };
 
@@ -668,10 +668,11 @@ bool tfm_use_tc(const mca_tfm_spec& t, long long B) {
 }
 
 // Scratch slots of the tensor-core Transformer kernels: candidate k < nscr of a batch writes its
-// residual streams and sequence losses to slot k, min(K, kTfmScrSlots) slots within 8 GiB.
+// residual streams (X and the mid streams) and sequence losses to slot k, min(K, kTfmScrSlots)
+// slots within 8 GiB.
 int tfm_scratch_slots(const mca_tfm_spec& t, long long B, int K, bool tc) {
   if (!tc || !adopt_enabled()) return 0;
-  const size_t slot = sizeof(float) * ((size_t)(t.n_layer + 1) * B * t.ctx * t.d_model + B);
+  const size_t slot = sizeof(float) * ((size_t)(2 * t.n_layer + 1) * B * t.ctx * t.d_model + B);
   const size_t cap = (size_t)8 << 30;
   return (int)std::min<size_t>((size_t)std::min(K, mca::kTfmScrSlots), cap / slot);
 }
@@ -699,8 +700,9 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc, int 
   M.prop = take(sizeof(mca_trace_rec) * mca::kKmax);
   M.scratch = take(sizeof(int) * 8);
   M.wimg = tc ? take(sizeof(float) * mca::tfm_tc_image_floats(t.d_ff, t.n_layer)) : 0;
+  M.Xmid = take(tc ? sizeof(float) * (size_t)t.n_layer * B * t.ctx * t.d_model : 0);
   M.nscr = tfm_scratch_slots(t, B, K, tc);
-  M.scrX = take(sizeof(float) * (size_t)M.nscr * (t.n_layer + 1) * B * t.ctx * t.d_model);
+  M.scrX = take(sizeof(float) * (size_t)M.nscr * (2 * t.n_layer + 1) * B * t.ctx * t.d_model);
   M.scr_ell = take(sizeof(float) * (size_t)M.nscr * B);
   M.total = o;
   return M;
@@ -738,6 +740,7 @@ mca::TfmArgs tfm_args(mca_handle* h) {
   a.params = h->params;
   a.tokens = h->tokens;
   a.X = h->X;
+  a.Xmid = h->tfm_Xmid;
   a.ell = h->ell;
   a.op = h->dom.op;
   a.lo = h->dom.lo;
@@ -1518,6 +1521,7 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->ex_out = reinterpret_cast<double*>(base + M.ex_out);
   h->prop = reinterpret_cast<mca_trace_rec*>(base + M.prop);
   h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
+  h->tfm_Xmid = h->tc ? reinterpret_cast<float*>(base + M.Xmid) : nullptr;
   h->nscr = M.nscr;
   h->tfm_scrX = reinterpret_cast<float*>(base + M.scrX);
   h->tfm_scr_ell = reinterpret_cast<float*>(base + M.scr_ell);

@@ -236,6 +236,7 @@ struct TfmArgs {
   float* params;             // [P]
   const int* tokens;         // [B x (T + 1)]
   float* X;                  // [(nL + 1) x B x T x d] residual stream entering block b (b = nL: final)
+  float* Xmid;               // [nL x B x T x d] block b's stream after its attention sub-block (tc)
   float* ell;                // [B] per-sequence loss sums
   int loss_unused;
   int op;
@@ -263,8 +264,8 @@ struct TfmArgs {
   int tc;                    // 1: the tensor-core kernels (mca_tfm_tc.cu) run the sequences
   float* wimg;               // their split-weight images (mca_tc_layout.h), tc = 1 only
   // scratch slots (tc = 1, trial loop only): candidate k < nscr of a batch writes the residual
-  // streams it recomputes to slot k of scrX ([nscr][(nL + 1) x B x T x d]) and its sequence losses
-  // to scr_ell ([nscr][B]); an accepted candidate with a slot is adopted from it
+  // streams it recomputes to slot k of scrX ([nscr][(2 nL + 1) x B x T x d]: X, then Xmid) and its
+  // sequence losses to scr_ell ([nscr][B]); an accepted candidate with a slot is adopted from it
   float* scrX;
   float* scr_ell;
   int nscr;
@@ -282,7 +283,7 @@ cudaError_t launch_tfm_tc_eval(const TfmArgs& a, cudaStream_t s);      // grid (
 cudaError_t launch_tfm_tc_commit(const TfmArgs& a, cudaStream_t s);    // grid B / 2
 cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s);   // grid B / 2
 // After the commit kernel: the accepted weight's image entry and, with a scratch slot, adoption.
-cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s);     // grid (B, nL + 1)
+cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s);     // grid (B, 2 nL + 1)
 
 // Launchers (mca_mlp2.cu). All enqueue on `stream` and return the CUDA error of the launch.
 cudaError_t launch_transpose_pad(const float* X, int N, int D, float* XT, int Np, cudaStream_t s);
@@ -420,6 +421,7 @@ struct mca_handle {
   int* tokens = nullptr;                 // [B x (ctx + 1)]
   float* X = nullptr;                    // cached residual stream at every stage
   float* tfm_img = nullptr;
+  float* tfm_Xmid = nullptr;             // its mid streams (after each block's attention)
   float* tfm_scrX = nullptr;             // Transformer tensor-core path: candidate scratch slots
   float* tfm_scr_ell = nullptr;          // (h->nscr of them)              // split-weight images of the tensor-core kernels (tc)
 };

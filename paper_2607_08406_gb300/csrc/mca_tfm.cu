@@ -409,12 +409,14 @@ __global__ void __launch_bounds__(kTfmThreads, 1) tfm_seq_kernel(TfmArgs a) {
   }
 }
 
-// FLOPs of recomputing one sequence from stage b0 (-1 = embeddings) to the loss.
-__device__ __forceinline__ unsigned long long tfm_seq_flops(const TfmArgs& a, int b0) {
+// FLOPs of recomputing one sequence from stage b0 (-1 = embeddings) to the loss; ffn: the first
+// block starts at its feed-forward sub-block (the tensor-core kernels).
+__device__ __forceinline__ unsigned long long tfm_seq_flops(const TfmArgs& a, int b0, bool ffn) {
   const unsigned long long T = a.T, d = a.d, F = a.F, H = a.H, dh = a.dh, V = a.V;
-  const unsigned long long blk = 3ull * T * d * d + 2ull * H * T * T * dh + T * d * d + 2ull * T * d * F;
+  const unsigned long long attn = 3ull * T * d * d + 2ull * H * T * T * dh + T * d * d;
+  const unsigned long long blk = attn + 2ull * T * d * F;
   const int nb = a.nL - (b0 < 0 ? 0 : b0);
-  return 2ull * ((unsigned long long)(nb > 0 ? nb : 0) * blk + T * d * V);
+  return 2ull * ((unsigned long long)(nb > 0 ? nb : 0) * blk - (ffn ? attn : 0ull) + T * d * V);
 }
 
 // One CTA: dS per candidate (fixed order over sequences, compensated fp32), the decision (Eq. 6),
@@ -513,7 +515,8 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
   for (int q = 0; q < Kb; ++q) {
     ncand += s_c[q].valid ? 1ull : 0ull;
     if (s_c[q].valid && s_c[q].delta != 0.0f)
-      flops += tfm_seq_flops(a, s_c[q].layer) * (unsigned long long)a.B;
+      flops += tfm_seq_flops(a, s_c[q].layer, a.tc && tfm_ffn_param(a, s_c[q].idx, s_c[q].layer)) *
+               (unsigned long long)a.B;
   }
   st->candidates += ncand;
   st->alg_flops += flops;

@@ -14,6 +14,14 @@ __device__ __forceinline__ int tfm_stage(const TfmArgs& a, unsigned long long id
   return a.nL;
 }
 
+// Whether parameter idx of block `stage` belongs to that block's feed-forward sub-block (LN2, W1,
+// b1, W2, b2, the last ones of a block): its block's attention sub-block is unchanged, so a
+// recomputation can start from the block's cached mid stream.
+__device__ __forceinline__ bool tfm_ffn_param(const TfmArgs& a, unsigned long long idx, int stage) {
+  return stage >= 0 && stage < a.nL &&
+         idx - a.o_blk0 - (unsigned long long)stage * a.blk_size >= a.r_ln2g;
+}
+
 __device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {
   unsigned int idx;
   uint32_t r1 = 0u;

@@ -1,7 +1,9 @@
 // Character-level Transformer on the 5th-generation tensor cores: the trial loop's recomputation of
-// a sequence from the first stage a mutated parameter feeds (Section 2.4's cached forward, applied to
-// the pre-LN GPT network of Section 2.5), with every dense projection as error-compensated 3xTF32
-// tcgen05 MMAs and the accumulators in tensor memory.
+// a sequence from the first sub-block a mutated parameter feeds (Section 2.4's cached forward,
+// applied to the pre-LN GPT network of Section 2.5), with every dense projection as
+// error-compensated 3xTF32 tcgen05 MMAs and the accumulators in tensor memory. Cached per sequence:
+// the stream entering each block and, after each block's attention sub-block, its mid stream; a
+// parameter of a block's feed-forward sub-block (LN2, W1, b1, W2, b2) restarts there.
 //
 // One CTA, 512 threads, recomputes two sequences for one candidate: M = 128 token rows, rows 0-63
 // the even sequence and 64-127 the odd one. Thread (warp w, lane) owns token row
@@ -115,7 +117,8 @@ __device__ __forceinline__ Target tc_target(const TfmArgs& a, unsigned long long
   return t;
 }
 
-// Stage of candidate k from its proposal alone.
+// Where candidate k's recomputation starts, from its proposal alone, as a key that orders the
+// recomputations by length: 2 stage, plus 1 for a block's feed-forward sub-block.
 __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
   unsigned int idx;
   if (a.n_explicit > 0) {
@@ -124,7 +127,8 @@ __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
     const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
     idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
   }
-  return tfm_stage(a, idx);
+  const int st = tfm_stage(a, idx);
+  return 2 * st + (tfm_ffn_param(a, idx, st) ? 1 : 0);
 }
 
 struct Ctx {
@@ -137,6 +141,8 @@ struct Ctx {
   uint32_t trow;             // this warp's lane quarter in a tensor-memory address
   int r, g, sl, t;           // token row, column part, sequence of the pair, position
   int b0s, nb, cpb, total;   // first block run, blocks run, chunks per block, chunks in all
+  int q0, nbc;               // the first block's first chunk (its FFN's when ffn0), block chunks run
+  bool ffn0;                 // the first block starts at its feed-forward sub-block
   unsigned long long midx;   // patched parameter (~0: none)
   float mval, dlt;           // its value, and the change of a weight-matrix entry
   int cstage;                // the stage the candidate feeds (-1 embeddings)
@@ -154,8 +160,8 @@ struct Issuer {
 
 __device__ __forceinline__ void chunk_src(const TfmArgs& a, const Ctx& c, int x, const float*& src,
                                           uint32_t& bytes) {
-  if (x < c.nb * c.cpb) {
-    const int jb = x / c.cpb, q = x - jb * c.cpb;
+  if (x < c.nbc) {
+    const int xx = x + c.q0, jb = xx / c.cpb, q = xx - jb * c.cpb;
     const float* base = a.wimg + (size_t)(c.b0s + jb) * tfm_tc_block_floats(a.F);
     if (q < kFfnChunk0) {
       src = base + (size_t)q * 4096;
@@ -170,7 +176,7 @@ __device__ __forceinline__ void chunk_src(const TfmArgs& a, const Ctx& c, int x,
     }
     bytes = 16384;
   } else {
-    src = a.wimg + (size_t)a.nL * tfm_tc_block_floats(a.F) + (size_t)(x - c.nb * c.cpb) * 4096;
+    src = a.wimg + (size_t)a.nL * tfm_tc_block_floats(a.F) + (size_t)(x - c.nbc) * 4096;
     bytes = 16384;
   }
 }
@@ -207,8 +213,8 @@ __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
     bool lo_tm = false;                          // A's lo part in tensor memory (A2)
     int kc;
     bool first;
-    if (x < c.nb * c.cpb) {
-      const int q = x % c.cpb;
+    if (x < c.nbc) {
+      const int q = (x + c.q0) % c.cpb;
       if (q < kWoChunk0) {                       // Wq, Wk, Wv
         dcol = kColQ + 128u * (uint32_t)(q >> 3);
         kc = q & 7;
@@ -230,7 +236,7 @@ __device__ bool issue(const TfmArgs& a, const Ctx& c, Issuer& is, int x0, int n,
         }
       }
     } else {                                     // head
-      kc = x - c.nb * c.cpb;
+      kc = x - c.nbc;
       first = kc == 0;
     }
     const uint32_t lbo = R * 16u;
@@ -510,8 +516,10 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   const size_t seq_floats = (size_t)kT * kD;
   const bool slot = MODE == kTfmEval && k < a.nscr;
   float* const xout = MODE != kTfmEval ? a.X
-                      : slot ? a.scrX + (size_t)k * (size_t)(a.nL + 1) * a.B * seq_floats
+                      : slot ? a.scrX + (size_t)k * (size_t)(2 * a.nL + 1) * a.B * seq_floats
                              : nullptr;
+  float* const xmout = MODE != kTfmEval ? a.Xmid
+                       : slot ? xout + (size_t)(a.nL + 1) * a.B * seq_floats : nullptr;
   float* const lout = MODE != kTfmEval ? a.ell : slot ? a.scr_ell + (size_t)k * a.B : nullptr;
   if (!cd.valid || cd.delta == 0.0f) {
     if (MODE == kTfmEval && tid < 2) part[tid] = 0.0f;
@@ -545,7 +553,10 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   c.b0s = b0 < 0 ? 0 : b0;
   c.nb = a.nL - c.b0s;
   c.cpb = kFfnChunk0 + kFfnPerPair * (a.F / kHp);
-  c.total = c.nb * c.cpb + kHeadChunks;
+  c.ffn0 = !fwd && tfm_ffn_param(a, cd.idx, cd.layer);
+  c.q0 = c.ffn0 ? kFfnChunk0 : 0;
+  c.nbc = c.nb * c.cpb - c.q0;
+  c.total = c.nbc + kHeadChunks;
 
   // tensor memory, the stage ring, the first chunks
   if (warp == 0) {
@@ -557,7 +568,10 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   Issuer& is = s_is;
   if (tid == 0) {
     is.nload = is.nwait = is.ncommit = 0;
-    is.limit = c.nb > 0 ? kWoChunk0 : kHeadChunks;
+    // loads stop at the first output projection after an attention step (K and V take the stages)
+    is.limit = c.nb == 0 ? kHeadChunks
+               : !c.ffn0 ? kWoChunk0
+               : c.nb > 1 ? c.cpb - c.q0 + kWoChunk0 : c.total;
   }
   if (tid == 0) {
     for (int q = 0; q < kStages; ++q) {
@@ -589,7 +603,8 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
         reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
     }
   } else {
-    const float* src = a.X + ((size_t)b0 * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+    const float* src = (c.ffn0 ? a.Xmid : a.X) + ((size_t)b0 * a.B + s0 + c.sl) * seq_floats +
+                       (size_t)c.t * kD + 32 * c.g;
 #pragma unroll
     for (int i = 0; i < 8; ++i)
       *reinterpret_cast<float4*>(xr + 4 * i) = reinterpret_cast<const float4*>(src)[i];
@@ -602,64 +617,72 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   for (int b = c.b0s; ok && b < a.nL; ++b) {
     const bool here = b == c.cstage;
     const unsigned long long base = a.o_blk0 + (unsigned long long)b * a.blk_size;
-    // ---- attention: LN1, Q K V, attention, output projection
-    ln_to_a(a, c, base + a.r_ln1g, base + a.r_ln1b,
-            (here && c.tg.mat >= kTcQ && c.tg.mat <= kTcV) ? c.tg.col : -1, s_part, s_acol);
-    tc_publish_operands();
-    __syncthreads();
-    mma_phase(a, c, is, gc, kQkvChunks, s_full, s_empty, fail);
-    gc += kQkvChunks;
-    if (!(ok = group_done(s_empty, gc - 1, fail))) break;
-    float q[32];
-    {
-      float v[32];
-#pragma unroll
-      for (int p = 0; p < 2; ++p) {
-        ld32(c, (p ? kColV : kColK) + 32u * (uint32_t)c.g, v);
-        const unsigned long long bb = base + (p ? a.r_bv : a.r_bk) + 32 * c.g;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] += prm(a, bb + i, c.midx, c.mval);
-        if (here && c.tg.mat == (p ? kTcV : kTcK)) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
-        float* dst = (p ? c.vs : c.ks) + (size_t)c.r * kD + 32 * c.g;
-#pragma unroll
+    if (!(c.ffn0 && b == c.b0s)) {   // (a feed-forward candidate's block starts at its mid stream)
+      // ---- attention: LN1, Q K V, attention, output projection
+      ln_to_a(a, c, base + a.r_ln1g, base + a.r_ln1b,
+              (here && c.tg.mat >= kTcQ && c.tg.mat <= kTcV) ? c.tg.col : -1, s_part, s_acol);
+      tc_publish_operands();
+      __syncthreads();
+      mma_phase(a, c, is, gc, kQkvChunks, s_full, s_empty, fail);
+      gc += kQkvChunks;
+      if (!(ok = group_done(s_empty, gc - 1, fail))) break;
+      float q[32];
+      {
+        float v[32];
+  #pragma unroll
+        for (int p = 0; p < 2; ++p) {
+          ld32(c, (p ? kColV : kColK) + 32u * (uint32_t)c.g, v);
+          const unsigned long long bb = base + (p ? a.r_bv : a.r_bk) + 32 * c.g;
+  #pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += prm(a, bb + i, c.midx, c.mval);
+          if (here && c.tg.mat == (p ? kTcV : kTcK)) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
+          float* dst = (p ? c.vs : c.ks) + (size_t)c.r * kD + 32 * c.g;
+  #pragma unroll
+          for (int i = 0; i < 8; ++i)
+            *reinterpret_cast<float4*>(dst + 4 * (i ^ (c.r & 7))) =
+                make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+        ld32(c, kColQ + 32u * (uint32_t)c.g, q);
+        const unsigned long long bq = base + a.r_bq + 32 * c.g;
+  #pragma unroll
+        for (int i = 0; i < 32; ++i) q[i] += prm(a, bq + i, c.midx, c.mval);
+        if (here && c.tg.mat == kTcQ) add_at(q, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
+      }
+      __syncthreads();             // K and V complete
+      {
+        float o[32];
+        attention(c, q, o);
+        __syncthreads();           // every row done with K and V: their memory takes the next A
+        if (here && c.tg.mat == kTcO) {
+  #pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (32 * c.g + i == c.tg.col) s_acol[c.r] = o[i];
+        }
+        store_a<32>(c, o, kColA + 32u * (uint32_t)c.g, c.alo, 32 * c.g);
+      }
+      if (tid == 0) {              // loads may now run into the next block's Q, K, V chunks
+        const int jb = b - c.b0s;
+        is.limit = jb + 1 < c.nb ? (jb + 1) * c.cpb - c.q0 + kWoChunk0 : c.total;
+      }
+      tc_publish_operands();
+      __syncthreads();
+      mma_phase(a, c, is, gc, kFfnChunk0 - kWoChunk0, s_full, s_empty, fail);
+      gc += kFfnChunk0 - kWoChunk0;
+      if (!(ok = group_done(s_empty, gc - 1, fail))) break;
+      {
+        float v[32];
+        ld32(c, kColU + 32u * (uint32_t)c.g, v);
+        if (here && c.tg.mat == kTcO) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
+        const unsigned long long bo = base + a.r_bo + 32 * c.g;
+  #pragma unroll
+        for (int i = 0; i < 32; ++i) xr[i] += v[i] + prm(a, bo + i, c.midx, c.mval);
+      }
+      if (xmout && !s_skip[c.sl]) {    // the mid stream: block b after its attention sub-block
+        float* dst = xmout + ((size_t)b * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+  #pragma unroll
         for (int i = 0; i < 8; ++i)
-          *reinterpret_cast<float4*>(dst + 4 * (i ^ (c.r & 7))) =
-              make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
       }
-      ld32(c, kColQ + 32u * (uint32_t)c.g, q);
-      const unsigned long long bq = base + a.r_bq + 32 * c.g;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) q[i] += prm(a, bq + i, c.midx, c.mval);
-      if (here && c.tg.mat == kTcQ) add_at(q, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
-    }
-    __syncthreads();             // K and V complete
-    {
-      float o[32];
-      attention(c, q, o);
-      __syncthreads();           // every row done with K and V: their memory takes the next A
-      if (here && c.tg.mat == kTcO) {
-#pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (32 * c.g + i == c.tg.col) s_acol[c.r] = o[i];
-      }
-      store_a<32>(c, o, kColA + 32u * (uint32_t)c.g, c.alo, 32 * c.g);
-    }
-    if (tid == 0) {              // loads may now run into the next block's Q, K, V chunks
-      const int jb = b - c.b0s;
-      is.limit = jb + 1 < c.nb ? (jb + 1) * c.cpb + kWoChunk0 : c.total;
-    }
-    tc_publish_operands();
-    __syncthreads();
-    mma_phase(a, c, is, gc, kFfnChunk0 - kWoChunk0, s_full, s_empty, fail);
-    gc += kFfnChunk0 - kWoChunk0;
-    if (!(ok = group_done(s_empty, gc - 1, fail))) break;
-    {
-      float v[32];
-      ld32(c, kColU + 32u * (uint32_t)c.g, v);
-      if (here && c.tg.mat == kTcO) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
-      const unsigned long long bo = base + a.r_bo + 32 * c.g;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) xr[i] += v[i] + prm(a, bo + i, c.midx, c.mval);
     }
     // ---- feed-forward network: W1 for two 64-wide hidden chunks at a time (N = 128), then per
     // chunk the activation as A2 and its W2 product
@@ -816,10 +839,12 @@ __device__ void image_update(const TfmArgs& a, const DeepCand& c) {
 }
 
 // After the decision and the commit kernel: the image entry of the accepted weight (CTA (0, 0)),
-// and, for an accepted candidate with a scratch slot, its residual streams (the stages its
-// evaluation recomputed: X[0 ..] for an embedding, X[b + 1 ..] for block b, none for the final LN
-// and head) and sequence losses, copied from the slot. CTA (s, x) copies sequence s of stream x;
-// sequences the evaluation skipped (a token embedding whose token they do not contain) keep theirs.
+// and, for an accepted candidate with a scratch slot, its residual streams (those its evaluation
+// recomputed: X[0 ..] and Xmid[0 ..] for an embedding; X[b + 1 ..] and Xmid[b ..] for block b,
+// Xmid[b + 1 ..] for its feed-forward sub-block; none for the final LN and head) and sequence
+// losses, copied from the slot. CTA (s, x) copies sequence s of stream x (X for x <= nL, then
+// Xmid); sequences the evaluation skipped (a token embedding whose token they do not contain) keep
+// theirs.
 __global__ void tfm_tc_adopt_kernel(TfmArgs a) {
   const int ks = a.ctl->kstar;
   if (ks < 0) return;
@@ -839,12 +864,17 @@ __global__ void tfm_tc_adopt_kernel(TfmArgs a) {
   __syncthreads();
   if (s_skip) return;
   if (x == 0 && threadIdx.x == 0) a.ell[s] = a.scr_ell[(size_t)ks * a.B + s];
-  if (x < (cd.layer < 0 ? 0 : cd.layer + 1)) return;
+  const bool mid = x > a.nL;
+  const int xs = mid ? x - a.nL - 1 : x;                // stream within X or Xmid
+  const int first = cd.layer < 0 ? 0
+                    : mid && !tfm_ffn_param(a, cd.idx, cd.layer) ? cd.layer : cd.layer + 1;
+  if (xs < first) return;
   const size_t seq_floats = (size_t)kT * kD;
-  const size_t at = ((size_t)x * a.B + s) * seq_floats;
-  const float4* src = reinterpret_cast<const float4*>(
-      a.scrX + (size_t)ks * (size_t)(a.nL + 1) * a.B * seq_floats + at);
-  float4* dst = reinterpret_cast<float4*>(a.X + at);
+  const size_t at = ((size_t)xs * a.B + s) * seq_floats;
+  const float* sb = a.scrX + (size_t)ks * (size_t)(2 * a.nL + 1) * a.B * seq_floats +
+                    (mid ? (size_t)(a.nL + 1) * a.B * seq_floats : 0);
+  const float4* src = reinterpret_cast<const float4*>(sb + at);
+  float4* dst = reinterpret_cast<float4*>((mid ? a.Xmid : a.X) + at);
   for (int q = threadIdx.x; q < (int)(seq_floats / 4); q += blockDim.x) dst[q] = src[q];
 }
 
@@ -878,7 +908,7 @@ cudaError_t launch_tfm_tc_forward(const TfmArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_tfm_tc_adopt(const TfmArgs& a, cudaStream_t s) {
-  tfm_tc_adopt_kernel<<<dim3(a.B, a.nL + 1), 256, 0, s>>>(a);
+  tfm_tc_adopt_kernel<<<dim3(a.B, 2 * a.nL + 1), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

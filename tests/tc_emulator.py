@@ -106,6 +106,7 @@ class Args:
         assert self.P == self.params.shape[0]
         self.tokens = np.asarray(tokens, dtype=np.int32)
         self.X = np.zeros((self.nL + 1, self.B, c, d), np.float32)
+        self.Xmid = np.zeros((self.nL, self.B, c, d), np.float32)   # after each block's attention
         self.ell = np.zeros(self.B, np.float32)
         self.wimg = None
 
@@ -163,6 +164,11 @@ def tfm_stage(a, idx):
     return a.nL
 
 
+def ffn_param(a, idx, stage):
+    """A parameter of block `stage`'s feed-forward sub-block (LN2, W1, b1, W2, b2)."""
+    return 0 <= stage < a.nL and idx - a.o_blk0 - stage * a.blk_size >= a.r_ln2g
+
+
 # ---------------------------------------------------------------- the CTA
 
 class Bar:
@@ -174,23 +180,28 @@ class Slot:
     """A candidate's scratch slot: the residual streams and sequence losses its evaluation writes."""
     def __init__(self, a):
         self.X = np.full_like(a.X, np.nan)
+        self.Xmid = np.full_like(a.Xmid, np.nan)
         self.ell = np.full_like(a.ell, np.nan)
 
 
 def adopt(a, slot, cand):
-    """The adopt kernel: the accepted candidate's recomputed streams (X[0..] for an embedding,
-    X[b+1..] for block b, none for the head stage) and losses from its slot, sequences it skipped
-    (a token embedding whose token they lack) left as they are."""
+    """The adopt kernel: the accepted candidate's recomputed streams (X[0..] and Xmid[0..] for an
+    embedding; X[b+1..] and Xmid[b..] for block b, Xmid[b+1..] for its feed-forward sub-block; none
+    for the head stage) and losses from its slot, sequences it skipped (a token embedding whose
+    token they lack) left as they are."""
     idx, neww, delta, layer, row = cand
     if delta == 0.0:
         return
     first = 0 if layer < 0 else layer + 1
+    first_mid = 0 if layer < 0 else (layer + 1 if ffn_param(a, idx, layer) else layer)
     for s in range(a.B):
         if row >= 0 and np.all(a.tokens[s, :kT] != row):
             continue
         a.ell[s] = slot.ell[s]
         for x in range(first, a.nL + 1):
             a.X[x, s] = slot.X[x, s]
+        for x in range(first_mid, a.nL):
+            a.Xmid[x, s] = slot.Xmid[x, s]
 
 
 class CTA:
@@ -215,8 +226,8 @@ class CTA:
     # -------- ring
     def chunk_src(self, x):
         A = self.a
-        if x < self.nb * self.cpb:
-            jb, q = divmod(x, self.cpb)
+        if x < self.nbc:
+            jb, q = divmod(x + self.q0, self.cpb)
             base = (self.b0s + jb) * blk_floats(A.F)
             if q < kFfnChunk0:
                 return base + q * 4096, 16384
@@ -225,7 +236,7 @@ class CTA:
             if u < 8:
                 return base + 131072 + (p * 8 + u) * 4096, 16384
             return base + 131072 + 256 * A.F + (p * 8 + u - 8) * 4096, 16384
-        return A.nL * blk_floats(A.F) + (x - self.nb * self.cpb) * 4096, 16384
+        return A.nL * blk_floats(A.F) + (x - self.nbc) * 4096, 16384
 
     def topup(self, upto):
         end = min(upto, self.limit)
@@ -277,8 +288,8 @@ class CTA:
             self.nwait = x + 1
             dcol, idsc, alo, acol, R = kColU, kIdN128, salo, kColA, 128
             lo_tm = False                       # A's lo part in tensor memory (A2)
-            if x < self.nb * self.cpb:
-                q = x % self.cpb
+            if x < self.nbc:
+                q = (x + self.q0) % self.cpb
                 if q < kWoChunk0:
                     dcol = kColQ + 128 * (q >> 3)
                     kc = q & 7
@@ -296,7 +307,7 @@ class CTA:
                         dcol, lo_tm, acol, kc = kColF, True, kColA2, (u - 8) & 3
                         first = p == 0 and u == 8
             else:
-                kc = x - self.nb * self.cpb
+                kc = x - self.nbc
                 first = kc == 0
             lbo = R * 16
             for ks in range(2):
@@ -445,14 +456,23 @@ class CTA:
         self.b0s = 0 if b0 < 0 else b0
         self.nb = a.nL - self.b0s
         self.cpb = kFfnChunk0 + kFfnPerPair * (a.F // kHp)
-        self.total = self.nb * self.cpb + kHeadChunks
+        self.ffn0 = mode != FORWARD and ffn_param(a, idx, layer)
+        self.q0 = kFfnChunk0 if self.ffn0 else 0
+        self.nbc = self.nb * self.cpb - self.q0
+        self.total = self.nbc + kHeadChunks
         self.nload = self.nwait = self.ncommit = 0
-        self.limit = kWoChunk0 if self.nb > 0 else kHeadChunks
+        if self.nb == 0:
+            self.limit = kHeadChunks
+        elif not self.ffn0:
+            self.limit = kWoChunk0
+        else:
+            self.limit = self.cpb - self.q0 + kWoChunk0 if self.nb > 1 else self.total
         self.loaded_regions = []
         self.topup(kStages)
         self.s_acol = np.zeros(128, np.float32)
         # residual
         xout = a.X if mode != EVAL else (self.slot.X if self.slot is not None else None)
+        xmout = a.Xmid if mode != EVAL else (self.slot.Xmid if self.slot is not None else None)
         lout = a.ell if mode != EVAL else (self.slot.ell if self.slot is not None else None)
         xs = np.zeros((128, kD), np.float32)
         if b0 < 0:
@@ -464,7 +484,7 @@ class CTA:
                     if not skip[q]:
                         xout[0, s0 + q] = xs[q * kT:(q + 1) * kT]
         else:
-            xs[:] = a.X[b0, s0 + sl, t]
+            xs[:] = (a.Xmid if self.ffn0 else a.X)[b0, s0 + sl, t]
         for g in range(4):
             self.sm[self.xr_addr(g)[:, None] + np.arange(32)[None, :]] = xs[:, 32 * g:32 * g + 32]
         gc = 0
@@ -472,61 +492,67 @@ class CTA:
         for b in range(self.b0s, a.nL):
             here = b == cstage
             base = a.o_blk0 + b * a.blk_size
-            self.ln_to_a(base + a.r_ln1g, base + a.r_ln1b, tg[2] if (here and kTcQ <= tg[0] <= kTcV) else -1)
-            self.issue(gc, kQkvChunks)
-            gc += kQkvChunks
-            self.group_done(gc - 1)
-            q = np.zeros((4, 128, 32), np.float32)
-            for g in range(4):
-                for p in range(2):
-                    v = self.tm[:, (kColV if p else kColK) + 32 * g:(kColV if p else kColK) + 32 * g + 32].copy()
-                    bb = base + (a.r_bv if p else a.r_bk) + 32 * g
+            if not (self.ffn0 and b == self.b0s):   # a feed-forward candidate starts at its mid stream
+                self.ln_to_a(base + a.r_ln1g, base + a.r_ln1b, tg[2] if (here and kTcQ <= tg[0] <= kTcV) else -1)
+                self.issue(gc, kQkvChunks)
+                gc += kQkvChunks
+                self.group_done(gc - 1)
+                q = np.zeros((4, 128, 32), np.float32)
+                for g in range(4):
+                    for p in range(2):
+                        v = self.tm[:, (kColV if p else kColK) + 32 * g:(kColV if p else kColK) + 32 * g + 32].copy()
+                        bb = base + (a.r_bv if p else a.r_bk) + 32 * g
+                        for i in range(32):
+                            v[:, i] = v[:, i] + self.prm(bb + i)
+                        if here and tg[0] == (kTcV if p else kTcK):
+                            at = tg[1] - 32 * g
+                            if 0 <= at < 32:
+                                v[:, at] += dlt * self.s_acol
+                        dst = kXsBytes // 4 + (0 if not p else 128 * 128) + r * kD + 32 * g
+                        for i in range(8):
+                            for e in range(4):
+                                self.sm[dst + 4 * (i ^ (r & 7)) + e] = v[:, 4 * i + e]
+                    qq = self.tm[:, kColQ + 32 * g:kColQ + 32 * g + 32].copy()
                     for i in range(32):
-                        v[:, i] = v[:, i] + self.prm(bb + i)
-                    if here and tg[0] == (kTcV if p else kTcK):
+                        qq[:, i] = qq[:, i] + self.prm(base + a.r_bq + 32 * g + i)
+                    if here and tg[0] == kTcQ:
+                        at = tg[1] - 32 * g
+                        if 0 <= at < 32:
+                            qq[:, at] += dlt * self.s_acol
+                    q[g] = qq
+                # K and V overlay the first stages: every load issued so far has been consumed
+                assert self.nload == gc == self.nwait, ("loads outstanding over K/V", self.nload, gc)
+                # check: no load has overwritten K / V since they were written -- loads issued so far
+                kv_lo, kv_hi = kXsBytes, kXsBytes + 2 * 128 * 128 * 4
+                self.kv_guard = len(self.loaded_regions)
+                o = self.attention(q)
+                for (x, st_b, nbytes) in self.loaded_regions[self.kv_guard:]:
+                    assert st_b + nbytes <= kv_lo or st_b >= kv_hi, ("load over K/V", x)
+                if here and tg[0] == kTcO:
+                    g = tg[2] // 32
+                    self.s_acol = o[g, :, tg[2] - 32 * g].copy()
+                for g in range(4):
+                    self.store_a(o[g], kColA + 32 * g, kXsBytes, 32 * g, g, 32)
+                jb = b - self.b0s
+                self.limit = (jb + 1) * self.cpb - self.q0 + kWoChunk0 if jb + 1 < self.nb else self.total
+                self.topup(gc + kStages)
+                self.issue(gc, kFfnChunk0 - kWoChunk0)
+                gc += kFfnChunk0 - kWoChunk0
+                self.group_done(gc - 1)
+                for g in range(4):
+                    v = self.tm[:, kColU + 32 * g:kColU + 32 * g + 32].copy()
+                    if here and tg[0] == kTcO:
                         at = tg[1] - 32 * g
                         if 0 <= at < 32:
                             v[:, at] += dlt * self.s_acol
-                    dst = kXsBytes // 4 + (0 if not p else 128 * 128) + r * kD + 32 * g
-                    for i in range(8):
-                        for e in range(4):
-                            self.sm[dst + 4 * (i ^ (r & 7)) + e] = v[:, 4 * i + e]
-                qq = self.tm[:, kColQ + 32 * g:kColQ + 32 * g + 32].copy()
-                for i in range(32):
-                    qq[:, i] = qq[:, i] + self.prm(base + a.r_bq + 32 * g + i)
-                if here and tg[0] == kTcQ:
-                    at = tg[1] - 32 * g
-                    if 0 <= at < 32:
-                        qq[:, at] += dlt * self.s_acol
-                q[g] = qq
-            # K and V overlay the first stages: every load issued so far has been consumed
-            assert self.nload == gc == self.nwait, ("loads outstanding over K/V", self.nload, gc)
-            # check: no load has overwritten K / V since they were written -- loads issued so far
-            kv_lo, kv_hi = kXsBytes, kXsBytes + 2 * 128 * 128 * 4
-            self.kv_guard = len(self.loaded_regions)
-            o = self.attention(q)
-            for (x, st_b, nbytes) in self.loaded_regions[self.kv_guard:]:
-                assert st_b + nbytes <= kv_lo or st_b >= kv_hi, ("load over K/V", x)
-            if here and tg[0] == kTcO:
-                g = tg[2] // 32
-                self.s_acol = o[g, :, tg[2] - 32 * g].copy()
-            for g in range(4):
-                self.store_a(o[g], kColA + 32 * g, kXsBytes, 32 * g, g, 32)
-            jb = b - self.b0s
-            self.limit = (jb + 1) * self.cpb + kWoChunk0 if jb + 1 < self.nb else self.total
-            self.topup(gc + kStages)
-            self.issue(gc, kFfnChunk0 - kWoChunk0)
-            gc += kFfnChunk0 - kWoChunk0
-            self.group_done(gc - 1)
-            for g in range(4):
-                v = self.tm[:, kColU + 32 * g:kColU + 32 * g + 32].copy()
-                if here and tg[0] == kTcO:
-                    at = tg[1] - 32 * g
-                    if 0 <= at < 32:
-                        v[:, at] += dlt * self.s_acol
-                xa = self.xr_addr(g)
-                for i in range(32):
-                    self.sm[xa + i] = self.sm[xa + i] + (v[:, i] + self.prm(base + a.r_bo + 32 * g + i))
+                    xa = self.xr_addr(g)
+                    for i in range(32):
+                        self.sm[xa + i] = self.sm[xa + i] + (v[:, i] + self.prm(base + a.r_bo + 32 * g + i))
+                if xmout is not None:                  # the mid stream
+                    for q in range(2):
+                        if not skip[q]:
+                            for g in range(4):
+                                xmout[b, s0 + q, :, 32 * g:32 * g + 32] = self.sm[self.xr_addr(g)[q * kT:(q + 1) * kT, None] + np.arange(32)[None, :]]
             self.ln_to_a(base + a.r_ln2g, base + a.r_ln2b, tg[2] if (here and tg[0] == kTcW1) else -1)
             self.issue(gc, 8)
             gc += 8

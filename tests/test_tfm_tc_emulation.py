@@ -84,10 +84,11 @@ def test_emulated_commit_writes_what_evaluation_computed(setup):
 
 
 def test_emulated_adoption_writes_what_the_commit_writes(setup):
-    """An evaluation with a scratch slot followed by the adopt kernel leaves the residual streams and
-    sequence losses exactly as the commit kernel would, for a candidate of every stage kind: token
-    embeddings (one whose token some sequences lack: they keep theirs), a position embedding, a
-    block-0 projection, the last block's FFN and the head."""
+    """An evaluation with a scratch slot followed by the adopt kernel leaves the residual streams
+    (block inputs and mid streams) and sequence losses exactly as the commit kernel would, for a
+    candidate of every stage kind: token embeddings (one whose token some sequences lack: they keep
+    theirs), a position embedding, a block-0 projection, LN2 of block 0 and the last block's FFN
+    (both restart at their block's mid stream) and the head."""
     spec, a0 = setup
     picks = _picks(a0)
     # a token that some sequences contain and others do not
@@ -96,7 +97,8 @@ def test_emulated_adoption_writes_what_the_commit_writes(setup):
     partial = np.nonzero(present.any(axis=1) & ~present.all(axis=1))[0]
     assert len(partial) > 0
     picks["tok_emb_partial"] = int(partial[0]) * a0.d + 11
-    for name in ("tok_emb", "tok_emb_partial", "pos_emb", "wq", "w2", "w_head"):
+    picks["ln2.b0"] = a0.o_blk0 + a0.r_ln2b + 3
+    for name in ("tok_emb", "tok_emb_partial", "pos_emb", "wq", "ln2.b0", "w2", "w_head"):
         a = copy.deepcopy(a0)
         c = _cand(a, picks[name], 0.37)
         slot = E.Slot(a)
@@ -109,6 +111,7 @@ def test_emulated_adoption_writes_what_the_commit_writes(setup):
             E.CTA(a, E.COMMIT, c, p).run()
         E.adopt(b, slot, c)
         np.testing.assert_array_equal(b.X, a.X, err_msg=name)
+        np.testing.assert_array_equal(b.Xmid, a.Xmid, err_msg=name)
         np.testing.assert_array_equal(b.ell, a.ell, err_msg=name)
 
 
