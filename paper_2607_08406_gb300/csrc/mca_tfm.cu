@@ -409,14 +409,17 @@ __global__ void __launch_bounds__(kTfmThreads, 1) tfm_seq_kernel(TfmArgs a) {
   }
 }
 
-// FLOPs of recomputing one sequence from stage b0 (-1 = embeddings) to the loss; ffn: the first
-// block starts at its feed-forward sub-block (the tensor-core kernels).
-__device__ __forceinline__ unsigned long long tfm_seq_flops(const TfmArgs& a, int b0, bool ffn) {
+// FLOPs of recomputing one sequence from stage b0 (-1 = embeddings) to the loss; restart: where
+// the tensor-core kernels start inside block b0 (kRestartFfn: its feed-forward sub-block;
+// kRestartUnit: block b0 + 1, the rank-1 step before it not counted).
+__device__ __forceinline__ unsigned long long tfm_seq_flops(const TfmArgs& a, int b0, int restart) {
   const unsigned long long T = a.T, d = a.d, F = a.F, H = a.H, dh = a.dh, V = a.V;
   const unsigned long long attn = 3ull * T * d * d + 2ull * H * T * T * dh + T * d * d;
   const unsigned long long blk = attn + 2ull * T * d * F;
-  const int nb = a.nL - (b0 < 0 ? 0 : b0);
-  return 2ull * ((unsigned long long)(nb > 0 ? nb : 0) * blk - (ffn ? attn : 0ull) + T * d * V);
+  int nb = a.nL - (b0 < 0 ? 0 : b0);
+  if (restart == kRestartUnit) --nb;
+  return 2ull * ((unsigned long long)(nb > 0 ? nb : 0) * blk -
+                 (restart == kRestartFfn ? attn : 0ull) + T * d * V);
 }
 
 // One CTA: dS per candidate (fixed order over sequences, compensated fp32), the decision (Eq. 6),
@@ -515,7 +518,8 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
   for (int q = 0; q < Kb; ++q) {
     ncand += s_c[q].valid ? 1ull : 0ull;
     if (s_c[q].valid && s_c[q].delta != 0.0f)
-      flops += tfm_seq_flops(a, s_c[q].layer, a.tc && tfm_ffn_param(a, s_c[q].idx, s_c[q].layer)) *
+      flops += tfm_seq_flops(a, s_c[q].layer,
+                             a.tc ? tfm_restart(a, s_c[q].idx, s_c[q].layer) : kRestartBlock) *
                (unsigned long long)a.B;
   }
   st->candidates += ncand;

@@ -14,12 +14,24 @@ __device__ __forceinline__ int tfm_stage(const TfmArgs& a, unsigned long long id
   return a.nL;
 }
 
-// Whether parameter idx of block `stage` belongs to that block's feed-forward sub-block (LN2, W1,
-// b1, W2, b2, the last ones of a block): its block's attention sub-block is unchanged, so a
-// recomputation can start from the block's cached mid stream.
+// Where the recomputation of a candidate in parameter idx of block `stage` starts (Section 2.4's
+// cached forward at sub-block granularity; the tensor-core kernels): kRestartBlock, the block's
+// input; kRestartFfn (LN2 gain or bias), the block's cached mid stream after its attention
+// sub-block; kRestartUnit (W1, b1, W2, b2), one hidden unit of the block's feed-forward network,
+// a rank-1 change of the block's output stream, after which block stage + 1 starts. The block's
+// parameters are laid out ln1, attention, ln2, W1, b1, W2, b2, so the last two kinds are its tail.
+enum TfmRestart { kRestartBlock = 0, kRestartFfn = 1, kRestartUnit = 2 };
+
+__device__ __forceinline__ int tfm_restart(const TfmArgs& a, unsigned long long idx, int stage) {
+  if (stage < 0 || stage >= a.nL) return kRestartBlock;
+  const unsigned long long off = idx - a.o_blk0 - (unsigned long long)stage * a.blk_size;
+  if (off < a.r_ln2g) return kRestartBlock;
+  return off < a.r_w1 ? kRestartFfn : kRestartUnit;
+}
+
+// Whether the candidate leaves its block's attention sub-block (and so its mid stream) unchanged.
 __device__ __forceinline__ bool tfm_ffn_param(const TfmArgs& a, unsigned long long idx, int stage) {
-  return stage >= 0 && stage < a.nL &&
-         idx - a.o_blk0 - (unsigned long long)stage * a.blk_size >= a.r_ln2g;
+  return tfm_restart(a, idx, stage) != kRestartBlock;
 }
 
 __device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {

@@ -118,7 +118,8 @@ __device__ __forceinline__ Target tc_target(const TfmArgs& a, unsigned long long
 }
 
 // Where candidate k's recomputation starts, from its proposal alone, as a key that orders the
-// recomputations by length: 2 stage, plus 1 for a block's feed-forward sub-block.
+// recomputations by length: 4 stage, plus 2 for a block's feed-forward sub-block, plus 3 for one of
+// its hidden units (then block stage + 1, key 4 stage + 4, follows a short rank-1 step).
 __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
   unsigned int idx;
   if (a.n_explicit > 0) {
@@ -128,7 +129,8 @@ __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
     idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
   }
   const int st = tfm_stage(a, idx);
-  return 2 * st + (tfm_ffn_param(a, idx, st) ? 1 : 0);
+  const int rs = tfm_restart(a, idx, st);
+  return 4 * st + (rs == kRestartFfn ? 2 : rs == kRestartUnit ? 3 : 0);
 }
 
 struct Ctx {
@@ -143,6 +145,7 @@ struct Ctx {
   int b0s, nb, cpb, total;   // first block run, blocks run, chunks per block, chunks in all
   int q0, nbc;               // the first block's first chunk (its FFN's when ffn0), block chunks run
   bool ffn0;                 // the first block starts at its feed-forward sub-block
+  bool unit0;                // a hidden unit of block cstage: rank-1 step, then block cstage + 1
   unsigned long long midx;   // patched parameter (~0: none)
   float mval, dlt;           // its value, and the change of a weight-matrix entry
   int cstage;                // the stage the candidate feeds (-1 embeddings)
@@ -382,6 +385,109 @@ __device__ void ln_to_a(const TfmArgs& a, const Ctx& c, unsigned long long og,
   store_a<32>(c, x, kColA + 32u * (uint32_t)c.g, c.alo, 32 * c.g);
 }
 
+// A candidate in W1, b1, W2 or b2 of block b changes one hidden unit j of the block's feed-forward
+// network, so the block's output stream (cached) moves by a rank-1 term: by W2[:, j] (f(u'_j) -
+// f(u_j)) for W1[j][k] and b1[j], by delta f(u_j) on column i for W2[i][j], by delta on column i
+// for b2[i], with u_j = LN2(mid stream) . W1[j, :] + b1[j] recomputed here on the CUDA cores (the
+// candidate's own entry at its old value: in a commit the parameter already holds the new one).
+// The new output stream of this thread's row part goes to xr.
+__device__ void ffn_unit(const TfmArgs& a, const Ctx& c, const DeepCand& cd, int s0, float* xr,
+                         float* s_part, float* s_acol) {
+  const int b = cd.layer;
+  const unsigned long long base = a.o_blk0 + (unsigned long long)b * a.blk_size;
+  const unsigned long long off = (unsigned long long)cd.idx - base;
+  const size_t seq_floats = (size_t)kT * kD;
+  int kind, j = 0, i0 = -1, kcol = -1;       // kind: 0 W1[j][kcol], 1 b1[j], 2 W2[i0][j], 3 b2[i0]
+  if (off < a.r_b1) {
+    kind = 0;
+    j = (int)((off - a.r_w1) / kD);
+    kcol = (int)((off - a.r_w1) % kD);
+  } else if (off < a.r_w2) {
+    kind = 1;
+    j = (int)(off - a.r_b1);
+  } else if (off < a.r_b2) {
+    kind = 2;
+    i0 = (int)((off - a.r_w2) / (unsigned long long)a.F);
+    j = (int)((off - a.r_w2) % (unsigned long long)a.F);
+  } else {
+    kind = 3;
+    i0 = (int)(off - a.r_b2);
+  }
+  const size_t row = ((size_t)(s0 + c.sl)) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+  float xn[32];
+  const float* xo = a.X + (size_t)(b + 1) * a.B * seq_floats + row;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 v = reinterpret_cast<const float4*>(xo)[i];
+    xn[4 * i] = v.x;
+    xn[4 * i + 1] = v.y;
+    xn[4 * i + 2] = v.z;
+    xn[4 * i + 3] = v.w;
+  }
+  if (kind == 3) {
+    add_at(xn, i0 - 32 * c.g, cd.delta);
+  } else {
+    float x[32];
+    const float* xm = a.Xmid + (size_t)b * a.B * seq_floats + row;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float4 v = reinterpret_cast<const float4*>(xm)[i];
+      x[4 * i] = v.x;
+      x[4 * i + 1] = v.y;
+      x[4 * i + 2] = v.z;
+      x[4 * i + 3] = v.w;
+    }
+    float sm = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) sm += x[i];
+    s_part[c.g * kRows + c.r] = sm;
+    __syncthreads();
+    const float mean = (((s_part[c.r] + s_part[kRows + c.r]) + s_part[2 * kRows + c.r]) +
+                        s_part[3 * kRows + c.r]) / (float)kD;
+    float v = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float e = x[i] - mean;
+      v = fmaf(e, e, v);
+    }
+    s_part[(4 + c.g) * kRows + c.r] = v;
+    __syncthreads();
+    const float var = (((s_part[4 * kRows + c.r] + s_part[5 * kRows + c.r]) +
+                        s_part[6 * kRows + c.r]) + s_part[7 * kRows + c.r]) / (float)kD;
+    const float rstd = rsqrtf(var + a.eps);
+    const unsigned long long w1 = base + a.r_w1 + (unsigned long long)j * kD;
+    float p = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int col = 32 * c.g + i;
+      const float ln = (x[i] - mean) * rstd * a.params[base + a.r_ln2g + col] +
+                       a.params[base + a.r_ln2b + col];
+      if (col == kcol) s_acol[c.r] = ln;
+      const float w = w1 + col == cd.idx ? cd.oldw : a.params[w1 + col];
+      p = fmaf(ln, w, p);
+    }
+    s_part[c.g * kRows + c.r] = p;           // every thread has read the means (barrier above)
+    __syncthreads();
+    const float bj = kind == 1 ? cd.oldw : a.params[base + a.r_b1 + j];
+    const float u = ((((s_part[c.r] + s_part[kRows + c.r]) + s_part[2 * kRows + c.r]) +
+                      s_part[3 * kRows + c.r])) + bj;
+    if (kind == 2) {
+      add_at(xn, i0 - 32 * c.g, cd.delta * act_rt(a.act, u, a.g));
+    } else {
+      const float un = kind == 0 ? fmaf(cd.delta, s_acol[c.r], u) : u + cd.delta;
+      const float da = act_rt(a.act, un, a.g) - act_rt(a.act, u, a.g);
+      const unsigned long long w2 = base + a.r_w2 + (unsigned long long)j;
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        xn[i] = fmaf(a.params[w2 + (unsigned long long)(32 * c.g + i) * a.F], da, xn[i]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    *reinterpret_cast<float4*>(xr + 4 * i) =
+        make_float4(xn[4 * i], xn[4 * i + 1], xn[4 * i + 2], xn[4 * i + 3]);
+}
+
 // Causal attention of query row r with head g over the keys of its sequence (K and V in shared
 // memory), with a running maximum and sum over blocks of 8 keys.
 __device__ __forceinline__ void attention(const Ctx& c, const float (&q)[32], float (&o)[32]) {
@@ -550,10 +656,12 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
     c.tg = tc_target(a, cd.idx, cd.layer);
   }
   const int b0 = (fwd || cd.layer < 0) ? -1 : cd.layer;
-  c.b0s = b0 < 0 ? 0 : b0;
+  const int rs = fwd ? kRestartBlock : tfm_restart(a, cd.idx, cd.layer);
+  c.unit0 = rs == kRestartUnit;
+  c.b0s = b0 < 0 ? 0 : b0 + (c.unit0 ? 1 : 0);
   c.nb = a.nL - c.b0s;
   c.cpb = kFfnChunk0 + kFfnPerPair * (a.F / kHp);
-  c.ffn0 = !fwd && tfm_ffn_param(a, cd.idx, cd.layer);
+  c.ffn0 = rs == kRestartFfn;
   c.q0 = c.ffn0 ? kFfnChunk0 : 0;
   c.nbc = c.nb * c.cpb - c.q0;
   c.total = c.nbc + kHeadChunks;
@@ -598,6 +706,14 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
     }
     if (xout && !s_skip[c.sl]) {
       float* dst = xout + (size_t)(s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
+    }
+  } else if (c.unit0) {
+    ffn_unit(a, c, cd, s0, xr, s_part, s_acol);
+    if (xout) {                  // block b0's new output stream
+      float* dst = xout + ((size_t)(b0 + 1) * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
         reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);

@@ -164,10 +164,71 @@ def tfm_stage(a, idx):
     return a.nL
 
 
+RESTART_BLOCK, RESTART_FFN, RESTART_UNIT = 0, 1, 2
+
+
+def restart(a, idx, stage):
+    """Where a recomputation starts in block `stage`: its input, its mid stream (LN2 parameters) or
+    one hidden unit of its feed-forward network (W1, b1, W2, b2: a rank-1 step, then stage + 1)."""
+    if not 0 <= stage < a.nL:
+        return RESTART_BLOCK
+    off = idx - a.o_blk0 - stage * a.blk_size
+    if off < a.r_ln2g:
+        return RESTART_BLOCK
+    return RESTART_FFN if off < a.r_w1 else RESTART_UNIT
+
+
 def ffn_param(a, idx, stage):
     """A parameter of block `stage`'s feed-forward sub-block (LN2, W1, b1, W2, b2)."""
-    return 0 <= stage < a.nL and idx - a.o_blk0 - stage * a.blk_size >= a.r_ln2g
+    return restart(a, idx, stage) != RESTART_BLOCK
 
+
+def ffn_unit(a, cand, s0):
+    """The kernel's rank-1 step for a hidden-unit candidate of block b: block b's new output
+    stream for sequences s0, s0 + 1 ([128, d], rows as in the CTA), from the cached streams. The
+    candidate's own entry enters at its old value (cand[5])."""
+    idx, neww, delta, b, row, old = cand
+    delta = f32(delta)
+    base = a.o_blk0 + b * a.blk_size
+    off = idx - base
+    d, F = a.d, a.F
+    P = a.params
+    xn = a.X[b + 1, s0:s0 + 2].reshape(128, d).copy()
+    if off >= a.r_b2:                                   # b2[i]
+        xn[:, off - a.r_b2] += delta
+        return xn
+    x = a.Xmid[b, s0:s0 + 2].reshape(128, d)
+
+    def part(v):        # the kernel's order: partial sums of four 32-column parts, left to right
+        q = [v[:, 32 * g:32 * g + 32].astype(np.float32).sum(1, dtype=np.float32) for g in range(4)]
+        return ((q[0] + q[1]) + q[2]) + q[3]
+
+    mean = (part(x) / f32(d)).astype(np.float32)
+    e = (x - mean[:, None]).astype(np.float32)
+    var = (part(e * e) / f32(d)).astype(np.float32)
+    rstd = (1.0 / np.sqrt(var.astype(np.float64) + float(a.eps))).astype(np.float32)
+    ln = (e * rstd[:, None] * P[base + a.r_ln2g:base + a.r_ln2g + d] +
+          P[base + a.r_ln2b:base + a.r_ln2b + d]).astype(np.float32)
+    kcol = -1
+    if off < a.r_b1:                                    # W1[j][kcol]
+        j, kcol = divmod(off - a.r_w1, d)
+    elif off < a.r_w2:                                  # b1[j]
+        j = off - a.r_b1
+    else:                                               # W2[i0][j]
+        i0, j = divmod(off - a.r_w2, F)
+    w1 = P[base + a.r_w1 + j * d:base + a.r_w1 + (j + 1) * d].copy()
+    if kcol >= 0:
+        w1[kcol] = old
+    bj = f32(old) if a.r_b1 <= off < a.r_w2 else P[base + a.r_b1 + j]
+    u = (part((ln * w1).astype(np.float32)) + bj).astype(np.float32)
+    fu = act_fn(a.act, u.astype(np.float64), a.g).astype(np.float32)
+    if off >= a.r_w2:
+        xn[:, i0] += delta * fu
+        return xn
+    un = (u + delta * ln[:, kcol]) if kcol >= 0 else (u + delta)
+    da = (act_fn(a.act, un.astype(np.float32).astype(np.float64), a.g).astype(np.float32) - fu)
+    w2 = P[base + a.r_w2 + j:base + a.r_w2 + d * F:F]
+    return (xn + w2[None, :] * da[:, None]).astype(np.float32)
 
 # ---------------------------------------------------------------- the CTA
 
@@ -189,7 +250,7 @@ def adopt(a, slot, cand):
     embedding; X[b+1..] and Xmid[b..] for block b, Xmid[b+1..] for its feed-forward sub-block; none
     for the head stage) and losses from its slot, sequences it skipped (a token embedding whose
     token they lack) left as they are."""
-    idx, neww, delta, layer, row = cand
+    idx, neww, delta, layer, row = cand[:5]
     if delta == 0.0:
         return
     first = 0 if layer < 0 else layer + 1
@@ -212,7 +273,7 @@ class CTA:
         self.tm = np.zeros((128, 512), np.float32)
         self.full = [Bar() for _ in range(kStages)]
         self.empty = [Bar() for _ in range(kStages)]
-        self.cand = cand    # (idx, neww, delta, layer, row) or None for forward
+        self.cand = cand    # (idx, neww, delta, layer, row, old) or None for forward
 
     # shared memory by byte address
     def smf(self, byte_addr):
@@ -441,7 +502,7 @@ class CTA:
         if mode == FORWARD:
             idx, neww, delta, layer, row = 0xFFFFFFFF, 0.0, 1.0, -1, -1
         else:
-            idx, neww, delta, layer, row = self.cand
+            idx, neww, delta, layer, row = self.cand[:5]
         skip = [0, 0]
         if mode != FORWARD and row >= 0:
             skip = [int(all(toks[q, :kT] != row)) for q in range(2)]
@@ -453,10 +514,12 @@ class CTA:
         cstage = -1 if mode == FORWARD else layer
         tg = (kNone, 0, 0) if mode == FORWARD else tc_target(a, idx, layer)
         b0 = -1 if (mode == FORWARD or layer < 0) else layer
-        self.b0s = 0 if b0 < 0 else b0
+        rs = RESTART_BLOCK if mode == FORWARD else restart(a, idx, layer)
+        self.unit0 = rs == RESTART_UNIT
+        self.b0s = 0 if b0 < 0 else b0 + (1 if self.unit0 else 0)
         self.nb = a.nL - self.b0s
         self.cpb = kFfnChunk0 + kFfnPerPair * (a.F // kHp)
-        self.ffn0 = mode != FORWARD and ffn_param(a, idx, layer)
+        self.ffn0 = rs == RESTART_FFN
         self.q0 = kFfnChunk0 if self.ffn0 else 0
         self.nbc = self.nb * self.cpb - self.q0
         self.total = self.nbc + kHeadChunks
@@ -483,6 +546,11 @@ class CTA:
                 for q in range(2):
                     if not skip[q]:
                         xout[0, s0 + q] = xs[q * kT:(q + 1) * kT]
+        elif self.unit0:
+            xs[:] = ffn_unit(a, self.cand, s0)
+            if xout is not None:
+                for q in range(2):
+                    xout[b0 + 1, s0 + q] = xs[q * kT:(q + 1) * kT]
         else:
             xs[:] = (a.Xmid if self.ffn0 else a.X)[b0, s0 + sl, t]
         for g in range(4):

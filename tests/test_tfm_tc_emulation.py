@@ -31,7 +31,8 @@ def setup():
 def _cand(a, idx, neww):
     neww = np.float32(neww)
     row = idx // a.d if idx < a.o_pos else -1
-    return (idx, neww, np.float32(neww - a.params[idx]), E.tfm_stage(a, idx), row)
+    old = np.float32(a.params[idx])
+    return (idx, neww, np.float32(neww - old), E.tfm_stage(a, idx), row, old)
 
 
 def _picks(a):
@@ -42,7 +43,8 @@ def _picks(a):
         "wk": b0 + a.r_wk + 70 * a.d + 3, "wv": b1 + a.r_wv + 127 * a.d + 64,
         "bq": b1 + a.r_bq + 31, "wo": b0 + a.r_wo + 12 * a.d + 99, "ln2.b": b1 + a.r_ln2b + 1,
         "w1": b0 + a.r_w1 + 77 * a.d + 18, "b1": b1 + a.r_b1 + 100,
-        "w2": b1 + a.r_w2 + 40 * a.F + 90, "lnf.g": a.o_lnf_g + 60,
+        "w2": b1 + a.r_w2 + 40 * a.F + 90, "w2.b0": b0 + a.r_w2 + 127 * a.F + 3,
+        "b2": b0 + a.r_b2 + 17, "lnf.g": a.o_lnf_g + 60,
         "w_head": a.o_wh + 20 * a.d + 66, "b_head": a.o_bh + 64,
     }
 
