@@ -237,6 +237,9 @@ __global__ void __launch_bounds__(kDeepThreads) deep_chain_kernel(DeepArgs a) {
 __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
   __shared__ DeepCand s_c[kKmax];
   __shared__ float s_dS[kKmax];
+  __shared__ int s_take[kKmax];
+  __shared__ float s_sum[kKmax];
+  __shared__ float s_buf[(kKmax / 32) * 256];
   __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
   const int k = threadIdx.x, lane = k & 31, warp = k >> 5;
   const int Kb = a.n_explicit > 0 ? a.n_explicit : a.Kb;
@@ -244,9 +247,13 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
   if (k < Kb) {
     const DeepCand c = deep_candidate(a, k);
     s_c[k] = c;
-    const float sum = c.valid && c.delta != 0.0f
-                          ? ordered_sum(a.partial + (size_t)k * a.ntiles, a.ntiles) : 0.0f;
-    const float d = c.valid ? sum : __int_as_float(0x7fc00000);
+    s_take[k] = c.valid && c.delta != 0.0f;
+  }
+  __syncthreads();
+  ordered_row_sums(a.partial, a.ntiles, Kb, s_take, s_sum, s_buf);
+  if (k < Kb) {
+    const DeepCand c = s_c[k];
+    const float d = c.valid ? s_sum[k] : __int_as_float(0x7fc00000);
     s_dS[k] = d;
     if (a.n_explicit > 0) {
       a.ex_out[k] = (double)d;
@@ -294,8 +301,8 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
   if (kbad >= 0 && (kstar < 0 || kbad <= kstar)) kstar = -2;
   DevState* st = a.st;
   const int last = kstar >= 0 ? kstar : Kb - 1;
-  double S = st->S;
   if (a.trace_cap > 0 && kstar != -2) {
+    const double S = st->S;
     for (int q = 0; q <= last; ++q) {
       mca_trace_rec rec;
       rec.tau = a.tau + (unsigned long long)q;
@@ -322,8 +329,10 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
     unsigned int m = s_mforced[w];
     const int hi = last - w * 32;
     if (hi < 31) m &= hi < 0 ? 0u : ((2u << hi) - 1u);
-    st->forced += (unsigned long long)__popc(m);
+    if (m) atomicAdd(&st->forced, (unsigned long long)__popc(m));
   }
+  // (the statistics below are reductions without a returned value, so this thread does not wait
+  // for their reads)
   // FLOPs of the evaluated chains: row update (2 per sample), rank-1 into layer l+1
   // (2 n_out[l+1] per sample), dense layers m = l+2 .. L-1 (2 n_out[m] n_in[m] per sample)
   unsigned long long ncand = 0, flops = 0;
@@ -337,17 +346,17 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
       per += 2ull * (unsigned long long)a.n_out[m] * (unsigned long long)a.n_in[m];
     flops += per * (unsigned long long)a.N;
   }
-  st->candidates += ncand;
-  st->alg_flops += flops;
-  st->batches += 1ull;
+  atomicAdd(&st->candidates, ncand);
+  atomicAdd(&st->alg_flops, flops);
+  atomicAdd(&st->batches, 1ull);
   if (kstar >= 0) {
     const DeepCand& c = s_c[kstar];
     ctl->acc = c;
     ctl->consumed = kstar + 1;
-    st->trials += (unsigned long long)(kstar + 1);
-    st->accepts += 1ull;
-    st->wasted += (unsigned long long)(Kb - kstar - 1);
-    st->S = S + (double)s_dS[kstar];
+    atomicAdd(&st->trials, (unsigned long long)(kstar + 1));
+    atomicAdd(&st->accepts, 1ull);
+    atomicAdd(&st->wasted, (unsigned long long)(Kb - kstar - 1));
+    atomicAdd(&st->S, (double)s_dS[kstar]);
     const int l = c.layer;
     const unsigned long long off = c.idx - a.off[l];
     a.w[l][off] = c.neww;
@@ -360,7 +369,7 @@ __global__ void __launch_bounds__(kKmax) deep_decide_kernel(DeepArgs a) {
     }
   } else {
     ctl->consumed = Kb;
-    st->trials += (unsigned long long)Kb;
+    atomicAdd(&st->trials, (unsigned long long)Kb);
   }
 }
 

@@ -436,6 +436,33 @@ __device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
   lo += err;
 }
 
+// Compensated sums of the rows of x (rows of n floats, n apart): out[k] for k < rows with
+// take[k] != 0 (else 0), each in index order with one two_sum_add per term, the arithmetic of
+// ordered_sum. Every thread of the CTA calls it: warp w takes rows w, w + nwarps, ..., loads 256
+// terms of a row at a time (coalesced) into its 256 floats of buf, and its lane 0 adds them.
+// Ends with a CTA barrier.
+__device__ __forceinline__ void ordered_row_sums(const float* x, int n, int rows, const int* take,
+                                                 float* out, float* buf) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  float* b = buf + warp * 256;
+  for (int k = warp; k < rows; k += nw) {
+    float hi = 0.0f, lo = 0.0f;
+    if (take[k]) {
+      for (int q0 = 0; q0 < n; q0 += 256) {
+        const int m = min(256, n - q0);
+#pragma unroll 8
+        for (int i = lane; i < m; i += 32) b[i] = x[(size_t)k * n + q0 + i];
+        __syncwarp();
+        if (lane == 0)
+          for (int i = 0; i < m; ++i) two_sum_add(hi, lo, b[i]);
+        __syncwarp();
+      }
+    }
+    if (lane == 0) out[k] = take[k] ? hi + lo : 0.0f;
+  }
+  __syncthreads();
+}
+
 // Compensated sum of x[0 .. n) in index order: the same additions, in the same order, as one
 // two_sum_add per term, with the loads of 32 terms in flight at a time.
 __device__ __forceinline__ float ordered_sum(const float* x, int n) {
