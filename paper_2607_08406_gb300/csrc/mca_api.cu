@@ -654,7 +654,7 @@ mca_status tfm_check(const mca_tfm_spec* t, int64_t n_seq) {
 
 struct TfmMem {
   size_t params, tokens, X, ell, partial, st, ctl, trace, ex_idx, ex_new, ex_out, prop, scratch,
-      wimg, Xmid, scrX, scr_ell, total;
+      wimg, Xmid, scrX, scr_ell, ctl2, tau_dev, total;
   int nscr;
 };
 
@@ -704,6 +704,8 @@ TfmMem tfm_plan(const mca_tfm_spec& t, long long B, int trace_cap, bool tc, int 
   M.nscr = tfm_scratch_slots(t, B, K, tc);
   M.scrX = take(sizeof(float) * (size_t)M.nscr * (2 * t.n_layer + 1) * B * t.ctx * t.d_model);
   M.scr_ell = take(sizeof(float) * (size_t)M.nscr * B);
+  M.ctl2 = take(2 * sizeof(mca::DeepCtl));
+  M.tau_dev = take(sizeof(unsigned long long));
   M.total = o;
   return M;
 }
@@ -763,6 +765,77 @@ mca::TfmArgs tfm_args(mca_handle* h) {
   a.tc = h->tc ? 1 : 0;
   a.wimg = h->tfm_img;
   return a;
+}
+
+// Transformer tensor-core batches with the host one batch ahead of the decisions: the kernels of
+// batch i + 1 are enqueued before the host reads batch i's decision. The batch's first trial lives
+// on the device (the decision advances it by the trials it consumed), so the GPU does not wait for
+// the host between batches; a batch enqueued past the end of the run does nothing. A batch's width
+// comes from the acceptance counts up to the batch before the previous one. Every batch has one of
+// two decision buffers, read by the host from pinned memory.
+mca_status run_tfm_pipelined(mca_handle* h, mca::TfmArgs ta, uint64_t n_trials) {
+  if (!h->pipe_host) {
+    CUDA_TRY(h, cudaMallocHost(reinterpret_cast<void**>(&h->pipe_host), sizeof(*h->pipe_host)));
+    for (auto& b : h->ev_p)
+      for (auto& e : b) CUDA_TRY(h, cudaEventCreate(&e));
+  }
+  auto* ph = h->pipe_host;
+  ph->tau = h->tau;
+  CUDA_TRY(h, cudaMemcpyAsync(h->tau_dev, &ph->tau, sizeof(ph->tau), cudaMemcpyHostToDevice,
+                              h->stream));
+  ta.tau_dev = h->tau_dev;
+  ta.tau_end = h->tau + n_trials;
+  ta.nscr = h->nscr;
+  ta.scrX = h->tfm_scrX;
+  ta.scr_ell = h->tfm_scr_ell;
+  auto launch = [&](int i) -> mca_status {
+    const int p = i & 1;
+    const int Kw = h->opt.fixed_K ? h->opt.K
+                                  : mca::batch_width_cost(h->rate_acc, h->rate_trials,
+                                                          mca::kBatchCostTfm, h->opt.K);
+    ta.Kb = (int)std::min<uint64_t>(n_trials, (uint64_t)Kw);
+    ta.ctl = h->ctl2 + p;
+    CUDA_TRY(h, cudaEventRecord(h->ev_p[p][0], h->stream));
+    CUDA_TRY(h, mca::launch_tfm_eval(ta, h->stream));
+    CUDA_TRY(h, cudaEventRecord(h->ev_p[p][1], h->stream));
+    CUDA_TRY(h, mca::launch_tfm_decide(ta, h->stream));
+    CUDA_TRY(h, mca::launch_tfm_commit(ta, h->stream));
+    CUDA_TRY(h, mca::launch_tfm_tc_adopt(ta, h->stream));
+    CUDA_TRY(h, cudaMemcpyAsync(&ph->ctl[p], h->ctl2 + p, sizeof(mca::DeepCtl),
+                                cudaMemcpyDeviceToHost, h->stream));
+    CUDA_TRY(h, cudaEventRecord(h->ev_p[p][2], h->stream));
+    h->launches += 4;
+    return MCA_OK;
+  };
+  uint64_t done = 0;
+  mca_status rc = launch(0);
+  if (rc != MCA_OK) return rc;
+  for (int i = 0;; ++i) {
+    NvtxRange nv_batch("mca batch (transformer, one ahead)");
+    rc = launch(i + 1);
+    if (rc != MCA_OK) return rc;
+    const int p = i & 1;
+    CUDA_TRY(h, cudaEventSynchronize(h->ev_p[p][2]));
+    float ms_eval = 0.0f, ms_rest = 0.0f;
+    CUDA_TRY(h, cudaEventElapsedTime(&ms_eval, h->ev_p[p][0], h->ev_p[p][1]));
+    CUDA_TRY(h, cudaEventElapsedTime(&ms_rest, h->ev_p[p][1], h->ev_p[p][2]));
+    h->eval_ns += (uint64_t)(ms_eval * 1e6f);
+    h->rest_ns += (uint64_t)(ms_rest * 1e6f);
+    const mca::DeepCtl ctl = ph->ctl[p];
+    if (ctl.kstar == -2 || ctl.consumed <= 0) {
+      cudaStreamSynchronize(h->stream);
+      h->broken = true;
+      return fail(h, MCA_ERR_NUMERIC, "non-finite loss change");
+    }
+    done += (uint64_t)ctl.consumed;
+    h->rate_acc = h->rate_acc * mca::kRateDecay + (ctl.kstar >= 0 ? 1.0f : 0.0f);
+    h->rate_trials = h->rate_trials * mca::kRateDecay + (float)ctl.consumed;
+    if (done >= n_trials) break;
+  }
+  // the batch enqueued last starts at the run's end and does nothing; let it finish
+  CUDA_TRY(h, cudaStreamSynchronize(h->stream));
+  h->tau += done;
+  return MCA_OK;
 }
 
 }  // namespace
@@ -1026,6 +1099,11 @@ mca_status mca_run(mca_handle* h, uint64_t n_trials, uint64_t seed, mca_run_stat
     a.seed = seed;
     ta.seed = seed;
     const uint64_t R = (uint64_t)h->opt.resync_period;
+    if (h->tfm && h->tc && R == 0 && remaining > 0) {
+      mca_status rc = run_tfm_pipelined(h, ta, remaining);
+      if (rc != MCA_OK) return rc;
+      remaining = 0;
+    }
     while (remaining > 0) {
       NvtxRange nv_batch(h->tfm ? "mca batch (transformer)" : "mca batch (deep)");
       const int Kw = h->opt.fixed_K ? h->opt.K
@@ -1522,6 +1600,8 @@ mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* do
   h->prop = reinterpret_cast<mca_trace_rec*>(base + M.prop);
   h->tfm_img = h->tc ? reinterpret_cast<float*>(base + M.wimg) : nullptr;
   h->tfm_Xmid = h->tc ? reinterpret_cast<float*>(base + M.Xmid) : nullptr;
+  h->ctl2 = reinterpret_cast<mca::DeepCtl*>(base + M.ctl2);
+  h->tau_dev = reinterpret_cast<unsigned long long*>(base + M.tau_dev);
   h->nscr = M.nscr;
   h->tfm_scrX = reinterpret_cast<float*>(base + M.scrX);
   h->tfm_scr_ell = reinterpret_cast<float*>(base + M.scr_ell);
@@ -1670,6 +1750,10 @@ void mca_destroy(mca_handle* h) {
     if (e) cudaEventDestroy(e);
   for (auto& e : h->ev_c)
     if (e) cudaEventDestroy(e);
+  for (auto& b : h->ev_p)
+    for (auto& e : b)
+      if (e) cudaEventDestroy(e);
+  if (h->pipe_host) cudaFreeHost(h->pipe_host);
   if (h->ws_owned && h->ws) cudaFree(h->ws);
   if (h->ftau) cudaFree(h->ftau);
   if (h->facc) cudaFree(h->facc);

@@ -269,6 +269,11 @@ struct TfmArgs {
   float* scrX;
   float* scr_ell;
   int nscr;
+  // batches run ahead of the host (tc = 1, trial loop): the batch's first trial is read from
+  // tau_dev, which the decision advances by the trials it consumed; trials at or past tau_end do not
+  // exist (a batch that starts there does nothing). nullptr: the batch starts at tau.
+  unsigned long long* tau_dev;
+  unsigned long long tau_end;
 };
 
 size_t tfm_smem_bytes(int T, int d, int dh, int V);
@@ -411,6 +416,15 @@ struct mca_handle {
   unsigned long long tau = 0;
   unsigned long long launches = 0, resyncs = 0;
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};   // per-batch kernel timing (deep, Transformer)
+  // Transformer tensor-core path, batches run ahead of the host: two decision buffers (device),
+  // the batch's first trial (device), their pinned host mirror, and per-buffer events
+  mca::DeepCtl* ctl2 = nullptr;
+  unsigned long long* tau_dev = nullptr;
+  struct PipeHost {
+    mca::DeepCtl ctl[2];
+    unsigned long long tau;
+  }* pipe_host = nullptr;
+  cudaEvent_t ev_p[2][3] = {{nullptr, nullptr, nullptr}, {nullptr, nullptr, nullptr}};
   unsigned long long eval_ns = 0, rest_ns = 0;
   bool broken = false;                   // a sticky CUDA error or device timeout was seen
   float rate_acc = 0.0f, rate_trials = 0.0f;   // deep path: acceptance counts (batch width)

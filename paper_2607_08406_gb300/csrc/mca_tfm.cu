@@ -432,7 +432,8 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
   __shared__ float s_buf[(kKmax / 32) * 256];
   __shared__ unsigned int s_macc[kKmax / 32], s_mbad[kKmax / 32], s_mforced[kKmax / 32];
   const int k = threadIdx.x, lane = k & 31, warp = k >> 5;
-  const int Kb = a.n_explicit > 0 ? a.n_explicit : a.Kb;
+  const unsigned long long tau = tfm_batch_tau(a);
+  const int Kb = tfm_batch_width(a, tau);
   bool acc = false, bad = false, forced = false;
   if (k < Kb) {
     const DeepCand c = tfm_candidate(a, k);
@@ -448,7 +449,7 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
     if (a.n_explicit > 0) {
       a.ex_out[k] = (double)d;
     } else if (c.valid) {
-      const unsigned long long tk = a.tau + (unsigned long long)k;
+      const unsigned long long tk = tau + (unsigned long long)k;
       bool facc = false;
       if (a.nforce > 0) {
         int lo2 = 0, hi2 = a.nforce;
@@ -495,7 +496,7 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
     const double S = st->S;
     for (int q = 0; q <= last; ++q) {
       mca_trace_rec rec;
-      rec.tau = a.tau + (unsigned long long)q;
+      rec.tau = tau + (unsigned long long)q;
       rec.idx = s_c[q].idx;
       rec.accept = q == kstar ? 1 : 0;
       rec.old_w = s_c[q].oldw;
@@ -512,6 +513,10 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
   ctl->kstar = kstar;
   if (kstar == -2) {
     atomicCAS(&st->err, 0, (int)MCA_ERR_NUMERIC);
+    ctl->consumed = 0;
+    return;
+  }
+  if (Kb == 0) {                 // a batch past the end of a run whose batches run ahead
     ctl->consumed = 0;
     return;
   }
@@ -547,6 +552,7 @@ __global__ void __launch_bounds__(kKmax) tfm_decide_kernel(TfmArgs a) {
     ctl->consumed = Kb;
     atomicAdd(&st->trials, (unsigned long long)Kb);
   }
+  if (a.tau_dev) *a.tau_dev = tau + (unsigned long long)(kstar >= 0 ? kstar + 1 : Kb);
 }
 
 template <int MODE>

@@ -34,6 +34,18 @@ __device__ __forceinline__ bool tfm_ffn_param(const TfmArgs& a, unsigned long lo
   return tfm_restart(a, idx, stage) != kRestartBlock;
 }
 
+// The batch's first trial, and its width (fewer at the end of a run whose batches run ahead of the
+// host).
+__device__ __forceinline__ unsigned long long tfm_batch_tau(const TfmArgs& a) {
+  return a.tau_dev ? *reinterpret_cast<volatile const unsigned long long*>(a.tau_dev) : a.tau;
+}
+
+__device__ __forceinline__ int tfm_batch_width(const TfmArgs& a, unsigned long long tau) {
+  if (a.n_explicit > 0) return a.n_explicit;
+  if (!a.tau_dev) return a.Kb;
+  return tau >= a.tau_end ? 0 : (int)min((unsigned long long)a.Kb, a.tau_end - tau);
+}
+
 __device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {
   unsigned int idx;
   uint32_t r1 = 0u;
@@ -43,7 +55,7 @@ __device__ __forceinline__ DeepCand tfm_candidate(const TfmArgs& a, int k) {
     idx = a.ex_idx[k];
     exv = a.ex_new[k];
   } else {
-    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
+    const uint4 w = trial_words(a.seed, tfm_batch_tau(a) + (unsigned long long)k);
     idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
     r1 = w.y;
   }

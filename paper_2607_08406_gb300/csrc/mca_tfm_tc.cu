@@ -125,7 +125,7 @@ __device__ __forceinline__ int candidate_stage(const TfmArgs& a, int k) {
   if (a.n_explicit > 0) {
     idx = a.ex_idx[k];
   } else {
-    const uint4 w = trial_words(a.seed, a.tau + (unsigned long long)k);
+    const uint4 w = trial_words(a.seed, tfm_batch_tau(a) + (unsigned long long)k);
     idx = (unsigned int)(((unsigned long long)w.x * a.P) >> 32);
   }
   const int st = tfm_stage(a, idx);
@@ -617,6 +617,10 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
   __syncthreads();
   const DeepCand cd = s_c;
   float* part = a.partial + (size_t)k * a.B + s0;
+  if (MODE == kTfmEval && k >= tfm_batch_width(a, tfm_batch_tau(a))) {   // past the run's end
+    if (tid < 2) part[tid] = 0.0f;
+    return;
+  }
   // where the recomputed residual streams and sequence losses go: the handle's (commit, forward)
   // or, in an evaluation, the candidate's scratch slot when it has one
   const size_t seq_floats = (size_t)kT * kD;
