@@ -34,7 +34,7 @@ METRIC = "MC mutation trials/sec (full-batch loss evals); fraction of HBM/TC roo
 # from one ncu capture (one pass, one launch: the first timed step, trials 200k..240k) of
 # `python bench.py --steps 20 --warmup 5 --no-e2e --no-cpu`, summarised in profiles/. It is only
 # valid for the kernel source and the workload it was measured on; anything else reports null.
-LOOP_TRAFFIC = {"source_sha1": "d226e40a5b6369a5b1cfa03226a2bb7319f8dc8f",
+LOOP_TRAFFIC = {"source_sha1": "2502508233974700a08bab261aa72e3018dd27bb",
                 "workload": "mlp784-16384-10_ce_n60000", "bytes_per_trial": 374000.0}
 LOOP_SOURCES = ("paper_2607_08406_gb300/csrc/mca_mlp2.cu", "paper_2607_08406_gb300/csrc/mca_device.cuh")
 
