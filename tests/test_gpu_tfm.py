@@ -120,3 +120,27 @@ def test_tfm_resync_keeps_loss(gpu_lib):
     L = gpu_lib.mca_loss(h)
     gpu_lib.mca_resync(h)
     assert gpu_lib.mca_loss(h) == pytest.approx(L, rel=1e-5)
+
+
+def test_tfm_one_ahead_batches_match_round_trip_batches(gpu_lib, monkeypatch):
+    """The tensor-core path enqueues each batch before the host reads the previous decision (the
+    trial counter lives on the device) unless the handle has a resync period; with a period longer
+    than the run (the round-trip loop, no resync) the trace, parameters and loss are bit-identical,
+    over runs of several lengths (one trial, a few batches, and a longer one) continuing the chain."""
+    monkeypatch.delenv("MCA_TFM_TENSOR_CORES", raising=False)
+    wl = W.char_transformer()
+    out = []
+    for R in (0, 10 ** 9):
+        h = gpu_lib.create_from_tfm_workload(wl, trace_cap=400, resync_period=R)
+        n = 0
+        for m in (1, 7, 150):
+            st = gpu_lib.mca_run(h, m, 11)
+            n += m
+            assert st["trials"] == n and st["tau"] == n and st["tensor_cores"] == 1
+        out.append((gpu_lib.mca_get_trace(h, n), gpu_lib.mca_get_params(h, wl.n_params),
+                    gpu_lib.mca_loss(h)))
+        assert st["resyncs"] == 0
+        h.close()
+    assert np.array_equal(out[0][0], out[1][0])
+    assert np.array_equal(out[0][1], out[1][1])
+    assert out[0][2] == out[1][2]
