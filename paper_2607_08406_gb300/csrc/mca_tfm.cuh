@@ -37,7 +37,7 @@ __device__ __forceinline__ bool tfm_ffn_param(const TfmArgs& a, unsigned long lo
 // The batch's first trial, and its width (fewer at the end of a run whose batches run ahead of the
 // host).
 __device__ __forceinline__ unsigned long long tfm_batch_tau(const TfmArgs& a) {
-  return a.tau_dev ? *reinterpret_cast<volatile const unsigned long long*>(a.tau_dev) : a.tau;
+  return a.tau_dev ? __ldcg(a.tau_dev) : a.tau;
 }
 
 __device__ __forceinline__ int tfm_batch_width(const TfmArgs& a, unsigned long long tau) {
