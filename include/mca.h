@@ -240,7 +240,14 @@ mca_status mca_tfm_workspace_size(const mca_tfm_spec* spec, int64_t n_seq, const
  * for other shapes, or when the process environment has MCA_TFM_TENSOR_CORES=0, on the SIMT fp32
  * kernels. The variable is read by this call and by mca_tfm_workspace_size (the tensor-core kernels'
  * weight images are part of the workspace), so it must not change between the two. mca_run_stats
- * .tensor_cores reports the choice. */
+ * .tensor_cores reports the choice. On the tensor-core kernels a candidate's recomputation starts at
+ * the first sub-block its parameter feeds (a block's input, its cached stream after the attention
+ * sub-block for LN2, a rank-1 step for one hidden unit of the feed-forward network), the evaluation
+ * of candidates k < min(K, 16) keeps what it recomputed in per-candidate scratch slots of the
+ * workspace (at most 8 GiB) from which an accepted candidate is adopted, and mca_run enqueues each
+ * batch before it reads the previous decision unless resync_period > 0. MCA_ADOPT=0 in the
+ * environment (read like MCA_TFM_TENSOR_CORES; it applies to deep MLPs on the tensor cores too)
+ * leaves out the slots: every accepted candidate is then recomputed by the commit kernels. */
 mca_status mca_create_transformer(const mca_tfm_spec* spec, const mca_domain* dom,
                                   const int32_t* tokens, int64_t n_seq, const float* init_params,
                                   const mca_options* opt, mca_handle** out);
