@@ -222,7 +222,11 @@ mca_status mca_workspace_size(const mca_layer* layers, int32_t n_layers, int32_t
  *  the last layer's n_out <= 16 (the number of classes), labels in range.
  *  Computes every cached field with a full forward pass (the trial counter tau starts at 0).
  *  On success *out owns a handle to release with mca_destroy. Errors: INVALID (spec/sizes),
- *  NUMERIC (non-finite x or init, or a non-finite initial loss), OOM, CUDA, UNSUPPORTED. */
+ *  NUMERIC (non-finite x or init, or a non-finite initial loss), OOM, CUDA, UNSUPPORTED.
+ *  Deep nets whose inner layers are all 256 x 256 run their dense chain on the tensor cores; the
+ *  evaluation of candidates k < min(K, 16) then keeps every field it computes in per-candidate
+ *  scratch slots of the workspace, from which an accepted candidate is adopted (MCA_ADOPT=0 in the
+ *  environment, read by this call and mca_workspace_size, leaves the slots out). */
 mca_status mca_create(const mca_layer* layers, int32_t n_layers, int32_t loss,
                       const mca_domain* dom, const mca_dataset* data, const float* init_params,
                       const mca_options* opt, mca_handle** out);
