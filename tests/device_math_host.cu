@@ -8,6 +8,7 @@
 //   idx2 P P1 SEED TAU R0 M               -> two-layer trial index
 //   idxd SEED TAU R0 M L off0 .. offL     -> deep trial index (L layers, L + 1 offsets)
 //   chan SEED TAU L n0 .. nL fin0 .. finL-1 -> channel nodes c_0 .. c_L, then the L He values
+//   width ACC TRIALS R K                  -> the host-driven batch width of the cost model
 #include <cstdio>
 #include <cstring>
 #include <iostream>
@@ -73,6 +74,11 @@ int main() {
         std::printf("%.9g ", (double)mca::channel_he_value(mca::channel_word(seed, tau, L + 1 + m),
                                                            fin[m]));
       std::printf("\n");
+    } else if (cmd == "width") {
+      float acc, trials, r;
+      int K;
+      in >> acc >> trials >> r >> K;
+      std::printf("%d\n", mca::batch_width_cost(acc, trials, r, K));
     } else if (!cmd.empty()) {
       std::printf("?\n");
     }

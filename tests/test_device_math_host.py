@@ -115,3 +115,23 @@ def test_channel_draws(harness):
             nodes = [c[2] for c in ch] + [ch[-1][1]]
             assert [int(v) for v in vals[:L + 1]] == nodes
             assert [np.float32(float(v)) for v in vals[L + 1:]] == [np.float32(c[4]) for c in ch]
+
+
+def test_batch_width_cost_model(harness):
+    """The width of the host-driven batches (deep nets, the Transformer) is the K in 1 .. Kmax that
+    maximises the expected trials a batch consumes, (1 - (1-p)^K) / p with p = (A + 1/2) / (T + 1),
+    per unit of its cost r + K: checked against a brute-force argmax in double precision, and
+    against its limits (a certain accept takes one candidate; a rarely accepting chain with a costly
+    batch takes many, capped at Kmax)."""
+    rng = np.random.default_rng(5)
+    cases = [(float(a), float(a + t), float(r), int(k))
+             for a, t, r, k in zip(rng.uniform(0, 30, 200), rng.uniform(0, 200, 200),
+                                   rng.choice([0.0, 0.38, 0.5, 1.9, 8.0], 200),
+                                   rng.integers(1, 129, 200))]
+    cases += [(1000.0, 1000.0, 1.9, 64), (0.0, 10000.0, 50.0, 64), (0.0, 10000.0, 50.0, 7)]
+    got = [int(v) for v in harness([f"width {a!r} {t!r} {r!r} {k}" for a, t, r, k in cases])]
+    for (a, t, r, k), w in zip(cases, got):
+        p = (np.float32(a) + 0.5) / (np.float32(t) + 1.0)
+        v = [(1.0 - (1.0 - p) ** K) / (r + K) for K in range(1, k + 1)]
+        assert w == int(np.argmax(v)) + 1, (a, t, r, k, w)
+    assert got[-3] == 1 and got[-2] > 40 and got[-1] == 7
