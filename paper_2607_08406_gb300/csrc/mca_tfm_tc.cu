@@ -749,22 +749,22 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
       float q[32];
       {
         float v[32];
-  #pragma unroll
+#pragma unroll
         for (int p = 0; p < 2; ++p) {
           ld32(c, (p ? kColV : kColK) + 32u * (uint32_t)c.g, v);
           const unsigned long long bb = base + (p ? a.r_bv : a.r_bk) + 32 * c.g;
-  #pragma unroll
+#pragma unroll
           for (int i = 0; i < 32; ++i) v[i] += prm(a, bb + i, c.midx, c.mval);
           if (here && c.tg.mat == (p ? kTcV : kTcK)) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
           float* dst = (p ? c.vs : c.ks) + (size_t)c.r * kD + 32 * c.g;
-  #pragma unroll
+#pragma unroll
           for (int i = 0; i < 8; ++i)
             *reinterpret_cast<float4*>(dst + 4 * (i ^ (c.r & 7))) =
                 make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
         ld32(c, kColQ + 32u * (uint32_t)c.g, q);
         const unsigned long long bq = base + a.r_bq + 32 * c.g;
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 32; ++i) q[i] += prm(a, bq + i, c.midx, c.mval);
         if (here && c.tg.mat == kTcQ) add_at(q, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
       }
@@ -774,7 +774,7 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
         attention(c, q, o);
         __syncthreads();           // every row done with K and V: their memory takes the next A
         if (here && c.tg.mat == kTcO) {
-  #pragma unroll
+#pragma unroll
           for (int i = 0; i < 32; ++i)
             if (32 * c.g + i == c.tg.col) s_acol[c.r] = o[i];
         }
@@ -794,12 +794,12 @@ __global__ void __launch_bounds__(kThreads, 1) tfm_tc_kernel(TfmArgs a) {
         ld32(c, kColU + 32u * (uint32_t)c.g, v);
         if (here && c.tg.mat == kTcO) add_at(v, c.tg.row - 32 * c.g, c.dlt * s_acol[c.r]);
         const unsigned long long bo = base + a.r_bo + 32 * c.g;
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 32; ++i) xr[i] += v[i] + prm(a, bo + i, c.midx, c.mval);
       }
       if (xmout && !s_skip[c.sl]) {    // the mid stream: block b after its attention sub-block
         float* dst = xmout + ((size_t)b * a.B + s0 + c.sl) * seq_floats + (size_t)c.t * kD + 32 * c.g;
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 8; ++i)
           reinterpret_cast<float4*>(dst)[i] = *reinterpret_cast<const float4*>(xr + 4 * i);
       }
