@@ -147,3 +147,22 @@ def test_binding_maps_beta_to_temperature():
     for bad in (0.0, -3.0, float("nan")):
         with pytest.raises(ValueError):
             mca._domain(W.Domain(beta=bad))
+
+
+def test_transformer_scratch_slots_in_the_workspace(lib, monkeypatch):
+    """Workspace of the tensor-core Transformer (sized on the host, no GPU): each of the
+    min(K, 16) scratch slots holds the streams a candidate's evaluation recomputes (the 2 nL + 1
+    block input and mid streams of every sequence) and its sequence losses; MCA_ADOPT=0 leaves the
+    slots out."""
+    wl = W.char_transformer()
+    sp = wl.spec
+    B = 256
+    stream = B * sp.ctx * sp.d_model * 4
+    slot = (2 * sp.n_layer + 1) * stream + B * 4          # both parts are multiples of 256 bytes
+    monkeypatch.delenv("MCA_TFM_TENSOR_CORES", raising=False)
+    monkeypatch.setenv("MCA_ADOPT", "0")
+    base = mca.mca_tfm_workspace_size(sp, B, 16)
+    assert mca.mca_tfm_workspace_size(sp, B, 1) == base
+    monkeypatch.delenv("MCA_ADOPT")
+    for K, nscr in ((1, 1), (5, 5), (16, 16), (64, 16)):
+        assert mca.mca_tfm_workspace_size(sp, B, K) == base + nscr * slot, K
