@@ -166,3 +166,21 @@ def test_transformer_scratch_slots_in_the_workspace(lib, monkeypatch):
     monkeypatch.delenv("MCA_ADOPT")
     for K, nscr in ((1, 1), (5, 5), (16, 16), (64, 16)):
         assert mca.mca_tfm_workspace_size(sp, B, K) == base + nscr * slot, K
+
+
+def test_deep_scratch_slots_in_the_workspace(monkeypatch):
+    """Workspace of a deep net on the tensor-core chain (sized on the host, no GPU): each of the
+    min(K, 16) scratch slots holds every layer's fields and the per-sample losses (the arrays an
+    accepted candidate's adoption exchanges), plus one row of the slots' pointer table; MCA_ADOPT=0
+    leaves them out."""
+    wl = W.mlp_deep(N=1100, width=256, depth=5, n_trials=10, K=16)
+    Np = (wl.N + 127) // 128 * 128
+    L = len(wl.layers)
+    slot = sum(ly.n_out for ly in wl.layers) * Np * 4 + Np * 4   # each array a multiple of 256 B
+    monkeypatch.setenv("MCA_ADOPT", "0")
+    base = mca.mca_workspace_size(wl.layers, wl.loss, wl.X, wl.y, 16)
+    monkeypatch.delenv("MCA_ADOPT")
+    for K, nscr in ((1, 1), (16, 16), (64, 16)):
+        table = -(-nscr * (L + 1) * 8 // 256) * 256
+        assert mca.mca_workspace_size(wl.layers, wl.loss, wl.X, wl.y, K) == \
+            base + nscr * slot + table, K
