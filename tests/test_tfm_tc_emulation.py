@@ -155,3 +155,47 @@ def test_emulated_kernel_at_the_largest_shape_it_takes():
     for p in range(a.B // 2):
         E.CTA(a, E.COMMIT, c, p).run()
     np.testing.assert_array_equal(a.ell, (ell0 + dS).astype(np.float32))
+
+
+def test_emulated_kernel_with_an_odd_number_of_hidden_pairs():
+    """d_ff 384 (three pairs of 64-wide hidden chunks per W1 product) in one Gaussian block: the
+    forward losses, and candidates at the first and last hidden unit of every pair (W1 rows, b1,
+    W2 columns: the rank-1 steps), LN2 (the mid-stream restart) and b2, against the oracle; an
+    evaluation with a scratch slot plus adoption equals the commit."""
+    spec = W.TfmSpec(d_ff=384, n_layer=1, act="gaussian", act_param=0.4)
+    wl = W.char_transformer(batch=2, spec=spec, text_len=20000)
+    a = E.Args(spec, wl.init, wl.tokens)
+    a.split()
+    for pair in range(a.B // 2):
+        E.CTA(a, E.FORWARD, None, pair).run()
+    ell = OT.tfm_seq_losses(spec, a.params.astype(np.float64), a.tokens)
+    assert np.all(np.abs(a.ell - ell) <= 2e-6 * ell)
+    d, F = a.d, a.F
+    b0 = a.o_blk0
+    picks = {"ln2.g": b0 + a.r_ln2g + 17, "b2": b0 + a.r_b2 + 100}
+    for u in (0, 127, 128, 255, 256, 383):
+        picks[f"w1[{u}]"] = b0 + a.r_w1 + u * d + (u * 7) % d
+        picks[f"b1[{u}]"] = b0 + a.r_b1 + u
+        picks[f"w2[:,{u}]"] = b0 + a.r_w2 + ((u * 5) % d) * F + u
+    for name, idx in picks.items():
+        c = _cand(a, idx, 0.43)
+        q = a.params.copy()
+        q[idx] = c[1]
+        want = OT.tfm_seq_losses(spec, q.astype(np.float64), a.tokens) - ell
+        got = np.concatenate([E.CTA(a, E.EVAL, c, p).run() for p in range(a.B // 2)])
+        assert np.all(np.abs(got - want) <= 2e-6 * ell), (name, got, want)
+    for name in ("w1[255]", "ln2.g"):
+        b = copy.deepcopy(a)
+        c = _cand(b, picks[name], -0.71)
+        slot = E.Slot(b)
+        for p in range(b.B // 2):
+            E.CTA(b, E.EVAL, c, p, slot).run()
+        r = copy.deepcopy(b)
+        b.params[c[0]] = c[1]
+        r.params[c[0]] = c[1]
+        for p in range(b.B // 2):
+            E.CTA(b, E.COMMIT, c, p).run()
+        E.adopt(r, slot, c)
+        np.testing.assert_array_equal(r.X, b.X, err_msg=name)
+        np.testing.assert_array_equal(r.Xmid, b.Xmid, err_msg=name)
+        np.testing.assert_array_equal(r.ell, b.ell, err_msg=name)
